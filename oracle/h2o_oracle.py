@@ -1,0 +1,204 @@
+"""Float64 CPU oracle for the H2O sparse-attention chunk step and cache update.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import or call
+this module: only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline
+leg of ``bench.py`` use it.  It shares no code with the CUDA library.
+
+It is a plain, slow, literal restatement of what the paper defines:
+
+* ``sdpa_chunk``: scaled dot product attention of §3.1, Eq. 2, with the
+  position-based causal mask of §3.1 / §3.3.1 (a key with token position t(j)
+  is hidden from query row i iff P + i < t(j)), plus the summed attention
+  weights sum_i m_ij that §3.3.1 and §A.6 ask the kernel to return, shape
+  (B, H_q, N_k).  Empty cache slots (position -1) are hidden as well.
+* ``update``: the H2O policy of §3.1.1: the score of Eq. 3 is the running sum
+  of attention weights a slot received since its token entered the cache; the
+  S slots with the smallest score are overwritten by the chunk's keys and
+  values (the scatter of §3.2 / §A.1.1), with the readings listed below.
+* ``run_sequence``: prefill then chunks (§3.1 last paragraph, §A.4.1).
+
+Readings where the paper is silent (each is also listed in the design notes):
+
+* Order within a chunk step: the chunk attends to the M cache slots plus,
+  causally, to itself (N_k = M + S); its attention weights are added to the
+  scores; then S slots are evicted and overwritten.
+* GQA: query head hq belongs to KV head hq // q_g; the score of a KV-head slot
+  is the sum of its q_g query heads' summed weights.
+* Recent window W: a slot whose token position is >= P + S - W is not a
+  candidate for eviction.  Empty slots rank before every occupied slot.
+* Total order for eviction: (empty first, score ascending, slot ascending);
+  the c-th smallest evicted slot index receives the chunk's c-th token.
+* The new slot's score is the summed weight its own column received in this
+  chunk (Eq. 3 sums over s >= t(j), and the chunk's queries are s >= t(j)).
+* Scores accumulate in one of two precisions: ``"fp64"`` (the oracle's own
+  trajectory) or ``"fp32"``, which adds, in float32, the q_g query heads in
+  ascending order (t = inc_0; t = t + inc_g) and then ``scores + t``; that is
+  the order any implementation must follow to be compared bit for bit.
+
+Parity: every function here is pinned by the not-gpu tests against dense
+causal attention, closed forms, the summed-weights identity of §A.6.2,
+invariants of §3.1-§3.3 and brute-force enumeration.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+__all__ = ["sdpa_chunk", "update", "run_sequence", "SequenceState", "lse_merge",
+           "chunk_bounds"]
+
+
+def _token_positions(slot_pos_bh: np.ndarray, pos0: int, S: int) -> np.ndarray:
+    """Token position of every key column: cache slots first, then the chunk's S tokens."""
+    return np.concatenate([slot_pos_bh.astype(np.int64), pos0 + np.arange(S, dtype=np.int64)])
+
+
+def sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale: float | None = None):
+    """One chunk of H2O sparse SDPA (§3.1 Eq. 2 + summed weights of §3.3.1 / §A.6).
+
+    Args:
+      q: (B, H_q, S, d) queries of tokens pos0 .. pos0+S-1.
+      k_cache, v_cache: (B, H_kv, M, d) cache buffers.
+      k_new, v_new: (B, H_kv, S, d) keys/values of the chunk's tokens.
+      slot_pos: (B, H_kv, M) int token position per slot, -1 = empty.
+      pos0: P, the number of tokens processed before this chunk.
+      scale: softmax scale, default d**-0.5 (Eq. 2).
+
+    Returns (out (B,H_q,S,d), score_inc (B,H_q,M+S), lse (B,H_q,S)), float64.
+    Key columns are ordered cache slots 0..M-1, then chunk tokens 0..S-1.
+    """
+    q = np.asarray(q, np.float64)
+    B, Hq, S, d = q.shape
+    Hkv, M = slot_pos.shape[1], slot_pos.shape[2]
+    assert Hq % Hkv == 0
+    qg = Hq // Hkv
+    if scale is None:
+        scale = 1.0 / math.sqrt(d)
+    out = np.zeros((B, Hq, S, d))
+    score_inc = np.zeros((B, Hq, M + S))
+    lse = np.zeros((B, Hq, S))
+    for b in range(B):
+        for hq in range(Hq):
+            h = hq // qg
+            keys = np.concatenate([np.asarray(k_cache[b, h], np.float64),
+                                   np.asarray(k_new[b, h], np.float64)])
+            vals = np.concatenate([np.asarray(v_cache[b, h], np.float64),
+                                   np.asarray(v_new[b, h], np.float64)])
+            t = _token_positions(slot_pos[b, h], pos0, S)
+            # mask: hidden iff the slot is empty or P + i < t(j)  (§3.3.1)
+            qpos = pos0 + np.arange(S)[:, None]
+            visible = (t[None, :] >= 0) & (t[None, :] <= qpos)
+            a = scale * (q[b, hq] @ keys.T)
+            a = np.where(visible, a, -np.inf)
+            amax = a.max(axis=1, keepdims=True)
+            lam = amax + np.log(np.exp(a - amax).sum(axis=1, keepdims=True))
+            m = np.where(visible, np.exp(a - lam), 0.0)
+            out[b, hq] = m @ vals
+            score_inc[b, hq] = m.sum(axis=0)
+            lse[b, hq] = lam[:, 0]
+    return out, score_inc, lse
+
+
+def lse_merge(l1, l2):
+    """Combine log-sum-exp values of two disjoint column sets (§A.6.1)."""
+    l1 = np.asarray(l1, np.float64)
+    l2 = np.asarray(l2, np.float64)
+    return np.maximum(l1, l2) + np.log1p(np.exp(-np.abs(l1 - l2)))
+
+
+def update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0: int,
+           recent_window: int, precision: str = "fp32"):
+    """H2O score accumulation, eviction and K/V write (§3.1.1 Eq. 3, §3.2, §A.1.1).
+
+    Inputs are not modified.  Returns a dict with new ``scores`` (float32 or
+    float64), ``slot_pos``, ``k_cache``, ``v_cache`` and ``evict_idx``
+    (B, H_kv, S) int32: slot receiving token pos0 + c, ascending in c.
+    """
+    B, Hkv, M = slot_pos.shape
+    Bq, Hq, N = score_inc.shape
+    S = N - M
+    assert Bq == B and Hq % Hkv == 0 and 1 <= S <= M
+    qg = Hq // Hkv
+    W = recent_window
+    if W < 0 or W > M:
+        raise ValueError("recent_window must lie in [0, M]")
+    ft = np.float32 if precision == "fp32" else np.float64
+    inc = np.asarray(score_inc, ft)
+    out_scores = np.array(scores, dtype=ft, copy=True)
+    out_pos = np.array(slot_pos, dtype=np.int32, copy=True)
+    out_k = np.array(k_cache, copy=True)
+    out_v = np.array(v_cache, copy=True)
+    evict = np.zeros((B, Hkv, S), np.int32)
+    for b in range(B):
+        for h in range(Hkv):
+            # group sum over the q_g query heads of KV head h, ascending order
+            t = inc[b, h * qg].copy()
+            for g in range(1, qg):
+                t = t + inc[b, h * qg + g]
+            acc = out_scores[b, h] + t[:M]          # Eq. 3: accumulate this chunk
+            new = t[M:]                              # scores of the chunk's own tokens
+            pos = out_pos[b, h]
+            cand = np.nonzero(pos < pos0 + S - W)[0]  # recent window is protected
+            if cand.size < S:
+                raise ValueError("fewer eviction candidates than chunk tokens")
+            occupied = pos[cand] >= 0
+            rank0 = occupied.astype(np.int64)               # 0 = empty: ranks first
+            rank1 = np.where(occupied, acc[cand], 0)        # empties tie, broken by slot
+            order = np.lexsort((cand, rank1, rank0))
+            chosen = np.sort(cand[order[:S]])
+            evict[b, h] = chosen
+            out_scores[b, h] = acc
+            for c, e in enumerate(chosen):            # scatter along the slot axis
+                out_k[b, h, e] = k_new[b, h, c]
+                out_v[b, h, e] = v_new[b, h, c]
+                out_pos[b, h, e] = pos0 + c
+                out_scores[b, h, e] = new[c]
+    return dict(scores=out_scores, slot_pos=out_pos, k_cache=out_k, v_cache=out_v,
+                evict_idx=evict)
+
+
+class SequenceState:
+    """Cache state of one attention layer: buffers of fixed length M (§3.1)."""
+
+    def __init__(self, B, Hkv, M, d, dtype=np.float32, score_dtype=np.float64):
+        self.k_cache = np.zeros((B, Hkv, M, d), dtype)
+        self.v_cache = np.zeros((B, Hkv, M, d), dtype)
+        self.slot_pos = -np.ones((B, Hkv, M), np.int32)
+        self.scores = np.zeros((B, Hkv, M), score_dtype)
+
+
+def chunk_bounds(T: int, M: int, S: int, prefill: int | None = None):
+    """[(start, end)] of the prefill chunk (default length M) then chunks of S (§A.4.1)."""
+    P0 = min(T, M if prefill is None else prefill)
+    bounds = [(0, P0)] if P0 > 0 else []
+    p = P0
+    while p < T:
+        bounds.append((p, min(T, p + S)))
+        p += S
+    return bounds
+
+
+def run_sequence(q, k, v, M: int, S: int, W: int, prefill: int | None = None,
+                 scale: float | None = None, precision: str = "fp64", on_step=None):
+    """Sparse-attention pass over whole sequences: prefill, then chunks of S.
+
+    q (B,H_q,T,d), k/v (B,H_kv,T,d).  Returns (out (B,H_q,T,d), final state).
+    ``on_step(i, bounds, state_before, result)`` is called after every chunk.
+    """
+    B, Hq, T, d = q.shape
+    Hkv = k.shape[1]
+    st = SequenceState(B, Hkv, M, d, score_dtype=np.float64 if precision == "fp64" else np.float32)
+    out = np.zeros((B, Hq, T, d))
+    for i, (p, e) in enumerate(chunk_bounds(T, M, S, prefill)):
+        o, inc, _ = sdpa_chunk(q[:, :, p:e], st.k_cache, st.v_cache, k[:, :, p:e], v[:, :, p:e],
+                               st.slot_pos, p, scale)
+        out[:, :, p:e] = o
+        res = update(st.scores, st.slot_pos, inc, k[:, :, p:e], v[:, :, p:e],
+                     st.k_cache, st.v_cache, p, W, precision)
+        before = (st.scores, st.slot_pos, st.k_cache, st.v_cache)
+        st.scores, st.slot_pos = res["scores"], res["slot_pos"]
+        st.k_cache, st.v_cache = res["k_cache"], res["v_cache"]
+        if on_step is not None:
+            on_step(i, (p, e), before, dict(out=o, score_inc=inc, **res))
+    return out, st

@@ -1,0 +1,436 @@
+"""Benchmark: H2O sparse attention over a whole long sequence on one GB300.
+
+A step is one pass of the whole hot path over one sequence batch of the
+workload: empty the cache, prefill M tokens, then every chunk of S tokens
+(h2o_sdpa_chunk + h2o_update).  Default workload: one Llama-3-8B-shaped layer
+(B=1, Hq=32, Hkv=8, d=128), T=32768 tokens, chunks of 512, cache of 4096 slots,
+recent window 512.  Inputs are seeded synthetic bf16 tensors resident in HBM
+(402 MB per step, more than the 129 MB L2, so each step streams them).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload NAME] [--no-e2e] [--no-cpu-baseline]
+
+Prints one JSON line.  ``--impl reference`` times the float64 CPU oracle on a
+bounded sample of the same workload instead (the reference arm).
+Under torchrun every rank runs its own replica of the workload (the path has
+no exchange step: batches and KV heads are independent), timing is the max
+over ranks and rank 0 prints.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_19920_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "H2O SDPA prefill tokens/s and TFLOP/s (% of GB300 bf16 tensor peak), 1 GPU"
+
+
+def chunk_flops(B, Hq, d, S, M_visible):
+    """Algorithmic flops of one chunk: QK^T and PV over the visible keys only
+    (M cache slots plus the causal half of the chunk's own S x S block)."""
+    return 4.0 * B * Hq * d * S * (M_visible + (S + 1) / 2.0)
+
+
+def step_plan(w: wl.Workload):
+    """[(start, end)] of the prefill and the chunks of one sequence."""
+    from paper_2608_19920_gb300.runner import chunk_bounds
+    return chunk_bounds(w.T, w.M, w.S)
+
+
+def step_flops(w: wl.Workload):
+    plan = step_plan(w)
+    prefill = chunk_flops(w.B, w.Hq, w.d, plan[0][1], 0)
+    chunks = [chunk_flops(w.B, w.Hq, w.d, e - p, w.M) for p, e in plan[1:]]
+    return prefill, chunks
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(bf16=p.get("bf16_tflops", 1896.2), bf16_sus=p.get("bf16_tflops_sustained", 1698.6),
+                    hbm=p.get("hbm_gbs", 6775.9), source="measured")
+    return dict(bf16=1900.0, bf16_sus=1700.0, hbm=6800.0, source="fallback")
+
+
+# ---------------------------------------------------------------- clocks --
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.file = None
+
+    def __enter__(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.file is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.file.flush()
+        rows = []
+        with open(self.file.name) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.file.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "samples": len(rows), "reasons": reasons}
+
+
+# ------------------------------------------------------------ distributed --
+def dist_setup(n_gpus):
+    """(rank, world, local_rank); initialises a gloo group for timing under torchrun."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("gloo", rank=rank, world_size=world)
+    return rank, world, local
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------- CPU baseline --
+def oracle_sample(w: wl.Workload, budget_s: float = 12.0, max_chunks: int = 8):
+    """Times the float64 oracle on chunk steps of the workload (cache full).
+
+    Sample: starting from a full cache (random state of the right shape), the
+    oracle runs chunk steps (sparse SDPA + update) until ``budget_s`` seconds
+    or ``max_chunks`` chunks; returns tokens/s and a description."""
+    from oracle import sdpa_chunk, update
+    rng = np.random.default_rng(0)
+    p0 = w.M + w.S  # a position in the steady state
+    st = wl.random_state(rng, w.B, w.Hkv, w.M, w.d, pos0=p0)
+    n, t_total = 0, 0.0
+    while n < max_chunks and t_total < budget_s:
+        p = p0 + n * w.S
+        if p + w.S > w.T:
+            break
+        q, k, v = wl.batch_tokens(w, p, p + w.S)
+        t0 = time.perf_counter()
+        _, inc, _ = sdpa_chunk(q, st["k_cache"], st["v_cache"], k, v, st["slot_pos"], p)
+        r = update(st["scores"], st["slot_pos"], inc, k, v, st["k_cache"], st["v_cache"], p, w.W,
+                   "fp64")
+        t_total += time.perf_counter() - t0
+        st = dict(scores=r["scores"], slot_pos=r["slot_pos"], k_cache=r["k_cache"],
+                  v_cache=r["v_cache"])
+        n += 1
+    tokens = n * w.S * w.B
+    return dict(value=tokens / t_total, unit="tokens/s", cores=os.cpu_count(), kind="oracle",
+                seconds=t_total,
+                sample=(f"{n} steady-state chunk steps ({w.S} tokens x B={w.B}, cache of {w.M} "
+                        f"slots full) of the {w.name} workload, float64 NumPy oracle"))
+
+
+def run_reference(args, w):
+    rank, world, _ = dist_setup(args.gpus)
+    if rank != 0:
+        return 0
+    times = []
+    tokens = 0
+    for i in range(args.warmup + args.steps):
+        r = oracle_sample(w, budget_s=args.ref_budget, max_chunks=1)
+        if i >= args.warmup:
+            times.append(r["seconds"])
+            tokens += w.S * w.B
+    value = tokens / sum(times)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d,
+                       "T": w.T, "S": w.S, "M": w.M, "W": w.W,
+                       "step": "one steady-state chunk step per step (CPU sample)"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(),
+                             "kind": "oracle",
+                             "sample": f"one {w.S}-token chunk step per step, cache of {w.M} full"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# ------------------------------------------------------------------ ours --
+def make_inputs(w, dev, pinned=False):
+    """Chunk-major bf16 inputs of one sequence batch: a list of (q, k, v) per chunk."""
+    import torch
+    chunks = []
+    for p, e in step_plan(w):
+        q, k, v = wl.batch_tokens(w, p, e)
+        ts = []
+        for x in (q, k, v):
+            t = torch.from_numpy(x).to(torch.bfloat16)
+            ts.append(t.pin_memory() if pinned else t.to(dev))
+        chunks.append(tuple(ts))
+    return chunks
+
+
+def run_ours(args, w):
+    import torch
+    from paper_2608_19920_gb300 import H2OLayer, h2o_device_errors
+    from paper_2608_19920_gb300 import build as build_mod
+
+    rank, world, local = dist_setup(args.gpus)
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    build_mod.build()
+    plan = step_plan(w)
+    pre_flops, chunk_fl = step_flops(w)
+    total_flops = pre_flops + sum(chunk_fl)
+    tokens_per_step = w.B * w.T
+
+    inputs = make_inputs(w, dev)
+    outs = [torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=dev)
+            for p, e in plan]
+    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, keep_evictions=True)
+    stream = torch.cuda.current_stream()
+    n_chunks = len(plan) - 1
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(n_chunks)]
+
+    def one_step(record=False):
+        layer.reset()
+        for i, ((p, e), (q, k, v)) in enumerate(zip(plan, inputs)):
+            if record and i > 0:
+                ev[i - 1][0].record(stream)
+                layer.step(q, k, v, p, out=outs[i])
+                ev[i - 1][1].record(stream)
+            else:
+                layer.step(q, k, v, p, out=outs[i])
+
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize()
+    if h2o_device_errors() != 0:
+        raise SystemExit("device-side error during warm-up")
+
+    # ---- timed region: K steps, inputs resident in HBM
+    sdpa_ms = []
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for s in range(args.steps):
+            one_step(record=(s == args.steps - 1))
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed_ms = t0.elapsed_time(t1)
+    barrier(world)
+    elapsed_ms = max_over_ranks(elapsed_ms, world)
+    step_ms = elapsed_ms / args.steps
+    # chunk-step durations (sdpa + update) of the last timed step
+    chunk_step_ms = [a.elapsed_time(b) for a, b in ev]
+    clocks = clk.summary()
+    if h2o_device_errors() != 0:
+        raise SystemExit("device-side error during the timed region")
+
+    # ---- dominant kernel: the chunk SDPA alone, timed on the same stream
+    kern = time_sdpa_kernel(w, layer, inputs, plan, stream, reps=max(3, args.steps))
+
+    value = tokens_per_step * world / (step_ms / 1e3)
+    pk = peaks()
+    alg_tflops = total_flops / (step_ms / 1e3) / 1e12
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded Gaussian Q/K/V with planted heavy-hitter keys)",
+        "config": {"workload": w.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d, "T": w.T,
+                   "S": w.S, "M": w.M, "W": w.W, "tokens_per_step": tokens_per_step,
+                   "chunks_per_step": n_chunks, "l2": "inputs larger than L2 (402 MB per step)",
+                   "parallelism": f"replicas x{world}"},
+        "tflops": alg_tflops,
+        "tflops_frac_of_peak": alg_tflops / pk["bf16_sus"],
+        "chunk_step_ms_median": statistics.median(chunk_step_ms) if chunk_step_ms else None,
+        "gpu_launches": args.steps * (2 * len(plan)),
+        "clocks": clocks,
+    }
+    line["roofline"] = {
+        "bound": "tensor", "kernel": "sdpa_chunk_kernel<128> (steady-state chunk)",
+        "achieved": kern["alg_tflops"], "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+        "frac": kern["alg_tflops"] / pk["bf16_sus"], "traffic": args.traffic,
+        "peak_source": f"{pk['source']} bf16 dense, sustained",
+        "avg_launch_us": kern["avg_us"], "flops_per_launch": kern["flops"],
+        "executed_tflops": kern["alg_tflops"] * kern["exec_ratio"],
+    }
+    if args.e2e:
+        line["e2e"] = run_e2e(w, layer, plan, outs, dev, args, world)
+    if args.cpu_baseline and rank == 0 and world == 1:
+        line["cpu_baseline"] = oracle_sample(w)
+    if rank == 0:
+        print(json.dumps(line))
+    return 0
+
+
+def time_sdpa_kernel(w, layer, inputs, plan, stream, reps):
+    """Average duration of the steady-state chunk SDPA launch (CUDA events)."""
+    import torch
+    from paper_2608_19920_gb300 import h2o_sdpa_chunk
+    idx = len(plan) // 2
+    p, e = plan[idx]
+    q, k, v = inputs[idx]
+    out = torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=q.device)
+    inc = torch.empty((w.B, w.Hq, w.M + e - p), dtype=torch.float32, device=q.device)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
+    times = []
+    for _ in range(reps + 2):
+        flush.zero_()  # evict the previous launch's data from L2
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out=out,
+                       score_inc=inc)
+        b.record(stream)
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(b))
+    times = times[2:]
+    avg_ms = sum(times) / len(times)
+    flops = chunk_flops(w.B, w.Hq, w.d, e - p, w.M)
+    exec_flops = executed_mma_flops(w, e - p)
+    return dict(avg_us=avg_ms * 1e3, flops=flops, alg_tflops=flops / (avg_ms / 1e3) / 1e12,
+                exec_ratio=exec_flops / flops)
+
+
+def executed_mma_flops(w, S):
+    """Tensor-core flops the two-pass kernel issues for one chunk with a full
+    cache: per visited 128x128 key tile, Q K^T twice and P V once."""
+    tile = 2.0 * 128 * 128 * w.d
+    n_cache = -(-w.M // 128)
+    total = 0.0
+    if S > 128:
+        for i0 in range(0, S, 128):
+            total += w.q_g * (n_cache + i0 // 128 + 1)
+    else:
+        per_tile = 128 // (-(-S // 32) * 32)
+        total += -(-w.q_g // per_tile) * (n_cache + 1)
+    return 3 * tile * total * w.B * w.Hkv
+
+
+def run_e2e(w, layer, plan, outs, dev, args, world):
+    """Same metric through the public API from pinned host buffers: per step,
+    copy the sequence's inputs host->device, run, copy the outputs back."""
+    import torch
+    host_in = make_inputs(w, dev, pinned=True)
+    dev_in = [tuple(torch.empty_like(x, device=dev) for x in c) for c in host_in]
+    host_out = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    h2d = sum(x.numel() * x.element_size() for c in host_in for x in c)
+    d2h = sum(o.numel() * o.element_size() for o in outs)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        layer.reset()
+        for (p, e), hx, dx, o, ho in zip(plan, host_in, dev_in, outs, host_out):
+            for a, b in zip(dx, hx):
+                a.copy_(b, non_blocking=True)
+            layer.step(dx[0], dx[1], dx[2], p, out=o)
+            ho.copy_(o, non_blocking=True)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    n = max(2, args.steps // 2)
+    t0.record(stream)
+    for _ in range(n):
+        step()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(t0.elapsed_time(t1) / n, world)
+    return {"value": w.B * w.T * world / (ms / 1e3), "unit": "tokens/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama8b_32k", choices=sorted(wl.WORKLOADS))
+    ap.add_argument("--no-e2e", dest="e2e", action="store_false")
+    ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="DRAM bytes per launch of the dominant kernel from an ncu capture")
+    ap.add_argument("--ref-budget", type=float, default=20.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    w = wl.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_ours(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

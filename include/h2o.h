@@ -1,0 +1,169 @@
+/*
+ * h2o.h - C ABI of the GB300 (sm_103a) H2O sparse-attention library.
+ *
+ * One attention layer with a fixed-size KV cache of M slots per (batch, KV
+ * head), processed chunk by chunk (paper §3.1: prefill, then chunks of S
+ * tokens).  Two calls make up one chunk step:
+ *
+ *   h2o_sdpa_chunk  the chunk's S queries attend to the M cache slots and,
+ *                   causally, to the chunk's own keys (§3.1 Eq. 2 with the
+ *                   position mask of §3.3.1); besides the attention output it
+ *                   returns the summed attention weights sum_i m_ij per key
+ *                   column (§3.3.1, §A.6), shape (B, H_q, M + S).
+ *   h2o_update      adds those weights into the per-(batch, KV head) H2O
+ *                   scores (§3.1.1 Eq. 3, summed over the query heads of the
+ *                   GQA group), evicts the S lowest-scoring slots outside the
+ *                   recent window and writes the chunk's keys and values into
+ *                   them (the scatter of §3.2 / §A.1.1).
+ *
+ * Conventions for every call:
+ *  - All array arguments are DEVICE pointers, allocated and owned by the
+ *    caller; the library allocates no memory and keeps no per-call state.
+ *    Every array is dense, row-major (C order) with the shape given, and must
+ *    be 16-byte aligned.
+ *  - bf16 arrays hold IEEE bfloat16 bit patterns (h2o_bf16 = uint16_t).
+ *  - Calls only enqueue work on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream) and return without synchronising.  Arguments are
+ *    validated on the host first; on any error nothing is enqueued.
+ *  - Return value: H2O_OK (0) or a negative H2O_ERR_* code; h2o_status_string
+ *    gives a message.  For H2O_ERR_CUDA, h2o_last_cuda_error() gives the
+ *    cudaError_t of the failing runtime call on this host thread.
+ *  - Device-side problems (a bounded wait that ran out, fewer eviction
+ *    candidates than S found in slot_pos) are recorded in a per-device error
+ *    word; h2o_device_errors() synchronises the device and reads and clears it.
+ *  - Token positions are int32; pos0 + S must stay below 2^31.
+ */
+#ifndef H2O_GB300_H2O_H_
+#define H2O_GB300_H2O_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define H2O_API __attribute__((visibility("default")))
+#else
+#define H2O_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t h2o_bf16;
+
+/* Problem sizes of one layer.  Hq % Hkv == 0 (GQA, §3.1: query head hq uses
+ * KV head hq / (Hq / Hkv)); d is the head dimension (64 or 128); S >= 1 is
+ * the chunk length; M >= 0 is the number of cache slots. */
+typedef struct h2o_dims {
+  int32_t B, Hq, Hkv, d, S, M;
+} h2o_dims_t;
+
+enum {
+  H2O_OK = 0,
+  H2O_ERR_NULL = -1,        /* a required pointer is NULL */
+  H2O_ERR_SHAPE = -2,       /* inconsistent or out-of-range sizes */
+  H2O_ERR_ALIGN = -3,       /* a pointer is not 16-byte aligned */
+  H2O_ERR_UNSUPPORTED = -4, /* valid request this build does not handle (e.g. d) */
+  H2O_ERR_WORKSPACE = -5,   /* workspace NULL or smaller than h2o_workspace_size */
+  H2O_ERR_ARG = -6,         /* bad scalar argument (window, budget, position) */
+  H2O_ERR_CUDA = -7,        /* a CUDA runtime call failed; see h2o_last_cuda_error */
+  H2O_ERR_TIMEOUT = -8,     /* device: a bounded wait ran out (reported by h2o_device_errors) */
+  H2O_ERR_DEVICE = -9,      /* device: fewer eviction candidates than S, etc. */
+  H2O_ERR_NODEVICE = -10    /* no usable sm_100-family GPU is current */
+};
+
+/* Device error bits reported by h2o_device_errors(). */
+enum {
+  H2O_DEVERR_TIMEOUT = 1,   /* a kernel's bounded wait on a barrier ran out */
+  H2O_DEVERR_CANDIDATES = 2 /* h2o_update found fewer than S evictable slots */
+};
+
+/* Bytes of scratch memory h2o_sdpa_chunk needs for `dims` (may be 0). */
+H2O_API int h2o_workspace_size(const h2o_dims_t* dims, size_t* bytes);
+
+/*
+ * One chunk of sparse SDPA with summed attention weights (§3.1 Eq. 2, mask of
+ * §3.3.1, summed weights of §3.3.1 / §A.6.1).
+ *
+ *   q         (B, Hq, S, d) bf16   queries of tokens pos0 .. pos0+S-1
+ *   k_cache   (B, Hkv, M, d) bf16  cache keys   (may be NULL when M == 0)
+ *   v_cache   (B, Hkv, M, d) bf16  cache values (may be NULL when M == 0)
+ *   k_new     (B, Hkv, S, d) bf16  the chunk's keys
+ *   v_new     (B, Hkv, S, d) bf16  the chunk's values
+ *   slot_pos  (B, Hkv, M) int32    token position held by each slot, -1 = empty
+ *   out       (B, Hq, S, d) bf16   attention output (written)
+ *   score_inc (B, Hq, M + S) f32   summed weights sum_i m_ij (written): columns
+ *                                  0..M-1 are the cache slots, M..M+S-1 the
+ *                                  chunk's own tokens in order
+ *
+ * Query row i (token pos0 + i) sees cache slot j iff 0 <= slot_pos[j] <=
+ * pos0 + i, and chunk token c iff c <= i.  softmax_scale <= 0 selects
+ * d^-1/2.  Every query row must see at least one key (it always sees its own
+ * token).  `workspace` may be NULL when h2o_workspace_size reports 0.
+ */
+H2O_API int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                   const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
+                   h2o_bf16* out, float* score_inc, void* workspace, size_t workspace_bytes,
+                   void* stream);
+
+/*
+ * H2O cache update after h2o_sdpa_chunk (§3.1.1 Eq. 3 and the eviction rule
+ * that follows it; scatter of §3.2 / §A.1.1).  Per (b, kv head h):
+ *
+ *   t_j   = score_inc[b, h*qg + 0, j] + ... + score_inc[b, h*qg + qg-1, j]
+ *           (float32, added in ascending g, no fused multiply-add)
+ *   acc_j = scores[b,h,j] + t_j                       for cache slots j < M
+ *   candidates: slots with slot_pos < pos0 + S - recent_window (empty slots,
+ *   position -1, always qualify); the S smallest under the total order
+ *   (empty first, then acc ascending, then slot index ascending) are evicted;
+ *   the c-th smallest evicted slot e receives token pos0 + c:
+ *   k_cache[b,h,e,:] = k_new[b,h,c,:], v_cache likewise, slot_pos = pos0 + c,
+ *   scores = t_{M+c}; every other slot keeps its K/V/position and gets acc_j.
+ *
+ *   scores    (B, Hkv, M) f32      in/out
+ *   slot_pos  (B, Hkv, M) int32    in/out
+ *   score_inc (B, Hq, M + S) f32   in (from h2o_sdpa_chunk)
+ *   k_new, v_new (B, Hkv, S, d) bf16 in
+ *   k_cache, v_cache (B, Hkv, M, d) bf16 in/out
+ *   budget    must equal dims->M (the cache length N_C of the paper)
+ *   recent_window  0 <= W <= M; needs M - max(0, W - S) >= S
+ *   evict_idx (B, Hkv, S) int32    out, optional (NULL = not written): the
+ *             slot that received token pos0 + c; this is the content of the
+ *             paper's replay log / scatter index (§3.2)
+ *
+ * If a (b, h) has fewer than S candidates at run time (slot_pos not produced
+ * by this policy), that (b, h) is left unchanged and H2O_DEVERR_CANDIDATES is
+ * recorded.
+ */
+H2O_API int h2o_update(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+               const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
+               h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget, int32_t recent_window,
+               int32_t* evict_idx, void* stream);
+
+/* Empties a cache before a new sequence: slot_pos (B, Hkv, M) int32 := -1 and
+ * scores (B, Hkv, M) f32 := 0, enqueued on `stream` (the K/V buffers need no
+ * clearing: empty slots are never attended and are overwritten first).  This
+ * is the state of §3.1 before the first token: a cache filled left to right. */
+H2O_API int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores,
+                            void* stream);
+
+/* Message for a status code (static storage). */
+H2O_API const char* h2o_status_string(int status);
+
+/* cudaError_t of the last failing CUDA runtime call on this host thread. */
+H2O_API int h2o_last_cuda_error(void);
+
+/* Synchronises the current device, returns the H2O_DEVERR_* bits recorded by
+ * kernels since the last call (0 = none) and clears them.  Negative on a CUDA
+ * failure. */
+H2O_API int h2o_device_errors(void);
+
+/* Library version as major*10000 + minor*100 + patch. */
+H2O_API int h2o_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* H2O_GB300_H2O_H_ */

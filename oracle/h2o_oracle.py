@@ -54,7 +54,8 @@ def _token_positions(slot_pos_bh: np.ndarray, pos0: int, S: int) -> np.ndarray:
     return np.concatenate([slot_pos_bh.astype(np.int64), pos0 + np.arange(S, dtype=np.int64)])
 
 
-def sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale: float | None = None):
+def sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale: float | None = None,
+               rows=None):
     """One chunk of H2O sparse SDPA (§3.1 Eq. 2 + summed weights of §3.3.1 / §A.6).
 
     Args:
@@ -67,17 +68,20 @@ def sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale: fl
 
     Returns (out (B,H_q,S,d), score_inc (B,H_q,M+S), lse (B,H_q,S)), float64.
     Key columns are ordered cache slots 0..M-1, then chunk tokens 0..S-1.
+    ``rows`` (optional) restricts the computation to those query rows i: out and
+    lse then have len(rows) rows and score_inc sums over those rows only.
     """
     q = np.asarray(q, np.float64)
     B, Hq, S, d = q.shape
+    ridx = np.arange(S) if rows is None else np.asarray(rows, np.int64)
     Hkv, M = slot_pos.shape[1], slot_pos.shape[2]
     assert Hq % Hkv == 0
     qg = Hq // Hkv
     if scale is None:
         scale = 1.0 / math.sqrt(d)
-    out = np.zeros((B, Hq, S, d))
+    out = np.zeros((B, Hq, len(ridx), d))
     score_inc = np.zeros((B, Hq, M + S))
-    lse = np.zeros((B, Hq, S))
+    lse = np.zeros((B, Hq, len(ridx)))
     for b in range(B):
         for hq in range(Hq):
             h = hq // qg
@@ -87,9 +91,9 @@ def sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale: fl
                                    np.asarray(v_new[b, h], np.float64)])
             t = _token_positions(slot_pos[b, h], pos0, S)
             # mask: hidden iff the slot is empty or P + i < t(j)  (§3.3.1)
-            qpos = pos0 + np.arange(S)[:, None]
+            qpos = pos0 + ridx[:, None]
             visible = (t[None, :] >= 0) & (t[None, :] <= qpos)
-            a = scale * (q[b, hq] @ keys.T)
+            a = scale * (q[b, hq][ridx] @ keys.T)
             a = np.where(visible, a, -np.inf)
             amax = a.max(axis=1, keepdims=True)
             lam = amax + np.log(np.exp(a - amax).sum(axis=1, keepdims=True))

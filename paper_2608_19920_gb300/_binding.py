@@ -1,0 +1,203 @@
+"""ctypes binding of libh2o_gb300.so (include/h2o.h): argument marshalling only.
+
+Every step of the computation runs in the CUDA library; these wrappers check
+tensor shapes, dtypes and devices, pass raw device pointers and the current
+CUDA stream, and turn negative status codes into exceptions.  There is no CPU
+or PyTorch fallback: without the built library every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libh2o_gb300.so")
+
+H2O_OK = 0
+H2O_DEVERR_TIMEOUT = 1
+H2O_DEVERR_CANDIDATES = 2
+
+# Every symbol include/h2o.h declares.
+EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_cache_reset",
+           "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors", "h2o_version")
+
+
+class H2ODims(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("Hq", ctypes.c_int32), ("Hkv", ctypes.c_int32),
+                ("d", ctypes.c_int32), ("S", ctypes.c_int32), ("M", ctypes.c_int32)]
+
+
+class H2OError(RuntimeError):
+    def __init__(self, fn: str, status: int, lib):
+        msg = lib.h2o_status_string(status).decode()
+        if status == -7:
+            msg += f" (cudaError {lib.h2o_last_cuda_error()})"
+        super().__init__(f"{fn} failed: {msg} [{status}]")
+        self.status = status
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Loads the library (once) and declares the C signatures."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(
+            f"CUDA library not built: {path} is missing. Build it with "
+            "`python -m paper_2608_19920_gb300.build` (needs nvcc); there is no fallback.")
+    lib = ctypes.CDLL(path)
+    vp, i32, i64, f32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+    dims_p = ctypes.POINTER(H2ODims)
+    lib.h2o_workspace_size.argtypes = [dims_p, ctypes.POINTER(ctypes.c_size_t)]
+    lib.h2o_sdpa_chunk.argtypes = [dims_p, i64, f32, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                   ctypes.c_size_t, vp]
+    lib.h2o_update.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, vp]
+    lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
+    lib.h2o_status_string.argtypes = [ctypes.c_int]
+    lib.h2o_status_string.restype = ctypes.c_char_p
+    for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_cache_reset",
+               "h2o_last_cuda_error",
+               "h2o_device_errors", "h2o_version"):
+        getattr(lib, fn).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def _check(fn: str, status: int):
+    if status != H2O_OK:
+        raise H2OError(fn, status, _lib)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _expect(t, name, shape, dtype, device):
+    if t is None:
+        raise ValueError(f"{name} is required")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: expected shape {tuple(shape)}, got {tuple(t.shape)}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name}: expected {dtype}, got {t.dtype}")
+    if t.device != device:
+        raise ValueError(f"{name}: expected device {device}, got {t.device}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def dims_of(q, k_cache_or_M, k_new):
+    B, Hq, S, d = q.shape
+    Hkv = k_new.shape[1]
+    M = k_cache_or_M if isinstance(k_cache_or_M, int) else k_cache_or_M.shape[2]
+    return H2ODims(B, Hq, Hkv, d, S, M)
+
+
+def h2o_workspace_size(dims: H2ODims) -> int:
+    lib = load()
+    n = ctypes.c_size_t(0)
+    _check("h2o_workspace_size", lib.h2o_workspace_size(ctypes.byref(dims), ctypes.byref(n)))
+    return n.value
+
+
+def h2o_sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale: float = 0.0,
+                   out=None, score_inc=None, workspace=None, stream=None):
+    """Sparse SDPA of one chunk + summed attention weights (see include/h2o.h).
+
+    q (B,Hq,S,d) bf16; k_cache/v_cache (B,Hkv,M,d) bf16; k_new/v_new (B,Hkv,S,d)
+    bf16; slot_pos (B,Hkv,M) int32.  Returns (out (B,Hq,S,d) bf16,
+    score_inc (B,Hq,M+S) f32).
+    """
+    lib = load()
+    dev = q.device
+    B, Hq, S, d = q.shape
+    Hkv = k_new.shape[1]
+    M = k_cache.shape[2]
+    bf = torch.bfloat16
+    _expect(q, "q", (B, Hq, S, d), bf, dev)
+    _expect(k_cache, "k_cache", (B, Hkv, M, d), bf, dev)
+    _expect(v_cache, "v_cache", (B, Hkv, M, d), bf, dev)
+    _expect(k_new, "k_new", (B, Hkv, S, d), bf, dev)
+    _expect(v_new, "v_new", (B, Hkv, S, d), bf, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    if out is None:
+        out = torch.empty((B, Hq, S, d), dtype=bf, device=dev)
+    if score_inc is None:
+        score_inc = torch.empty((B, Hq, M + S), dtype=torch.float32, device=dev)
+    _expect(out, "out", (B, Hq, S, d), bf, dev)
+    _expect(score_inc, "score_inc", (B, Hq, M + S), torch.float32, dev)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.h2o_sdpa_chunk(ctypes.byref(dims), int(pos0), float(scale), _ptr(q), _ptr(k_cache),
+                            _ptr(v_cache), _ptr(k_new), _ptr(v_new), _ptr(slot_pos), _ptr(out),
+                            _ptr(score_inc), _ptr(workspace), ws_bytes, _stream(stream))
+    _check("h2o_sdpa_chunk", st)
+    return out, score_inc
+
+
+def h2o_update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0: int,
+               recent_window: int, evict_idx=None, budget: int | None = None, stream=None):
+    """H2O score accumulation, eviction and K/V write, in place (see include/h2o.h).
+
+    scores (B,Hkv,M) f32, slot_pos (B,Hkv,M) int32, score_inc (B,Hq,M+S) f32,
+    k_new/v_new (B,Hkv,S,d) bf16, k_cache/v_cache (B,Hkv,M,d) bf16,
+    evict_idx (B,Hkv,S) int32 or None.  Returns evict_idx.
+    """
+    lib = load()
+    dev = scores.device
+    B, Hkv, M = scores.shape
+    S, d = k_new.shape[2], k_new.shape[3]
+    Hq = score_inc.shape[1]
+    _expect(scores, "scores", (B, Hkv, M), torch.float32, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    _expect(score_inc, "score_inc", (B, Hq, M + S), torch.float32, dev)
+    _expect(k_new, "k_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect(v_new, "v_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect(k_cache, "k_cache", (B, Hkv, M, d), torch.bfloat16, dev)
+    _expect(v_cache, "v_cache", (B, Hkv, M, d), torch.bfloat16, dev)
+    if evict_idx is not None:
+        _expect(evict_idx, "evict_idx", (B, Hkv, S), torch.int32, dev)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    st = lib.h2o_update(ctypes.byref(dims), int(pos0), _ptr(scores), _ptr(slot_pos),
+                        _ptr(score_inc), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache),
+                        int(M if budget is None else budget), int(recent_window), _ptr(evict_idx),
+                        _stream(stream))
+    _check("h2o_update", st)
+    return evict_idx
+
+
+def h2o_cache_reset(slot_pos, scores, stream=None):
+    """slot_pos := -1, scores := 0 (an empty cache), enqueued on the stream."""
+    lib = load()
+    B, Hkv, M = slot_pos.shape
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, slot_pos.device)
+    _expect(scores, "scores", (B, Hkv, M), torch.float32, slot_pos.device)
+    dims = H2ODims(B, Hkv, Hkv, 64, 1, M)
+    _check("h2o_cache_reset", lib.h2o_cache_reset(ctypes.byref(dims), _ptr(slot_pos),
+                                                  _ptr(scores), _stream(stream)))
+
+
+def h2o_device_errors() -> int:
+    lib = load()
+    r = lib.h2o_device_errors()
+    if r < 0:
+        _check("h2o_device_errors", r)
+    return r
+
+
+def h2o_status_string(status: int) -> str:
+    return load().h2o_status_string(status).decode()
+
+
+def h2o_version() -> int:
+    return load().h2o_version()

@@ -1,0 +1,281 @@
+// C ABI of the H2O sparse-attention library: argument checking, tensor-map
+// encoding and kernel launches.  Declarations and contracts: include/h2o.h.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/h2o.h"
+#include "h2o_internal.h"
+
+namespace h2o {
+
+// Device-side error bits (H2O_DEVERR_*), one word per device.
+__device__ int g_device_errors;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+thread_local int t_last_cuda_error = 0;
+
+struct DeviceInfo {
+  std::once_flag once;
+  cudaError_t status = cudaSuccess;
+  bool supported = false;
+  int* err_word = nullptr;
+};
+DeviceInfo g_dev[kMaxDevices];
+
+std::once_flag g_encode_once;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int cuda_fail(cudaError_t e) {
+  t_last_cuda_error = static_cast<int>(e);
+  return H2O_ERR_CUDA;
+}
+
+// Resolves the current device once: architecture check and error-word address.
+int current_device(DeviceInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e == cudaErrorNoDevice || e == cudaErrorInsufficientDriver
+                                   ? H2O_ERR_NODEVICE
+                                   : cuda_fail(e);
+  if (dev < 0 || dev >= kMaxDevices) return H2O_ERR_NODEVICE;
+  DeviceInfo& di = g_dev[dev];
+  std::call_once(di.once, [&di, dev] {
+    cudaDeviceProp prop;
+    di.status = cudaGetDeviceProperties(&prop, dev);
+    if (di.status != cudaSuccess) return;
+    di.supported = prop.major == 10;
+    if (!di.supported) return;
+    di.status = cudaGetSymbolAddress(reinterpret_cast<void**>(&di.err_word), g_device_errors);
+  });
+  if (di.status != cudaSuccess) return cuda_fail(di.status);
+  if (!di.supported) return H2O_ERR_NODEVICE;
+  *out = &di;
+  return H2O_OK;
+}
+
+int get_encoder() {
+  std::call_once(g_encode_once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_encode ? H2O_OK : H2O_ERR_NODEVICE;
+}
+
+bool misaligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
+
+// bf16 tensor map, 128-byte swizzle, dims/box innermost first.
+int encode(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint32_t* box) {
+  cuuint64_t gd[5], gs[4];
+  cuuint32_t bx[5], es[5];
+  uint64_t stride = 2;
+  for (int r = 0; r < rank; ++r) {
+    gd[r] = dims[r];
+    bx[r] = box[r];
+    es[r] = 1;
+    if (r > 0) gs[r - 1] = stride;
+    stride *= dims[r];
+  }
+  const CUresult res = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base),
+                                gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS ? H2O_OK : H2O_ERR_SHAPE;
+}
+
+int check_dims(const h2o_dims_t* d) {
+  if (!d) return H2O_ERR_NULL;
+  if (d->B < 1 || d->Hq < 1 || d->Hkv < 1 || d->S < 1 || d->M < 0 || d->d < 1) return H2O_ERR_SHAPE;
+  if (d->Hq % d->Hkv != 0) return H2O_ERR_SHAPE;
+  if (d->d != 64 && d->d != 128) return H2O_ERR_UNSUPPORTED;
+  if (d->B * static_cast<int64_t>(d->Hkv) > 65535) return H2O_ERR_UNSUPPORTED;
+  const int64_t tiles = (d->M + kTileN - 1) / kTileN + (d->S + kTileN - 1) / kTileN;
+  if (tiles > kMaxKeyTiles) return H2O_ERR_UNSUPPORTED;
+  const int64_t elems = static_cast<int64_t>(d->B) * d->Hq * (static_cast<int64_t>(d->M) + d->S);
+  if (elems > (int64_t(1) << 40)) return H2O_ERR_SHAPE;
+  return H2O_OK;
+}
+
+}  // namespace
+}  // namespace h2o
+
+using namespace h2o;
+
+extern "C" {
+
+int h2o_version(void) { return 100; }
+
+const char* h2o_status_string(int s) {
+  switch (s) {
+    case H2O_OK: return "ok";
+    case H2O_ERR_NULL: return "a required pointer is NULL";
+    case H2O_ERR_SHAPE: return "inconsistent or out-of-range sizes";
+    case H2O_ERR_ALIGN: return "a pointer is not 16-byte aligned";
+    case H2O_ERR_UNSUPPORTED: return "unsupported configuration (head dim must be 64 or 128)";
+    case H2O_ERR_WORKSPACE: return "workspace missing or too small";
+    case H2O_ERR_ARG: return "bad scalar argument (position, budget or recent window)";
+    case H2O_ERR_CUDA: return "a CUDA runtime call failed (see h2o_last_cuda_error)";
+    case H2O_ERR_TIMEOUT: return "a device-side bounded wait ran out";
+    case H2O_ERR_DEVICE: return "device-side error (fewer eviction candidates than S)";
+    case H2O_ERR_NODEVICE: return "no usable sm_100-family GPU is current";
+    default: return "unknown status";
+  }
+}
+
+int h2o_last_cuda_error(void) { return t_last_cuda_error; }
+
+int h2o_workspace_size(const h2o_dims_t* dims, size_t* bytes) {
+  const int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  if (!bytes) return H2O_ERR_NULL;
+  *bytes = 0;
+  return H2O_OK;
+}
+
+int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
+                   const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
+                   const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out,
+                   float* score_inc, void* workspace, size_t workspace_bytes, void* stream) {
+  (void)workspace;
+  (void)workspace_bytes;
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (!q || !k_new || !v_new || !out || !score_inc) return H2O_ERR_NULL;
+  if (D.M > 0 && (!k_cache || !v_cache || !slot_pos)) return H2O_ERR_NULL;
+  if (misaligned(q) || misaligned(k_new) || misaligned(v_new) || misaligned(out) ||
+      misaligned(score_inc) || (D.M > 0 && (misaligned(k_cache) || misaligned(v_cache) ||
+                                            misaligned(slot_pos))))
+    return H2O_ERR_ALIGN;
+  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  if ((st = get_encoder()) != H2O_OK) return st;
+
+  const int qg = D.Hq / D.Hkv;
+  SdpaArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = qg;
+  a.pos0 = static_cast<int>(pos0);
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
+  a.scale_log2 = scale * 1.4426950408889634f;
+  if (D.S > kTileM) {
+    a.rows_box = kTileM;
+    a.heads_box = 1;
+    a.tiles_per_head = (D.S + kTileM - 1) / kTileM;
+    a.n_row_tiles = qg * a.tiles_per_head;
+  } else {
+    a.rows_box = (D.S + 31) / 32 * 32;
+    a.heads_box = kTileM / a.rows_box;
+    a.tiles_per_head = 0;
+    a.n_row_tiles = (qg + a.heads_box - 1) / a.heads_box;
+  }
+  a.n_cache_tiles = (D.M + kTileN - 1) / kTileN;
+  a.n_chunk_tiles = (D.S + kTileN - 1) / kTileN;
+  a.slot_pos = slot_pos;
+  a.out = out;
+  a.score_inc = score_inc;
+  a.err = di->err_word;
+
+  const uint64_t G = static_cast<uint64_t>(D.B) * D.Hkv;
+  {
+    const uint64_t dq[4] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S),
+                            static_cast<uint64_t>(qg), G};
+    const uint32_t bq[4] = {64, static_cast<uint32_t>(a.rows_box), static_cast<uint32_t>(a.heads_box), 1};
+    if ((st = encode(&a.tm_q, q, 4, dq, bq)) != H2O_OK) return st;
+    const uint64_t dn[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S), G};
+    const uint32_t bk[3] = {64, kTileN, 1};
+    if ((st = encode(&a.tm_kn, k_new, 3, dn, bk)) != H2O_OK) return st;
+    if ((st = encode(&a.tm_vn, v_new, 3, dn, bk)) != H2O_OK) return st;
+    if (D.M > 0) {
+      const uint64_t dc[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.M), G};
+      if ((st = encode(&a.tm_kc, k_cache, 3, dc, bk)) != H2O_OK) return st;
+      if ((st = encode(&a.tm_vc, v_cache, 3, dc, bk)) != H2O_OK) return st;
+    }
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t inc_bytes = static_cast<size_t>(G) * qg * (static_cast<size_t>(D.M) + D.S) * sizeof(float);
+  cudaError_t e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = launch_sdpa(a, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return H2O_OK;
+}
+
+int h2o_update(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+               const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
+               h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget, int32_t recent_window,
+               int32_t* evict_idx, void* stream) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (!scores || !slot_pos || !score_inc || !k_new || !v_new || !k_cache || !v_cache)
+    return H2O_ERR_NULL;
+  if (misaligned(scores) || misaligned(slot_pos) || misaligned(score_inc) || misaligned(k_new) ||
+      misaligned(v_new) || misaligned(k_cache) || misaligned(v_cache) ||
+      (evict_idx && misaligned(evict_idx)))
+    return H2O_ERR_ALIGN;
+  if (budget != D.M) return H2O_ERR_ARG;
+  if (D.M < 1 || D.S > D.M) return H2O_ERR_SHAPE;
+  if (recent_window < 0 || recent_window > D.M) return H2O_ERR_ARG;
+  if (D.M - std::max(0, recent_window - D.S) < D.S) return H2O_ERR_ARG;
+  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  UpdateArgs a;
+  a.scores = scores; a.slot_pos = slot_pos; a.score_inc = score_inc;
+  a.k_new = k_new; a.v_new = v_new; a.k_cache = k_cache; a.v_cache = v_cache;
+  a.evict_idx = evict_idx; a.err = di->err_word;
+  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = D.Hq / D.Hkv;
+  a.pos0 = static_cast<int>(pos0);
+  a.W = recent_window;
+  const cudaError_t e = launch_update(a, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e);
+  return H2O_OK;
+}
+
+int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores, void* stream) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  if (dims->M < 1) return H2O_ERR_SHAPE;
+  if (!slot_pos || !scores) return H2O_ERR_NULL;
+  if (misaligned(slot_pos) || misaligned(scores)) return H2O_ERR_ALIGN;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  const size_t n = static_cast<size_t>(dims->B) * dims->Hkv * dims->M;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemsetAsync(slot_pos, 0xFF, n * sizeof(int32_t), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(scores, 0, n * sizeof(float), s);
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_device_errors(void) {
+  DeviceInfo* di = nullptr;
+  const int st = current_device(&di);
+  if (st != H2O_OK) return st;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e);
+  int bits = 0;
+  e = cudaMemcpy(&bits, di->err_word, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (bits) {
+    const int zero = 0;
+    e = cudaMemcpy(di->err_word, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  return bits;
+}
+
+}  // extern "C"

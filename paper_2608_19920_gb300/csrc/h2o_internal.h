@@ -1,0 +1,55 @@
+// Internal interface between the C-ABI layer (h2o_api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+namespace h2o {
+
+constexpr int kTileM = 128;        // query rows per CTA (tcgen05 M)
+constexpr int kTileN = 128;        // keys per tile (tcgen05 N of Q K^T, K of P V)
+constexpr int kMaxKeyTiles = 4096; // cache tiles + chunk tiles a CTA may visit
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded waits: 2 s
+
+struct SdpaArgs {
+  CUtensorMap tm_q;        // 4D {d, S, q_g, B*Hkv}, box {64, rows_box, heads_box, 1}
+  CUtensorMap tm_kc;       // 3D {d, M, B*Hkv}, box {64, 128, 1}
+  CUtensorMap tm_vc;
+  CUtensorMap tm_kn;       // 3D {d, S, B*Hkv}, box {64, 128, 1}
+  CUtensorMap tm_vn;
+  const int32_t* slot_pos; // (B, Hkv, M)
+  uint16_t* out;           // (B, Hq, S, d) bf16
+  float* score_inc;        // (B, Hq, M + S)
+  int* err;                // device error word
+  int B, Hq, Hkv, d, S, M, qg;
+  int pos0;
+  float scale_log2;        // softmax scale * log2(e)
+  int rows_box;            // query rows per head in a tile (S_pad when S <= 128, else 128)
+  int heads_box;           // query heads per tile (1 when S > 128)
+  int tiles_per_head;      // ceil(S / 128) when S > 128, else 0
+  int n_row_tiles;         // CTAs per (b, kv head)
+  int n_cache_tiles;       // ceil(M / 128)
+  int n_chunk_tiles;       // ceil(S / 128)
+};
+
+struct UpdateArgs {
+  float* scores;
+  int32_t* slot_pos;
+  const float* score_inc;
+  const uint16_t* k_new;
+  const uint16_t* v_new;
+  uint16_t* k_cache;
+  uint16_t* v_cache;
+  int32_t* evict_idx;      // may be null
+  int* err;
+  int B, Hq, Hkv, d, S, M, qg;
+  int pos0;
+  int W;
+};
+
+cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
+cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);
+
+}  // namespace h2o

@@ -1,0 +1,228 @@
+// H2O cache update: score accumulation, eviction selection and K/V scatter.
+//
+// One CTA of 1024 threads per (batch, KV head); per §3.1.1 Eq. 3 the score of
+// a slot is the running sum of the attention weights its column received, and
+// the S slots with the smallest scores are overwritten by the chunk (§3.1.1);
+// the write is the scatter along the slot axis of §3.2 / §A.1.1.
+//
+//  1. acc_j = scores_j + (inc_0j + inc_1j + ... ) in float32, query heads of the
+//     GQA group added in ascending order with no fused multiply-add, so the
+//     result is bit-identical to any implementation that follows that order.
+//  2. Each candidate slot gets a 32-bit key that orders (empty first, then acc
+//     ascending): 0 for an empty slot, bits(acc) + 1 otherwise (non-negative
+//     floats order like their bit patterns); protected slots (inside the recent
+//     window) get 0xFFFFFFFF.  Ties on the key are broken by the slot index.
+//  3. S = 1 is an argmin over (key, slot).  Otherwise a 4-pass radix select
+//     (8-bit digits, shared-memory histogram) finds the S-th smallest key T and
+//     how many keys equal to T are taken (the lowest slots first).
+//  4. One sweep in slot order, 1024 slots per round, computes with warp ballots
+//     and a block scan the rank c of every evicted slot (the c-th smallest
+//     evicted slot receives token pos0 + c) and writes slot_pos, scores,
+//     evict_idx; each warp then copies the K and V rows of its evicted slots
+//     with 16-byte vector loads and stores.
+#include "h2o_internal.h"
+#include "sm100.cuh"
+
+namespace h2o {
+namespace {
+
+constexpr int kUpdThreads = 1024;
+constexpr int kUpdWarps = kUpdThreads / 32;
+constexpr uint32_t kProtected = 0xFFFFFFFFu;
+
+struct UpdSmem {
+  uint32_t hist[256];
+  uint32_t warp_tot[kUpdWarps];
+  uint32_t warp_tot2[kUpdWarps];
+  unsigned long long warp_min[kUpdWarps];
+  uint32_t bcast[4];
+};
+
+__device__ __forceinline__ float group_sum(const float* inc, int stride, int qg, int j) {
+  float t = __ldg(inc + j);
+  for (int g = 1; g < qg; ++g) t = __fadd_rn(t, __ldg(inc + static_cast<size_t>(g) * stride + j));
+  return t;
+}
+
+__device__ __forceinline__ uint32_t slot_key(const UpdateArgs& a, const float* sc, const int* sp,
+                                             const float* inc, int j, int thr, float* acc_out) {
+  const int pos = sp[j];
+  const float acc = __fadd_rn(sc[j], group_sum(inc, a.M + a.S, a.qg, j));
+  *acc_out = acc;
+  if (pos >= thr) return kProtected;
+  if (pos < 0) return 0u;
+  return min(__float_as_uint(acc) + 1u, kProtected - 1u);
+}
+
+// Exclusive block scan of one bit per thread; returns the prefix, total in *tot.
+__device__ __forceinline__ uint32_t block_scan_bit(bool f, uint32_t* warp_tot, uint32_t* tot) {
+  const int tid = threadIdx.x, w = tid >> 5, l = tid & 31;
+  const uint32_t m = __ballot_sync(0xffffffffu, f);
+  if (l == 0) warp_tot[w] = __popc(m);
+  __syncthreads();
+  uint32_t before = 0, total = 0;
+  for (int x = 0; x < kUpdWarps; ++x) {
+    const uint32_t c = warp_tot[x];
+    before += x < w ? c : 0u;
+    total += c;
+  }
+  __syncthreads();
+  *tot = total;
+  return before + __popc(m & ((1u << l) - 1u));
+}
+
+__device__ __forceinline__ void copy_row(const UpdateArgs& a, int grp, int c, int e, int lane) {
+  // 32 lanes: lanes 0-15 copy the K row, 16-31 the V row, in 16-byte pieces.
+  const int vec = a.d / 8;  // uint4 per row
+  const bool is_v = lane >= 16;
+  const int l = lane & 15;
+  const uint16_t* src = (is_v ? a.v_new : a.k_new) + (static_cast<size_t>(grp) * a.S + c) * a.d;
+  uint16_t* dst = (is_v ? a.v_cache : a.k_cache) + (static_cast<size_t>(grp) * a.M + e) * a.d;
+  for (int x = l; x < vec; x += 16)
+    reinterpret_cast<uint4*>(dst)[x] = __ldg(reinterpret_cast<const uint4*>(src) + x);
+}
+
+__global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs a) {
+  __shared__ UpdSmem sm;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int grp = blockIdx.x;
+  const int b = grp / a.Hkv, h = grp % a.Hkv;
+  float* sc = a.scores + static_cast<size_t>(grp) * a.M;
+  int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
+  const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * a.qg) * (a.M + a.S);
+  const int thr = a.pos0 + a.S - a.W;  // slots holding positions >= thr are protected
+  const int M = a.M, S = a.S;
+
+  uint32_t T = 0;         // threshold key
+  uint32_t take_eq = 0;   // keys equal to T that are evicted (lowest slots first)
+  if (S == 1) {
+    unsigned long long best = ~0ull;
+    for (int j = tid; j < M; j += kUpdThreads) {
+      float acc;
+      const uint32_t key = slot_key(a, sc, sp, inc, j, thr, &acc);
+      const unsigned long long k64 = (static_cast<unsigned long long>(key) << 32) | static_cast<uint32_t>(j);
+      best = k64 < best ? k64 : best;
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+      best = other < best ? other : best;
+    }
+    if (lane == 0) sm.warp_min[warp] = best;
+    __syncthreads();
+    if (warp == 0) {
+      best = sm.warp_min[lane];
+      for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+        best = other < best ? other : best;
+      }
+      if (lane == 0) {
+        sm.bcast[0] = static_cast<uint32_t>(best >> 32);
+        sm.bcast[1] = 1u;
+      }
+    }
+    __syncthreads();
+    T = sm.bcast[0];
+    if (T == kProtected) {  // every slot is inside the recent window
+      if (tid == 0) atomicOr(a.err, 2);
+      return;
+    }
+    take_eq = 1;  // the argmin slot is the first slot with key T
+  } else {
+    uint32_t prefix = 0, mask = 0, kth = static_cast<uint32_t>(S);
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      for (int x = tid; x < 256; x += kUpdThreads) sm.hist[x] = 0u;
+      __syncthreads();
+      for (int j = tid; j < M; j += kUpdThreads) {
+        float acc;
+        const uint32_t key = slot_key(a, sc, sp, inc, j, thr, &acc);
+        if ((key & mask) == prefix) atomicAdd(&sm.hist[(key >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (warp == 0) {
+        // lane l owns bins 8l .. 8l+7; find the bin holding the kth key
+        uint32_t c[8], s = 0;
+#pragma unroll
+        for (int x = 0; x < 8; ++x) {
+          c[x] = sm.hist[8 * lane + x];
+          s += c[x];
+        }
+        uint32_t incl = s;
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        uint32_t run = incl - s;
+#pragma unroll
+        for (int x = 0; x < 8; ++x) {
+          if (run < kth && kth <= run + c[x]) {
+            sm.bcast[0] = static_cast<uint32_t>(8 * lane + x);
+            sm.bcast[1] = kth - run;
+          }
+          run += c[x];
+        }
+      }
+      __syncthreads();
+      if (pass == 0) {
+        // protected keys all fall into the top bin; count the candidates
+        const uint32_t n_cand = static_cast<uint32_t>(M) - sm.hist[255];
+        if (n_cand < static_cast<uint32_t>(S)) {
+          if (tid == 0) atomicOr(a.err, 2);
+          return;
+        }
+      }
+      prefix |= sm.bcast[0] << shift;
+      mask |= 255u << shift;
+      kth = sm.bcast[1];
+      __syncthreads();
+    }
+    T = prefix;
+    take_eq = kth;
+  }
+
+  // Sweep in slot order: evicted slots get ranks 0..S-1.
+  uint32_t eq_base = 0, sel_base = 0;
+  for (int base = 0; base < M; base += kUpdThreads) {
+    const int j = base + tid;
+    float acc = 0.f;
+    const uint32_t key = j < M ? slot_key(a, sc, sp, inc, j, thr, &acc) : kProtected;
+    const bool lt = key < T;
+    const bool eq = j < M && key == T;
+    uint32_t eq_tot;
+    const uint32_t eq_rank = eq_base + block_scan_bit(eq, sm.warp_tot, &eq_tot);
+    // (c < S always holds by construction; the guard keeps every access in bounds)
+    const bool sel0 = lt || (eq && eq_rank < take_eq);
+    uint32_t sel_tot;
+    const uint32_t c = sel_base + block_scan_bit(sel0, sm.warp_tot2, &sel_tot);
+    const bool sel = sel0 && c < static_cast<uint32_t>(S);
+    if (j < M) {
+      if (sel) {
+        sc[j] = group_sum(inc + M, M + S, a.qg, static_cast<int>(c));  // the new token's own column
+        sp[j] = a.pos0 + static_cast<int>(c);
+        if (a.evict_idx) a.evict_idx[static_cast<size_t>(grp) * S + c] = j;
+      } else {
+        sc[j] = acc;
+      }
+    }
+    // warp-cooperative K/V copies of this warp's evicted slots
+    uint32_t m = __ballot_sync(0xffffffffu, sel);
+    while (m) {
+      const int src_lane = __ffs(m) - 1;
+      m &= m - 1;
+      const int cc = __shfl_sync(0xffffffffu, static_cast<int>(c), src_lane);
+      const int jj = __shfl_sync(0xffffffffu, j, src_lane);
+      copy_row(a, grp, cc, jj, lane);
+    }
+    eq_base += eq_tot;
+    sel_base += sel_tot;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
+  update_kernel<<<a.B * a.Hkv, kUpdThreads, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace h2o

@@ -1,0 +1,66 @@
+"""Chunk-loop driver for one attention layer with an H2O cache (§3.1, §A.4.1).
+
+The layer state (cache buffers, slot positions, scores) lives in torch tensors
+on the GPU; every step runs the library's two calls on the current stream:
+``h2o_sdpa_chunk`` then ``h2o_update``.  A sequence is a prefill of M tokens
+(attending to an empty cache) followed by chunks of S tokens.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import _binding as lib
+
+
+def chunk_bounds(T: int, M: int, S: int):
+    """[(start, end)]: the prefill [0, min(T, M)) then chunks of S (last one ragged)."""
+    p0 = min(T, M)
+    out = [(0, p0)] if p0 else []
+    p = p0
+    while p < T:
+        out.append((p, min(T, p + S)))
+        p += S
+    return out
+
+
+class H2OLayer:
+    """Device-resident H2O cache state of one layer: M slots per (b, KV head)."""
+
+    def __init__(self, B: int, Hq: int, Hkv: int, d: int, M: int, S: int, W: int,
+                 device="cuda", scale: float = 0.0, keep_evictions: bool = True):
+        self.B, self.Hq, self.Hkv, self.d, self.M, self.S, self.W = B, Hq, Hkv, d, M, S, W
+        self.scale = scale
+        dev = torch.device(device)
+        self.k_cache = torch.zeros((B, Hkv, M, d), dtype=torch.bfloat16, device=dev)
+        self.v_cache = torch.zeros_like(self.k_cache)
+        self.slot_pos = torch.full((B, Hkv, M), -1, dtype=torch.int32, device=dev)
+        self.scores = torch.zeros((B, Hkv, M), dtype=torch.float32, device=dev)
+        self._inc = {}
+        self._evict = {}
+        self.keep_evictions = keep_evictions
+        self.device = dev
+
+    def reset(self, stream=None):
+        """Empty cache for a new sequence (slot positions -1, scores 0)."""
+        lib.h2o_cache_reset(self.slot_pos, self.scores, stream=stream)
+
+    def _buf(self, s: int):
+        if s not in self._inc:
+            self._inc[s] = torch.empty((self.B, self.Hq, self.M + s), dtype=torch.float32,
+                                       device=self.device)
+            self._evict[s] = torch.empty((self.B, self.Hkv, s), dtype=torch.int32,
+                                         device=self.device)
+        return self._inc[s], self._evict[s]
+
+    def step(self, q, k_new, v_new, pos0: int, out=None, stream=None):
+        """One chunk: attend (writes out, score_inc), then update the cache in place.
+
+        Returns (out, score_inc, evict_idx); the last two are reused buffers.
+        """
+        s = q.shape[2]
+        inc, ev = self._buf(s)
+        out, inc = lib.h2o_sdpa_chunk(q, self.k_cache, self.v_cache, k_new, v_new, self.slot_pos,
+                                      pos0, self.scale, out=out, score_inc=inc, stream=stream)
+        lib.h2o_update(self.scores, self.slot_pos, inc, k_new, v_new, self.k_cache, self.v_cache,
+                       pos0, self.W, evict_idx=ev if self.keep_evictions else None, stream=stream)
+        return out, inc, ev

@@ -1,0 +1,93 @@
+"""The C-ABI library builds, loads and exports every declared symbol; host-side
+argument checking returns the documented codes without touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_19920_gb300 import _binding as b
+from paper_2608_19920_gb300 import build as build_mod
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "h2o.h")
+
+OK, NULL, SHAPE, ALIGN, UNSUP, ARG = 0, -1, -2, -3, -4, -6
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build_mod.build()
+    return b.load()
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return set(re.findall(r"H2O_API\s+[\w\s\*]*?\b(h2o_\w+)\s*\(", text))
+
+
+def test_header_declares_the_binding_exports():
+    assert declared_symbols() == set(b.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_symbols():
+        assert hasattr(lib, name), name
+    assert lib.h2o_version() >= 100
+    for code in range(-10, 1):
+        assert lib.h2o_status_string(code)
+
+
+def _dims(B=1, Hq=4, Hkv=2, d=64, S=32, M=256):
+    return b.H2ODims(B, Hq, Hkv, d, S, M)
+
+
+def _sdpa(lib, dims, ptrs=None, pos0=256, scale=0.0):
+    p = ptrs or [0x1000] * 8
+    vp = ctypes.c_void_p
+    return lib.h2o_sdpa_chunk(ctypes.byref(dims) if dims is not None else None, pos0, scale,
+                              *[vp(x) for x in p], None, 0, None)
+
+
+def test_sdpa_argument_checks(lib):
+    assert _sdpa(lib, None) == NULL
+    assert _sdpa(lib, _dims(Hq=5, Hkv=2)) == SHAPE
+    assert _sdpa(lib, _dims(S=0)) == SHAPE
+    assert _sdpa(lib, _dims(M=-1)) == SHAPE
+    assert _sdpa(lib, _dims(d=96)) == UNSUP
+    assert _sdpa(lib, _dims(), ptrs=[0x1000] * 7 + [0]) == NULL
+    assert _sdpa(lib, _dims(), ptrs=[0x1000] * 6 + [0x1004, 0x1000]) == ALIGN
+    assert _sdpa(lib, _dims(), pos0=-1) == ARG
+    assert _sdpa(lib, _dims(), pos0=2 ** 31 - 8) == ARG
+    assert _sdpa(lib, _dims(), scale=float("inf")) == ARG
+    n = ctypes.c_size_t(7)
+    assert lib.h2o_workspace_size(ctypes.byref(_dims()), ctypes.byref(n)) == OK and n.value == 0
+    assert lib.h2o_workspace_size(ctypes.byref(_dims(d=32)), ctypes.byref(n)) == UNSUP
+
+
+def _upd(lib, dims, budget=256, W=32, pos0=256, ptrs=None, evict=None):
+    p = ptrs or [0x1000] * 7
+    vp = ctypes.c_void_p
+    return lib.h2o_update(ctypes.byref(dims), pos0, *[vp(x) for x in p], budget, W,
+                          vp(evict) if evict else None, None)
+
+
+def test_update_argument_checks(lib):
+    assert _upd(lib, _dims(), budget=255) == ARG
+    assert _upd(lib, _dims(), W=-1) == ARG
+    assert _upd(lib, _dims(), W=257) == ARG
+    assert _upd(lib, _dims(S=300)) == SHAPE
+    assert _upd(lib, _dims(), pos0=-3) == ARG
+    assert _upd(lib, _dims(), ptrs=[0x1000] * 6 + [0]) == NULL
+    assert _upd(lib, _dims(), evict=0x1002) == ALIGN
+    assert _upd(lib, _dims(M=0, S=1), budget=0) == SHAPE
+
+
+def test_binding_refuses_to_run_without_the_library(tmp_path):
+    saved = b._lib
+    try:
+        b._lib = None
+        with pytest.raises(RuntimeError, match="not built"):
+            b.load(str(tmp_path / "missing.so"))
+    finally:
+        b._lib = saved

@@ -311,3 +311,17 @@ def test_chunk_bounds():
     assert len(chunk_bounds(1024, 256, 32)) == 1 + 24
     assert chunk_bounds(10, 4, 4) == [(0, 4), (4, 8), (8, 10)]
     assert chunk_bounds(3, 8, 2) == [(0, 3)]
+
+
+def test_row_subset_matches_full_chunk():
+    rng = np.random.default_rng(9)
+    B, Hq, Hkv, M, S, d, pos0 = 1, 4, 2, 20, 9, 8, 50
+    st = _state(rng, B, Hkv, M, d, pos0, n_empty=2)
+    q, kn, vn = _rand_seq(rng, B, Hq, Hkv, S, d)
+    out, inc, lse = sdpa_chunk(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"], pos0)
+    rows = [0, 3, 8]
+    o2, inc2, l2 = sdpa_chunk(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"], pos0,
+                              rows=rows)
+    np.testing.assert_allclose(o2, out[:, :, rows], atol=1e-14)
+    np.testing.assert_allclose(l2, lse[:, :, rows], atol=1e-14)
+    np.testing.assert_allclose(inc2.sum(axis=-1), len(rows), rtol=1e-12)

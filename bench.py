@@ -331,11 +331,11 @@ def run_ours(args, w):
     return 0
 
 
-def time_sdpa_kernel(w, layer, inputs, plan, stream, reps):
+def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
     """Average duration of the steady-state chunk SDPA launch (CUDA events)."""
     import torch
     from paper_2608_19920_gb300 import h2o_sdpa_chunk
-    idx = len(plan) // 2
+    idx = len(plan) // 2 if idx is None else idx
     p, e = plan[idx]
     q, k, v = inputs[idx]
     out = torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=q.device)
@@ -423,13 +423,42 @@ def main():
     ap.add_argument("--traffic", type=float, default=None,
                     help="DRAM bytes per launch of the dominant kernel from an ncu capture")
     ap.add_argument("--ref-budget", type=float, default=20.0)
+    ap.add_argument("--mode", default="step", choices=["step", "kernel"],
+                    help="kernel: only repeat the steady-state chunk SDPA launch (for profiling)")
+    ap.add_argument("--reps", type=int, default=5)
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     w = wl.WORKLOADS[args.workload]
     if args.impl == "reference":
         return run_reference(args, w)
+    if args.mode == "kernel":
+        return run_kernel_only(args, w)
     return run_ours(args, w)
+
+
+def run_kernel_only(args, w, n_fill: int = 8):
+    """Fills the cache with a prefill and ``n_fill`` chunks, then launches the
+    chunk after them ``--reps`` times (a small, fixed launch list for ncu)."""
+    import torch
+    from paper_2608_19920_gb300 import H2OLayer, build as build_mod, h2o_device_errors
+    build_mod.build()
+    dev = torch.device("cuda", 0)
+    plan = step_plan(w)[:n_fill + 2]
+    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev)
+    ins = []
+    for p, e in plan:
+        ins.append(tuple(torch.from_numpy(x).to(torch.bfloat16).to(dev)
+                         for x in wl.batch_tokens(w, p, e)))
+    layer.reset()
+    for (p, e), (q, k, v) in zip(plan[:-1], ins[:-1]):
+        layer.step(q, k, v, p)
+    kern = time_sdpa_kernel(w, layer, ins, plan, torch.cuda.current_stream(), reps=args.reps,
+                            idx=len(plan) - 1)
+    torch.cuda.synchronize()
+    assert h2o_device_errors() == 0
+    print(json.dumps({"mode": "kernel", "workload": w.name, **kern}))
+    return 0
 
 
 if __name__ == "__main__":

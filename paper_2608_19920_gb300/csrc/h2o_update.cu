@@ -15,11 +15,18 @@
 //  3. S = 1 is an argmin over (key, slot).  Otherwise a 4-pass radix select
 //     (8-bit digits, shared-memory histogram) finds the S-th smallest key T and
 //     how many keys equal to T are taken (the lowest slots first).
-//  4. One sweep in slot order, 1024 slots per round, computes with warp ballots
-//     and a block scan the rank c of every evicted slot (the c-th smallest
-//     evicted slot receives token pos0 + c) and writes slot_pos, scores,
-//     evict_idx; each warp then copies the K and V rows of its evicted slots
-//     with 16-byte vector loads and stores.
+//  4. One sweep in slot order computes with block scans the rank c of every
+//     evicted slot (the c-th smallest evicted slot receives token pos0 + c) and
+//     writes slot_pos, scores, evict_idx; whole warps copy the K and V rows of
+//     the evicted slots with 16-byte vector loads and stores.
+//
+// Two variants.  When the keys of one (b, kv head) fit in shared memory and
+// S > 1, a cluster of C CTAs handles the (b, kv head): every CTA computes the
+// keys into shared memory and runs the same deterministic selection, a cluster
+// barrier separates all reads of the old state from the writes, CTA 0 writes
+// scores / slot_pos / evict_idx, and the C CTAs share the row copies.
+// Otherwise one CTA per (b, kv head) recomputes keys from global memory on
+// every pass (S = 1 takes the argmin path).
 #include "h2o_internal.h"
 #include "sm100.cuh"
 
@@ -218,11 +225,196 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
   }
 }
 
+// ----------------------------------------------------- cluster variant --
+constexpr int kCThreads = 512;
+constexpr int kCWarps = kCThreads / 32;
+constexpr int kMaxSmemSlots = 24576;
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// Exclusive prefix sum over the block of one value per thread.
+__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_tot,
+                                                    uint32_t* total) {
+  const int tid = threadIdx.x, w = tid >> 5, l = tid & 31;
+  uint32_t incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (l >= o) incl += y;
+  }
+  if (l == 31) warp_tot[w] = incl;
+  __syncthreads();
+  if (w == 0) {
+    uint32_t x = l < kCWarps ? warp_tot[l] : 0u;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+      if (l >= o) x += y;
+    }
+    if (l < kCWarps) warp_tot[l] = x;
+  }
+  __syncthreads();
+  const uint32_t base = w > 0 ? warp_tot[w - 1] : 0u;
+  *total = warp_tot[kCWarps - 1];
+  __syncthreads();
+  return base + incl - v;
+}
+
+__global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const UpdateArgs a, int C) {
+  extern __shared__ uint32_t dyn[];
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t warp_tot[kCWarps];
+  __shared__ uint32_t bcast[4];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rank = static_cast<int>(cluster_rank());
+  const int grp = blockIdx.x / C;
+  const int b = grp / a.Hkv, h = grp % a.Hkv;
+  const int M = a.M, S = a.S;
+  float* sc = a.scores + static_cast<size_t>(grp) * M;
+  int* sp = a.slot_pos + static_cast<size_t>(grp) * M;
+  const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * a.qg) * (M + S);
+  const int thr = a.pos0 + S - a.W;
+  uint32_t* keys = dyn;                                   // [M]
+  int* elist = reinterpret_cast<int*>(dyn + M);           // [S] evicted slot of rank c
+
+  for (int j = tid; j < M; j += kCThreads) {
+    float acc;
+    keys[j] = slot_key(a, sc, sp, inc, j, thr, &acc);
+  }
+  // Every CTA of the cluster has read the old state before CTA 0 rewrites it.
+  cluster_sync_all();
+
+  // radix select: the S-th smallest key T, and how many keys equal to T are taken
+  uint32_t prefix = 0, mask = 0, kth = static_cast<uint32_t>(S);
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    for (int x = tid; x < 256; x += kCThreads) hist[x] = 0u;
+    __syncthreads();
+    for (int j = tid; j < M; j += kCThreads) {
+      const uint32_t key = keys[j];
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (pass == 0 && static_cast<uint32_t>(M) - hist[255] < static_cast<uint32_t>(S)) {
+      if (tid == 0 && rank == 0) atomicOr(a.err, 2);
+      return;  // uniform over the cluster: every CTA computed the same histogram
+    }
+    if (warp == 0) {
+      uint32_t c[8], s = 0;
+#pragma unroll
+      for (int x = 0; x < 8; ++x) {
+        c[x] = hist[8 * lane + x];
+        s += c[x];
+      }
+      uint32_t incl = s;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      uint32_t run = incl - s;
+#pragma unroll
+      for (int x = 0; x < 8; ++x) {
+        if (run < kth && kth <= run + c[x]) {
+          bcast[0] = static_cast<uint32_t>(8 * lane + x);
+          bcast[1] = kth - run;
+        }
+        run += c[x];
+      }
+    }
+    __syncthreads();
+    prefix |= bcast[0] << shift;
+    mask |= 255u << shift;
+    kth = bcast[1];
+    __syncthreads();
+  }
+  const uint32_t T = prefix, take_eq = kth;
+
+  // ranks in slot order: thread t owns slots [t*R, t*R + R)
+  const int R = (M + kCThreads - 1) / kCThreads;
+  const int j0 = min(M, tid * R), j1 = min(M, j0 + R);
+  uint32_t n_eq = 0;
+  for (int j = j0; j < j1; ++j) n_eq += keys[j] == T;
+  uint32_t tot;
+  uint32_t eq_run = block_excl_scan(n_eq, warp_tot, &tot);
+  uint32_t n_sel = 0;
+  {
+    uint32_t e = eq_run;
+    for (int j = j0; j < j1; ++j) {
+      const uint32_t key = keys[j];
+      const bool eq = key == T;
+      n_sel += key < T || (eq && e < take_eq);
+      e += eq;
+    }
+  }
+  uint32_t c = block_excl_scan(n_sel, warp_tot, &tot);
+  for (int j = j0; j < j1; ++j) {
+    const uint32_t key = keys[j];
+    const bool eq = key == T;
+    const bool sel = (key < T || (eq && eq_run < take_eq)) && c < static_cast<uint32_t>(S);
+    eq_run += eq;
+    if (sel) {
+      elist[c] = j;
+      if (rank == 0) {
+        sc[j] = group_sum(inc + M, M + S, a.qg, static_cast<int>(c));
+        sp[j] = a.pos0 + static_cast<int>(c);
+        if (a.evict_idx) a.evict_idx[static_cast<size_t>(grp) * S + c] = j;
+      }
+      ++c;
+    } else if (rank == 0) {
+      sc[j] = __fadd_rn(sc[j], group_sum(inc, M + S, a.qg, j));
+    }
+  }
+  __syncthreads();
+  // this CTA's share of the K/V row copies: ranks c = rank (mod C)
+  const int n_sel_tot = min(static_cast<int>(tot), S);
+  for (int cc = rank + C * warp; cc < n_sel_tot; cc += C * kCWarps)
+    copy_row(a, grp, cc, elist[cc], lane);
+}
+
 }  // namespace
 
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
-  update_kernel<<<a.B * a.Hkv, kUpdThreads, 0, stream>>>(a);
-  return cudaGetLastError();
+  const bool smem_path = a.S > 1 && a.M <= kMaxSmemSlots;
+  if (!smem_path) {
+    update_kernel<<<a.B * a.Hkv, kUpdThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+  }
+  const size_t smem = (static_cast<size_t>(a.M) + a.S) * sizeof(uint32_t);
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 64 && !configured[dev]) {
+    e = cudaFuncSetAttribute(update_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>((kMaxSmemSlots * 2) * sizeof(uint32_t)));
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  int C = (a.S + 63) / 64;
+  C = C < 1 ? 1 : (C > 8 ? 8 : C);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(a.B * a.Hkv * C));
+  cfg.blockDim = dim3(kCThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(C);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, update_cluster_kernel, a, C);
 }
 
 }  // namespace h2o

@@ -16,15 +16,19 @@
 //    columns into score_inc and accumulates P V.  Because lambda is final in
 //    pass 2, the P V accumulator never needs rescaling.
 //  * Warp roles: warp 0 issues TMA loads (Q once, then K and V tiles through a
-//    2-stage ring), warp 1 issues tcgen05 MMAs (accumulators in TMEM: two S
-//    buffers and the O accumulator), warps 4-11 are two softmax warpgroups;
-//    warpgroup w owns key columns 64w..64w+63 of every S tile and TMEM lanes =
-//    query rows.  P is written back to TMEM as bf16 over its own S columns and
-//    consumed by the P V MMA directly from TMEM.
-//  * Column sums use the fp32 P (not the bf16 copy fed to the MMA): a warp
-//    reduce-scatter leaves two column sums per lane, the four warps of a
+//    ring of shared-memory slots), warp 1 issues tcgen05 MMAs (accumulators in
+//    TMEM: two S buffers and the O accumulator), warps 2-17 form four softmax
+//    warpgroups; warpgroup w owns key columns 32w..32w+31 of every S tile.
+//    Four warps per SM sub-partition overlap the exp-bound and shuffle-bound
+//    phases of different tiles.  P is written back to TMEM as bf16 over its own
+//    S columns and consumed by the P V MMA directly from TMEM.
+//  * Column sums use the fp32 P (not the bf16 copy fed to the MMA).  Pass 2
+//    reads S in TMEM's 16x256b layout, where a thread holds 4 rows x 8
+//    columns: it adds its 4 rows, a 3-step warp reduce-scatter leaves one
+//    column sum (over the warp's 32 rows) per lane, the four warps of a
 //    warpgroup combine through shared memory, and one red.global.add per
 //    column and query head goes to score_inc (zeroed by the host call).
+//    Pass 1 keeps one row per thread (32x32b layout) for the row statistics.
 //  * Key tiles are classified up front from slot_pos: tiles no row of the CTA
 //    can see are skipped, tiles every row sees need no mask, the rest are
 //    masked per element.
@@ -38,26 +42,33 @@
 namespace h2o {
 namespace {
 
-constexpr int kStages = 2;
-constexpr int kThreads = 384;
+constexpr int kNumWG = 4;                       // softmax warpgroups
+constexpr int kColsPerWG = kTileN / kNumWG;     // 32 key columns each
+constexpr int kFirstSoftmaxWarp = 2;
+constexpr int kSoftmaxWarps = 4 * kNumWG;
+constexpr int kThreads = 32 * (kFirstSoftmaxWarp + kSoftmaxWarps);  // 576
 constexpr uint16_t kTileChunk = 0x8000;
 constexpr uint16_t kTilePartial = 0x4000;
 constexpr uint16_t kTileIdxMask = 0x3FFF;
 constexpr uint8_t kClsSkip = 0, kClsFull = 1, kClsPartial = 2;
 
+// K and V tiles share one ring of shared-memory slots, loaded in exactly the
+// order the MMA issuer consumes them (pass 1: K0..Kn-1; pass 2: K0, K1, V0,
+// K2, V1, ..., Vn-1), so a slot is released by the MMA that read it.
+template <int D>
+__host__ __device__ constexpr int ring_slots() { return D == 128 ? 5 : 10; }
+
 template <int D>
 struct __align__(1024) SdpaSmem {
   static constexpr int kPanels = D / 64;
   uint8_t q[kPanels][kTileM * 128];
-  uint8_t k[kStages][kPanels][kTileN * 128];
-  uint8_t v[kStages][kPanels][kTileN * 128];
-  float colsum[2][2][4][64];  // [buffer][warpgroup][warp][column]
-  float rowstat[2][kTileM][2];
+  uint8_t kv[ring_slots<D>()][kPanels][kTileN * 128];
+  float colsum[2][kNumWG][4][kColsPerWG];  // [buffer][warpgroup][warp][column]
+  float rowstat[kNumWG][kTileM][2];
   uint64_t bar_q;
-  uint64_t bar_kfull[kStages], bar_kempty[kStages];
-  uint64_t bar_vfull[kStages], bar_vempty[kStages];
+  uint64_t bar_full[ring_slots<D>()], bar_empty[ring_slots<D>()];
   uint64_t bar_sfull[2], bar_pfull[2], bar_pvdone[2];
-  uint64_t bar_cs[2][2];
+  uint64_t bar_cs[2][kNumWG];
   uint64_t bar_rowstat, bar_ofull, bar_drain;
   uint32_t taddr;
   int abort_flag;
@@ -66,10 +77,11 @@ struct __align__(1024) SdpaSmem {
   uint16_t tiles[kMaxKeyTiles];
 };
 
-// Butterfly reduce-scatter of 64 values over the 32 lanes of a warp: on
-// return v[0], v[1] hold the warp-wide sums of columns 2*lane, 2*lane+1.
+// One butterfly reduce-scatter step over lane bit O: of the L values a lane
+// holds, it keeps the upper half if its bit O is set (the lower half
+// otherwise) and adds the partner lane's copy of that half.
 template <int L, int O>
-__device__ __forceinline__ void rs_step(float (&v)[64], uint32_t lane) {
+__device__ __forceinline__ void rs_step(float (&v)[8], uint32_t lane) {
   const bool up = (lane & O) != 0;
 #pragma unroll
   for (int k = 0; k < L / 2; ++k) {
@@ -77,14 +89,6 @@ __device__ __forceinline__ void rs_step(float (&v)[64], uint32_t lane) {
     const float keep = up ? v[k + L / 2] : v[k];
     v[k] = keep + __shfl_xor_sync(0xffffffffu, send, O);
   }
-}
-
-__device__ __forceinline__ void reduce_scatter64(float (&v)[64], uint32_t lane) {
-  rs_step<64, 16>(v, lane);
-  rs_step<32, 8>(v, lane);
-  rs_step<16, 4>(v, lane);
-  rs_step<8, 2>(v, lane);
-  rs_step<4, 1>(v, lane);
 }
 
 template <int D>
@@ -117,20 +121,17 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
 
   if (tid == 0) {
     bar_init(&sm.bar_q, 1);
-    for (int s = 0; s < kStages; ++s) {
-      bar_init(&sm.bar_kfull[s], 1);
-      bar_init(&sm.bar_kempty[s], 1);
-      bar_init(&sm.bar_vfull[s], 1);
-      bar_init(&sm.bar_vempty[s], 1);
+    for (int s = 0; s < ring_slots<D>(); ++s) {
+      bar_init(&sm.bar_full[s], 1);
+      bar_init(&sm.bar_empty[s], 1);
     }
     for (int x = 0; x < 2; ++x) {
       bar_init(&sm.bar_sfull[x], 1);
-      bar_init(&sm.bar_pfull[x], 8);
+      bar_init(&sm.bar_pfull[x], kSoftmaxWarps);
       bar_init(&sm.bar_pvdone[x], 1);
-      bar_init(&sm.bar_cs[x][0], 4);
-      bar_init(&sm.bar_cs[x][1], 4);
+      for (int w = 0; w < kNumWG; ++w) bar_init(&sm.bar_cs[x][w], 4);
     }
-    bar_init(&sm.bar_rowstat, 8);
+    bar_init(&sm.bar_rowstat, kSoftmaxWarps);
     bar_init(&sm.bar_ofull, 1);
     bar_init(&sm.bar_drain, 1);
     sm.abort_flag = 0;
@@ -149,12 +150,12 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     fence_proxy_async_smem();
   }
   // Classify key tiles against this CTA's rows.
-  if (warp >= 4) {
-    const int sw = warp - 4;
+  if (warp >= kFirstSoftmaxWarp) {
+    const int sw = warp - kFirstSoftmaxWarp;
     const int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
     const int lim_any = a.pos0 + i_hi;
     const int lim_all = a.pos0 + i_lo;
-    for (int ct = sw; ct < a.n_cache_tiles; ct += 8) {
+    for (int ct = sw; ct < a.n_cache_tiles; ct += kSoftmaxWarps) {
       bool any = false, all = true;
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
@@ -167,7 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       all = __all_sync(0xffffffffu, all);
       if (lane == 0) sm.cls[ct] = any ? (all ? kClsFull : kClsPartial) : kClsSkip;
     }
-    for (int c = sw; c < a.n_chunk_tiles; c += 8) {
+    for (int c = sw; c < a.n_chunk_tiles; c += kSoftmaxWarps) {
       const int c0 = c * kTileN;
       uint8_t cl = kClsPartial;
       if (c0 > i_hi) cl = kClsSkip;
@@ -176,7 +177,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     }
   }
   __syncthreads();
-  if (warp == 4) {
+  if (warp == kFirstSoftmaxWarp) {
     const int total = a.n_cache_tiles + a.n_chunk_tiles;
     int n = 0;
     for (int base = 0; base < total; base += 32) {
@@ -216,39 +217,35 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       }
       bar_expect_tx(&sm.bar_q, P * 128 * a.rows_box * a.heads_box);
       for (int p = 0; p < P; ++p) tma_load_4d(sm.q[p], &a.tm_q, &sm.bar_q, 64 * p, i_lo, g_first, grp);
-      int nk = 0, nv = 0;
-      for (int n = 0; n < 2 * n_t; ++n) {
-        const bool pass2 = n >= n_t;
-        const int t = pass2 ? n - n_t : n;
+      constexpr int R = ring_slots<D>();
+      int L = 0;  // loads issued so far; slot L % R
+      auto load = [&](bool is_v, int t) -> bool {
         const uint16_t e = sm.tiles[t];
         const bool chunk = (e & kTileChunk) != 0;
         const int row0 = (e & kTileIdxMask) * kTileN;
-        const CUtensorMap* mk = chunk ? &a.tm_kn : &a.tm_kc;
-        const CUtensorMap* mv = chunk ? &a.tm_vn : &a.tm_vc;
-        const int s = n % kStages;
-        if (n >= kStages &&
-            !wait_bar(&sm.bar_kempty[s], ((n / kStages) - 1) & 1, abort_flag, kWaitLimitNs))
-          break;
-        bar_expect_tx(&sm.bar_kfull[s], P * kTileN * 128);
-        for (int p = 0; p < P; ++p) tma_load_3d(sm.k[s][p], mk, &sm.bar_kfull[s], 64 * p, row0, grp);
-        ++nk;
-        if (pass2) {
-          const int vs = t % kStages;
-          if (t >= kStages &&
-              !wait_bar(&sm.bar_vempty[vs], ((t / kStages) - 1) & 1, abort_flag, kWaitLimitNs))
-            break;
-          bar_expect_tx(&sm.bar_vfull[vs], P * kTileN * 128);
-          for (int p = 0; p < P; ++p) tma_load_3d(sm.v[vs][p], mv, &sm.bar_vfull[vs], 64 * p, row0, grp);
-          ++nv;
-        }
+        const CUtensorMap* m =
+            is_v ? (chunk ? &a.tm_vn : &a.tm_vc) : (chunk ? &a.tm_kn : &a.tm_kc);
+        const int s = L % R;
+        if (L >= R && !wait_bar(&sm.bar_empty[s], ((L / R) - 1) & 1, abort_flag, kWaitLimitNs))
+          return false;
+        bar_expect_tx(&sm.bar_full[s], P * kTileN * 128);
+        for (int p = 0; p < P; ++p) tma_load_3d(sm.kv[s][p], m, &sm.bar_full[s], 64 * p, row0, grp);
+        ++L;
+        return true;
+      };
+      bool ok = true;
+      for (int t = 0; ok && t < n_t; ++t) ok = load(false, t);
+      if (ok) ok = load(false, 0);
+      for (int t = 1; ok && t < n_t; ++t) {
+        ok = load(false, t);
+        if (ok) ok = load(true, t - 1);
       }
+      if (ok) ok = load(true, n_t - 1);
       if (*abort_flag) {
         // Let copies still in flight land before the CTA's shared memory goes away.
         volatile int never = 0;
-        for (int x = max(0, nk - kStages); x < nk; ++x)
-          wait_bar(&sm.bar_kfull[x % kStages], (x / kStages) & 1, &never, 100000000ull);
-        for (int x = max(0, nv - kStages); x < nv; ++x)
-          wait_bar(&sm.bar_vfull[x % kStages], (x / kStages) & 1, &never, 100000000ull);
+        for (int x = max(0, L - R); x < L; ++x)
+          wait_bar(&sm.bar_full[x % R], (x / R) & 1, &never, 100000000ull);
       }
     }
   } else if (warp == 1) {
@@ -256,22 +253,43 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     if (lane == 0 && n_t > 0) {
       constexpr uint32_t kIdescQK = idesc_bf16_f32(kTileM, kTileN, false);
       constexpr uint32_t kIdescPV = idesc_bf16_f32(kTileM, D, true);
+      // Descriptors are built once; per MMA only the 14-bit start-address
+      // field advances, by compile-time immediates (bytes >> 4): a K-step of
+      // 16 bf16 is 32 B inside a 128-B swizzle row, a 64-column panel is
+      // 16 KB, a ring slot is P panels, 16 rows of V are 2 KB.
+      constexpr uint32_t kPanel = (kTileN * 128) >> 4;
+      constexpr uint32_t kSlot = P * kPanel;
+      const uint64_t q_desc = sdesc_sw128(smem_addr(sm.q[0]), 16, 1024);
+      const uint64_t k_desc0 = sdesc_sw128(smem_addr(sm.kv[0][0]), 16, 1024);
+      const uint64_t v_desc0 = sdesc_sw128(smem_addr(sm.kv[0][0]), kTileN * 128, 1024);
       bool ok = wait_bar(&sm.bar_q, 0, abort_flag, kWaitLimitNs);
       uint32_t pv_phase[2] = {0u, 0u};
+      constexpr int R = ring_slots<D>();
+      int L = 0;  // ring slots consumed so far (same order as the producer's loads)
+      auto acquire = [&]() -> int {
+        const int s = L % R;
+        return wait_bar(&sm.bar_full[s], (L / R) & 1, abort_flag, kWaitLimitNs) ? s : -1;
+      };
+      auto release = [&](int s) {
+        mma_commit(&sm.bar_empty[s]);
+        ++L;
+      };
       auto issue_pv = [&](int t) -> bool {
         const int n = n_t + t;
         const int buf = n & 1;
         if (!wait_bar(&sm.bar_pfull[buf], (n >> 1) & 1, abort_flag, kWaitLimitNs)) return false;
-        const int vs = t % kStages;
-        if (!wait_bar(&sm.bar_vfull[vs], (t / kStages) & 1, abort_flag, kWaitLimitNs)) return false;
+        const int vs = acquire();
+        if (vs < 0) return false;
         tc_fence_after_sync();
+        const uint64_t vd = v_desc0 + static_cast<uint64_t>(vs) * kSlot;
+        const uint32_t a_base = tS + buf * 128;
+        const uint32_t acc0 = t > 0 ? 1u : 0u;
+        // keys 16kk..16kk+15 were written as bf16 pairs by warpgroup kk/2
 #pragma unroll
-        for (int kk = 0; kk < kTileN / 16; ++kk) {
-          const uint32_t a_tmem = tS + buf * 128 + 64 * (kk / 4) + 8 * (kk % 4);
-          const uint64_t bd = sdesc_sw128(smem_addr(sm.v[vs][0]) + 2048 * kk, kTileN * 128, 1024);
-          mma_ts(tO, a_tmem, bd, kIdescPV, (t > 0 || kk > 0) ? 1u : 0u);
-        }
-        mma_commit(&sm.bar_vempty[vs]);
+        for (int kk = 0; kk < kTileN / 16; ++kk)
+          mma_ts(tO, a_base + kColsPerWG * (kk / 2) + 8 * (kk % 2), vd + 128 * kk, kIdescPV,
+                 kk > 0 ? 1u : acc0);
+        release(vs);
         mma_commit(&sm.bar_pvdone[buf]);
         return true;
       };
@@ -288,20 +306,21 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           }
           if (!ok) break;
         }
-        const int s = n % kStages;
-        if (!wait_bar(&sm.bar_kfull[s], (n / kStages) & 1, abort_flag, kWaitLimitNs)) {
+        const int s = acquire();
+        if (s < 0) {
           ok = false;
           break;
         }
         tc_fence_after_sync();
+        const uint64_t kd = k_desc0 + static_cast<uint64_t>(s) * kSlot;
+        const uint32_t d_tmem = tS + buf * 128;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(smem_addr(sm.q[kk / 4]) + 32 * (kk % 4), 16, 1024);
-          const uint64_t bd = sdesc_sw128(smem_addr(sm.k[s][kk / 4]) + 32 * (kk % 4), 16, 1024);
-          mma_ss(tS + buf * 128, ad, bd, kIdescQK, kk > 0 ? 1u : 0u);
+          const uint32_t off = kPanel * (kk / 4) + 2 * (kk % 4);
+          mma_ss(d_tmem, q_desc + off, kd + off, kIdescQK, kk > 0 ? 1u : 0u);
         }
         mma_commit(&sm.bar_sfull[buf]);
-        mma_commit(&sm.bar_kempty[s]);
+        release(s);
         if (n >= n_t) {
           if (pending_pv >= 0 && !issue_pv(pending_pv)) {
             ok = false;
@@ -317,29 +336,44 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       volatile int never = 0;
       wait_bar(&sm.bar_drain, 0, &never, kWaitLimitNs);
     }
-  } else if (warp >= 4) {
+  } else {
     // ------------------------------------------- softmax / column sums --
-    const int wg = (warp - 4) >> 2;  // key columns 64*wg .. 64*wg + 63 of each tile
-    const int q4 = warp & 3;         // TMEM lane quarter
+    const int sw = warp - kFirstSoftmaxWarp;
+    const int wg = sw >> 2;          // key columns 32*wg .. 32*wg + 31 of each tile
+    const int q4 = warp & 3;         // TMEM lane quarter (hardware: warp id % 4)
     const int row = q4 * 32 + static_cast<int>(lane);
+    // tile row -> (head within the group, chunk row i); false for padding rows
+    auto row_info = [&](int r, int& gg, int& ii) -> bool {
+      if (a.tiles_per_head > 0) {
+        gg = g_first;
+        ii = i_lo + r;
+        return ii < a.S;
+      }
+      gg = g_first + r / a.rows_box;
+      ii = r % a.rows_box;
+      return r < rows_used && ii < a.S && gg < a.qg;
+    };
     int g, i;
-    bool valid;
-    if (a.tiles_per_head > 0) {
-      g = g_first;
-      i = i_lo + row;
-      valid = i < a.S;
-    } else {
-      g = g_first + row / a.rows_box;
-      i = row % a.rows_box;
-      valid = row < rows_used && i < a.S && g < a.qg;
-    }
+    const bool valid = row_info(row, g, i);
     const int qpos = a.pos0 + i;
     const int hq = hkv * a.qg + g;
+    // Pass 2 reads S in the 16x256b layout: this thread then holds rows
+    // 32 q4 + lane/4 + 8x (x = 0..3) and columns 8k + 2(lane%4) + {0,1}.
+    int i4[4];
+    bool v4[4];
+#pragma unroll
+    for (int x = 0; x < 4; ++x) {
+      int gg;
+      v4[x] = row_info(q4 * 32 + static_cast<int>(lane >> 2) + 8 * x, gg, i4[x]);
+    }
+    // After the column reduce-scatter this lane holds column cl of the 32.
+    const int cl = 8 * static_cast<int>((lane >> 3) & 3) + 2 * static_cast<int>(lane & 3) +
+                   static_cast<int>((lane >> 2) & 1);
     const uint32_t lane_addr = static_cast<uint32_t>(q4 * 32) << 16;
     const float sl2 = a.scale_log2;
     const int* sp_base = a.slot_pos + static_cast<size_t>(grp) * a.M;
     float* inc_base = a.score_inc + static_cast<size_t>(b * a.Hq + hkv * a.qg) * NK;
-    // head (within the group) of each warp of this warpgroup; -1 = no valid rows
+    // head (within the group) of each lane quarter's rows; -1 = no valid rows
     int warp_head[4];
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
@@ -348,14 +382,15 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       else gw = (w * 32 < rows_used) ? g_first + (w * 32) / a.rows_box : -1;
       warp_head[w] = (gw >= 0 && gw < a.qg) ? gw : -1;
     }
-    float m_run = -INFINITY, l_run = 0.f, lam2 = INFINITY;
+    float m_run = -INFINITY, l_run = 0.f;
+    float lam4[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
     bool ok = true;
     for (int n = 0; n < 2 * n_t; ++n) {
       const int buf = n & 1;
       const bool pass2 = n >= n_t;
       const int t = pass2 ? n - n_t : n;
       if (n == n_t) {
-        // combine the two warpgroups' halves of every row (§A.6.1 merge)
+        // combine the warpgroups' parts of every row (§A.6.1 merge)
         sm.rowstat[wg][row][0] = m_run;
         sm.rowstat[wg][row][1] = l_run;
         __syncwarp();
@@ -364,54 +399,45 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           ok = false;
           break;
         }
-        const float m0 = sm.rowstat[0][row][0], l0 = sm.rowstat[0][row][1];
-        const float m1 = sm.rowstat[1][row][0], l1 = sm.rowstat[1][row][1];
-        const float mm = fmaxf(m0, m1);
-        const float l = l0 * fast_exp2(m0 - mm) + l1 * fast_exp2(m1 - mm);
-        lam2 = (valid && mm > -INFINITY) ? mm + fast_log2(l) : INFINITY;
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+          const int r = q4 * 32 + static_cast<int>(lane >> 2) + 8 * x;
+          float mm = -INFINITY;
+#pragma unroll
+          for (int w = 0; w < kNumWG; ++w) mm = fmaxf(mm, sm.rowstat[w][r][0]);
+          float l = 0.f;
+#pragma unroll
+          for (int w = 0; w < kNumWG; ++w)
+            l += sm.rowstat[w][r][1] * fast_exp2(sm.rowstat[w][r][0] - mm);
+          lam4[x] = (v4[x] && mm > -INFINITY) ? mm + fast_log2(l) : INFINITY;
+        }
       }
       if (!wait_bar(&sm.bar_sfull[buf], (n >> 1) & 1, abort_flag, kWaitLimitNs)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
-      float v[64];
-      {
-        uint32_t r[32];
-        tmem_ld32(tS + lane_addr + buf * 128 + wg * 64, r);
-#pragma unroll
-        for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
-        tmem_ld32(tS + lane_addr + buf * 128 + wg * 64 + 32, r);
-#pragma unroll
-        for (int k = 0; k < 32; ++k) v[32 + k] = __uint_as_float(r[k]);
-      }
       const uint16_t e = sm.tiles[t];
       const bool chunk = (e & kTileChunk) != 0;
       const bool partial = (e & kTilePartial) != 0;
-      const int col0 = (e & kTileIdxMask) * kTileN + wg * 64;
-      uint64_t vis_lo = ~0ull;  // bit k: column col0 + k visible to this row
-      if (partial) {
-        vis_lo = 0ull;
-        if (chunk) {
-#pragma unroll
-          for (int k = 0; k < 64; ++k) {
-            const int c = col0 + k;
-            if (c <= i && c < a.S) vis_lo |= 1ull << k;
-          }
-        } else {
-          for (int k = 0; k < 64; ++k) {
-            const int j = col0 + k;
-            const int pos = j < a.M ? __ldg(sp_base + j) : -1;
-            if (pos >= 0 && pos <= qpos) vis_lo |= 1ull << k;
-          }
-        }
-      }
+      const int col0 = (e & kTileIdxMask) * kTileN + wg * kColsPerWG;
+      const uint32_t s_addr = tS + lane_addr + buf * 128 + wg * kColsPerWG;
       if (!pass2) {
-        // pass 1: running max and sum of exp2 (log2 domain)
+        // pass 1 (one row per thread): running max and sum of exp2, log2 domain
+        float v[32];
+        {
+          uint32_t r[32];
+          tmem_ld32(s_addr, r);
+#pragma unroll
+          for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
+        }
+        tc_fence_before_sync();
+        __syncwarp();
+        if (lane == 0) bar_arrive(&sm.bar_pfull[buf]);  // S buffer may be overwritten
         if (!partial) {
           float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
 #pragma unroll
-          for (int k = 4; k < 64; k += 4) {
+          for (int k = 4; k < 32; k += 4) {
             mx0 = fmaxf(mx0, v[k]);
             mx1 = fmaxf(mx1, v[k + 1]);
             mx2 = fmaxf(mx2, v[k + 2]);
@@ -420,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           const float m_new = fmaxf(m_run, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2);
           float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-          for (int k = 0; k < 64; k += 4) {
+          for (int k = 0; k < 32; k += 4) {
             s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
             s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
             s2 += fast_exp2(fmaf(v[k + 2], sl2, -m_new));
@@ -429,53 +455,116 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           l_run = l_run * fast_exp2(m_run - m_new) + ((s0 + s1) + (s2 + s3));
           m_run = m_new;
         } else {
+          uint32_t vis = 0u;  // bit k: column col0 + k visible to this row
+          if (chunk) {
+#pragma unroll
+            for (int k = 0; k < 32; ++k)
+              if (col0 + k <= i && col0 + k < a.S) vis |= 1u << k;
+          } else {
+            for (int k = 0; k < 32; ++k) {
+              const int j = col0 + k;
+              const int pos = j < a.M ? __ldg(sp_base + j) : -1;
+              if (pos >= 0 && pos <= qpos) vis |= 1u << k;
+            }
+          }
           float mx = -INFINITY;
 #pragma unroll
-          for (int k = 0; k < 64; ++k)
-            if ((vis_lo >> k) & 1ull) mx = fmaxf(mx, v[k] * sl2);
+          for (int k = 0; k < 32; ++k)
+            if ((vis >> k) & 1u) mx = fmaxf(mx, v[k] * sl2);
           const float m_new = fmaxf(m_run, mx);
           if (m_new > -INFINITY) {
             float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-            for (int k = 0; k < 64; k += 2) {
-              if ((vis_lo >> k) & 1ull) s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
-              if ((vis_lo >> (k + 1)) & 1ull) s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
+            for (int k = 0; k < 32; k += 2) {
+              if ((vis >> k) & 1u) s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
+              if ((vis >> (k + 1)) & 1u) s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
             }
             l_run = l_run * fast_exp2(m_run - m_new) + (s0 + s1);
             m_run = m_new;
           }
         }
-        tc_fence_before_sync();
-        __syncwarp();
-        if (lane == 0) bar_arrive(&sm.bar_pfull[buf]);
       } else {
-        // pass 2: P in fp32, bf16 copy to TMEM for the P V MMA
+        // pass 2 (16x256b layout): P in fp32, bf16 copy back to TMEM for P V
+        float pa[16], pb[16];  // rows lane/4 + {0, 8} and + {16, 24}
+        {
+          uint32_t r[16];
+          tmem_ld_16x256b_x4(s_addr, r);
 #pragma unroll
-        for (int k = 0; k < 64; ++k) {
-          const float p = fast_exp2(fmaf(v[k], sl2, -lam2));
-          v[k] = ((vis_lo >> k) & 1ull) ? p : 0.f;
+          for (int k = 0; k < 16; ++k) pa[k] = __uint_as_float(r[k]);
+          tmem_ld_16x256b_x4(s_addr + (16u << 16), r);
+#pragma unroll
+          for (int k = 0; k < 16; ++k) pb[k] = __uint_as_float(r[k]);
+        }
+        if (!partial) {
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            pa[k] = fast_exp2(fmaf(pa[k], sl2, -lam4[(k >> 1) & 1]));
+            pb[k] = fast_exp2(fmaf(pb[k], sl2, -lam4[2 + ((k >> 1) & 1)]));
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+#pragma unroll
+            for (int ee = 0; ee < 2; ++ee) {
+              const int c = col0 + 8 * k + 2 * static_cast<int>(lane & 3) + ee;
+              bool vis[4];
+              if (chunk) {
+#pragma unroll
+                for (int x = 0; x < 4; ++x) vis[x] = c <= i4[x] && c < a.S;
+              } else {
+                const int pos = c < a.M ? __ldg(sp_base + c) : -1;
+#pragma unroll
+                for (int x = 0; x < 4; ++x) vis[x] = pos >= 0 && pos <= a.pos0 + i4[x];
+              }
+              const int ia = 4 * k + ee, ib = 4 * k + 2 + ee;
+              pa[ia] = vis[0] ? fast_exp2(fmaf(pa[ia], sl2, -lam4[0])) : 0.f;
+              pa[ib] = vis[1] ? fast_exp2(fmaf(pa[ib], sl2, -lam4[1])) : 0.f;
+              pb[ia] = vis[2] ? fast_exp2(fmaf(pb[ia], sl2, -lam4[2])) : 0.f;
+              pb[ib] = vis[3] ? fast_exp2(fmaf(pb[ib], sl2, -lam4[3])) : 0.f;
+            }
+          }
         }
         {
-          uint32_t pk[32];
+          uint32_t pk[8];
 #pragma unroll
-          for (int x = 0; x < 32; ++x) pk[x] = pack_bf16x2(v[2 * x], v[2 * x + 1]);
-          tmem_st32(tS + lane_addr + buf * 128 + wg * 64, pk);
+          for (int k = 0; k < 4; ++k) {
+            pk[2 * k] = pack_bf16x2(pa[4 * k], pa[4 * k + 1]);
+            pk[2 * k + 1] = pack_bf16x2(pa[4 * k + 2], pa[4 * k + 3]);
+          }
+          tmem_st_16x128b_x4(s_addr, pk);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            pk[2 * k] = pack_bf16x2(pb[4 * k], pb[4 * k + 1]);
+            pk[2 * k + 1] = pack_bf16x2(pb[4 * k + 2], pb[4 * k + 3]);
+          }
+          tmem_st_16x128b_x4(s_addr + (16u << 16), pk);
         }
         tc_fence_before_sync();
         __syncwarp();
         if (lane == 0) bar_arrive(&sm.bar_pfull[buf]);
-        // column sums of P over this warp's 32 rows, then over the warpgroup
-        reduce_scatter64(v, lane);
+        // column sums: 4 rows in-thread, then a reduce-scatter over lane bits
+        // 4, 3, 2 leaves one column (summed over the warp's 32 rows) per lane
+        float v[8];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          v[2 * k] = (pa[4 * k] + pa[4 * k + 2]) + (pb[4 * k] + pb[4 * k + 2]);
+          v[2 * k + 1] = (pa[4 * k + 1] + pa[4 * k + 3]) + (pb[4 * k + 1] + pb[4 * k + 3]);
+        }
+        rs_step<8, 16>(v, lane);
+        rs_step<4, 8>(v, lane);
+        rs_step<2, 4>(v, lane);
         const int cb = t & 1;
-        *reinterpret_cast<float2*>(&sm.colsum[cb][wg][q4][2 * lane]) = make_float2(v[0], v[1]);
+        sm.colsum[cb][wg][q4][cl] = v[0];
         __syncwarp();
         if (lane == 0) bar_arrive(&sm.bar_cs[cb][wg]);
         if (!wait_bar(&sm.bar_cs[cb][wg], (t >> 1) & 1, abort_flag, kWaitLimitNs)) {
           ok = false;
           break;
         }
-        if (q4 < 2) {
-          const int c = q4 * 32 + static_cast<int>(lane);
+        // one warp of the warpgroup (a different one every tile) adds the
+        // four quarters' partial sums per query head and issues the reductions
+        if (q4 == (t & 3)) {
+          const int c = static_cast<int>(lane);
           const int col = col0 + c;
           if (chunk ? col < a.S : col < a.M) {
             float* dst = inc_base + (chunk ? a.M + col : col);
@@ -497,22 +586,27 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     // ------------------------------------------------------------ epilogue --
     if (ok && n_t > 0 && wait_bar(&sm.bar_ofull, 0, abort_flag, kWaitLimitNs)) {
       tc_fence_after_sync();
-      constexpr int kHalf = D / 2;
-      uint16_t* dst = a.out + (static_cast<size_t>(b * a.Hq + hq) * a.S + i) * D + wg * kHalf;
-#pragma unroll
-      for (int c = 0; c < kHalf; c += 32) {
+      constexpr int kPart = D / kNumWG;  // O columns per warpgroup: 32 or 16
+      uint16_t* dst = a.out + (static_cast<size_t>(b * a.Hq + hq) * a.S + i) * D + wg * kPart;
+      uint32_t pk[kPart / 2];
+      if constexpr (kPart == 32) {
         uint32_t r[32];
-        tmem_ld32(tO + lane_addr + wg * kHalf + c, r);
-        uint32_t pk[16];
+        tmem_ld32(tO + lane_addr + wg * kPart, r);
 #pragma unroll
         for (int x = 0; x < 16; ++x)
           pk[x] = pack_bf16x2(__uint_as_float(r[2 * x]), __uint_as_float(r[2 * x + 1]));
-        if (valid) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+      } else {
+        uint32_t r[16];
+        tmem_ld16(tO + lane_addr + wg * kPart, r);
 #pragma unroll
-          for (int x = 0; x < 4; ++x)
-            d4[x] = make_uint4(pk[4 * x], pk[4 * x + 1], pk[4 * x + 2], pk[4 * x + 3]);
-        }
+        for (int x = 0; x < 8; ++x)
+          pk[x] = pack_bf16x2(__uint_as_float(r[2 * x]), __uint_as_float(r[2 * x + 1]));
+      }
+      if (valid) {
+        uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+        for (int x = 0; x < kPart / 8; ++x)
+          d4[x] = make_uint4(pk[4 * x], pk[4 * x + 1], pk[4 * x + 2], pk[4 * x + 3]);
       }
     }
   }

@@ -195,14 +195,17 @@ int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, co
                             static_cast<uint64_t>(qg), G};
     const uint32_t bq[4] = {64, static_cast<uint32_t>(a.rows_box), static_cast<uint32_t>(a.heads_box), 1};
     if ((st = encode(&a.tm_q, q, 4, dq, bq)) != H2O_OK) return st;
+    // d = 128 runs on CTA pairs: each CTA loads 64 keys of a K tile and 64
+    // columns of a V tile; d = 64 loads whole 128-key tiles.
     const uint64_t dn[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S), G};
-    const uint32_t bk[3] = {64, kTileN, 1};
+    const uint32_t bk[3] = {64, D.d == 128 ? kTileN / 2u : kTileN, 1};
+    const uint32_t bv[3] = {64, kTileN, 1};
     if ((st = encode(&a.tm_kn, k_new, 3, dn, bk)) != H2O_OK) return st;
-    if ((st = encode(&a.tm_vn, v_new, 3, dn, bk)) != H2O_OK) return st;
+    if ((st = encode(&a.tm_vn, v_new, 3, dn, bv)) != H2O_OK) return st;
     if (D.M > 0) {
       const uint64_t dc[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.M), G};
       if ((st = encode(&a.tm_kc, k_cache, 3, dc, bk)) != H2O_OK) return st;
-      if ((st = encode(&a.tm_vc, v_cache, 3, dc, bk)) != H2O_OK) return st;
+      if ((st = encode(&a.tm_vc, v_cache, 3, dc, bv)) != H2O_OK) return st;
     }
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -15,10 +15,10 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded waits: 2 s
 
 struct SdpaArgs {
   CUtensorMap tm_q;        // 4D {d, S, q_g, B*Hkv}, box {64, rows_box, heads_box, 1}
-  CUtensorMap tm_kc;       // 3D {d, M, B*Hkv}, box {64, 128, 1}
-  CUtensorMap tm_vc;
-  CUtensorMap tm_kn;       // 3D {d, S, B*Hkv}, box {64, 128, 1}
-  CUtensorMap tm_vn;
+  CUtensorMap tm_kc;       // 3D {d, M, B*Hkv}, box {64, 64 (d = 128) or 128, 1}
+  CUtensorMap tm_vc;       // 3D {d, M, B*Hkv}, box {64, 128, 1}
+  CUtensorMap tm_kn;       // 3D {d, S, B*Hkv}, box as tm_kc
+  CUtensorMap tm_vn;       // 3D {d, S, B*Hkv}, box as tm_vc
   const int32_t* slot_pos; // (B, Hkv, M)
   uint16_t* out;           // (B, Hq, S, d) bf16
   float* score_inc;        // (B, Hq, M + S)

@@ -15,10 +15,19 @@
 //    Q K^T, forms P = exp2(S log2e scale - lambda log2e) in fp32, reduces P's
 //    columns into score_inc and accumulates P V.  Because lambda is final in
 //    pass 2, the P V accumulator never needs rescaling.
+//  * d = 128 runs on CTA pairs (a cluster of two CTAs, adjacent row tiles of
+//    the same group) with the 2-SM tcgen05 MMA (M = 256): each CTA loads only
+//    half of every K tile (64 keys) and half of every V tile (64 of the d
+//    columns), which halves the L2-to-SM traffic per MMA.  The even CTA
+//    issues all MMAs; the odd CTA's softmax warps signal it through its
+//    barriers.  Both CTAs walk the union of their key-tile lists; a tile only
+//    the other CTA can see is fully masked here.  d = 64 runs one CTA per row
+//    tile with the 1-SM MMA.
 //  * Warp roles: warp 0 issues TMA loads (Q once, then K tiles through ring A
-//    and V tiles through ring B of shared-memory slots); warp 1 issues every
-//    Q K^T and warp 2 every P V tcgen05 MMA, so one issuer keeps the tensor pipe
-//    busy while the other waits on a barrier; warps 3-18 form four softmax
+//    and V tiles through ring B of shared-memory slots); warps 1 and 2 issue
+//    the tcgen05 MMAs (pass 1: Q K^T of alternate tiles; pass 2: warp 1 every
+//    Q K^T, warp 2 every P V), so one issuer keeps the tensor pipe busy while
+//    the other waits on a barrier; warps 3-18 form four softmax
 //    warpgroups in two teams that take alternate tiles; the two warpgroups of a
 //    team own key columns 0-63 and 64-127 of their tiles.
 //  * TMEM holds two fp32 S buffers, two bf16 P buffers and the O accumulator.
@@ -29,9 +38,10 @@
 //    reads S in TMEM's 16x256b layout, where a thread holds 4 rows x 8
 //    columns: it adds its 4 rows, a 3-step warp reduce-scatter leaves one
 //    column sum (over the warp's 32 rows) per lane and 32-column block, the
-//    four warps of a warpgroup combine through shared memory, and one red.global.add per
-//    column and query head goes to score_inc (zeroed by the host call).
-//    Pass 1 keeps one row per thread (32x32b layout) for the row statistics.
+//    last of the four warps of a warpgroup to finish a tile combines them
+//    through shared memory, and one red.global.add per column and query head
+//    goes to score_inc (zeroed by the host call).  Pass 1 keeps one row per
+//    thread (32x32b layout) for the row statistics.
 //  * Key tiles are classified up front from slot_pos: tiles no row of the CTA
 //    can see are skipped, tiles every row sees need no mask, the rest are
 //    masked per element.
@@ -53,41 +63,70 @@ constexpr uint16_t kTileChunk = 0x8000;
 constexpr uint16_t kTilePartial = 0x4000;
 constexpr uint16_t kTileIdxMask = 0x3FFF;
 constexpr uint8_t kClsSkip = 0, kClsFull = 1, kClsPartial = 2;
-// TMEM: two S buffers (fp32, 128 columns each), two P buffers (bf16 pairs, 64
-// columns each) and the O accumulator: 2*128 + 2*64 + 128 = 512 columns.  An S
-// buffer is free again as soon as the softmax has loaded it; a P buffer when
-// the P V that read it has completed.
+// TMEM (512 columns).  Pass 1 needs no P or O: four S buffers (fp32, 128
+// columns each).  Pass 2: S buffers 0 and 1, two P buffers (bf16 pairs, 64
+// columns each) over the columns of S buffer 2, and the O accumulator over
+// those of S buffer 3.  An S buffer is free again as soon as the softmax has
+// loaded it; a P buffer when the P V that read it has completed.
+constexpr int kSBufs1 = 4;
 constexpr int kSBufs = 2;
 constexpr int kPBufs = 2;
 constexpr int kPCols = kTileN / 2;
 
-// K tiles go through ring A (consumed by the Q K^T issuer), V tiles through
-// ring B (consumed by the P V issuer); each ring has a single consumer that
-// takes its loads in order, which keeps every mbarrier wait at most one phase
-// ahead.  Slots are 32 KB (d = 128) or 16 KB (d = 64).
-template <int D>
-__host__ __device__ constexpr int ring_a_slots() { return D == 128 ? 3 : 6; }
-template <int D>
-__host__ __device__ constexpr int ring_b_slots() { return D == 128 ? 2 : 4; }
-template <int D>
-__host__ __device__ constexpr int ring_slots() { return ring_a_slots<D>() + ring_b_slots<D>(); }
+// S buffer of step n (pass-1 tile n < n_t, pass-2 tile n - n_t) and how many
+// times that buffer was filled before.
+__device__ __forceinline__ void s_buffer(int n, int n_t, int& buf, int& use) {
+  if (n < n_t) {
+    buf = n % kSBufs1;
+    use = n / kSBufs1;
+  } else {
+    buf = (n - n_t) % kSBufs;
+    use = (n_t > buf ? (n_t - 1 - buf) / kSBufs1 + 1 : 0) + (n - n_t) / kSBufs;
+  }
+}
 
-template <int D>
-struct __align__(1024) SdpaSmem {
+// Shared-memory ring geometry.  Pass 1 streams K tiles through all slots;
+// pass 2 sends K tiles through ring A (consumed by the Q K^T issuer) and V
+// tiles through ring B (consumed by the P V issuer).  Within each pass a slot
+// has a single consumer that takes its loads in order, and pass 2 starts on a
+// slot only after pass 1 has consumed it, which keeps every mbarrier wait at
+// most one phase ahead.
+//   1-SM (d = 64):  a slot holds a whole K or V tile, 16 KB.
+//   pair (d = 128): a slot holds this CTA's half of a K tile (64 keys x 128
+//                   columns, two 8 KB panels) or of a V tile (128 keys x 64
+//                   columns, one 16 KB panel).
+template <int D, bool kPair>
+struct Geom {
   static constexpr int kPanels = D / 64;
-  uint8_t q[kPanels][kTileM * 128];
-  uint8_t kv[ring_slots<D>()][kPanels][kTileN * 128];
+  static constexpr int kSlotBytes = kPair ? 16384 : kPanels * kTileN * 128;
+  static constexpr int kKPanelBytes = kPair ? (kTileN / 2) * 128 : kTileN * 128;
+  static constexpr int kRA = kPair ? 6 : (D == 128 ? 3 : 6);
+  static constexpr int kRB = kPair ? 4 : (D == 128 ? 2 : 4);
+  static constexpr int kR = kRA + kRB;
+  static constexpr int kCtas = kPair ? 2 : 1;
+};
+
+// Loads of pass 1 (tiles 0 .. n_t - 1, slot t % R) that land in slot s.
+__device__ __forceinline__ int pass1_uses(int n_t, int R, int s) {
+  return n_t > s ? (n_t - 1 - s) / R + 1 : 0;
+}
+
+template <int D, bool kPair>
+struct __align__(1024) SdpaSmem {
+  using G = Geom<D, kPair>;
+  uint8_t q[G::kPanels][kTileM * 128];
+  uint8_t kv[G::kR][G::kSlotBytes];
   float colsum[2][kNumWG][4][64];  // [buffer][warpgroup][warp][column]
   float rowstat[kNumWG][kTileM][2];
   uint64_t bar_q;
-  uint64_t bar_full[ring_slots<D>()], bar_empty[ring_slots<D>()];
-  uint64_t bar_sfull[kSBufs], bar_sread[kSBufs], bar_pfull[kPBufs], bar_pvdone[kPBufs];
-  uint64_t bar_cs[2][kNumWG];
-  uint64_t bar_rowstat, bar_ofull, bar_drain[2];
+  uint64_t bar_full[G::kR], bar_empty[G::kR];
+  uint64_t bar_sfull[kSBufs1], bar_sread[kSBufs1], bar_pfull[kPBufs], bar_pvdone[kPBufs];
+  uint64_t bar_rowstat, bar_ofull, bar_drain[2], bar_p1done;
+  uint32_t cs_count[2][kNumWG];  // column-sum partials deposited (4 per tile)
   uint32_t taddr;
   int abort_flag;
   int n_tiles;
-  uint8_t cls[kMaxKeyTiles];
+  uint8_t cls[kMaxKeyTiles];  // bits 0-1: this CTA's class, bits 2-3: the other CTA's
   uint16_t tiles[kMaxKeyTiles];
 };
 
@@ -105,109 +144,162 @@ __device__ __forceinline__ void rs_step(float (&v)[8], uint32_t lane) {
   }
 }
 
-template <int D>
+// Bounded barrier wait.  Every signal between the CTAs of a pair orders
+// tcgen05 operations or TMA writes only (tcgen05 fences around the barrier,
+// complete_tx accounting), so CTA-scope acquire suffices.
+template <bool kPair>
+__device__ __forceinline__ bool wait_b(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  return wait_bar(bar, parity, abort, kWaitLimitNs);
+}
+
+// Arrival of a softmax warp on a barrier of the MMA-issuing CTA.
+template <bool kPair>
+__device__ __forceinline__ void arrive_issuer(uint64_t* bar) {
+  if constexpr (kPair) bar_arrive_remote(cluster_addr(bar, 0));
+  else bar_arrive(bar);
+}
+
+template <bool kPair>
+__device__ __forceinline__ void commit_all(uint64_t* bar) {
+  if constexpr (kPair) mma_commit_pair(bar, 3);
+  else mma_commit(bar);
+}
+
+// Query rows of row tile r: head of the first row, first/last chunk row.
+// False when r is past the last row tile (the odd CTA of the last pair).
+__device__ __forceinline__ bool row_range(const SdpaArgs& a, int r, int& g_first, int& i_lo,
+                                          int& i_hi) {
+  if (r >= a.n_row_tiles) return false;
+  if (a.tiles_per_head > 0) {
+    g_first = r / a.tiles_per_head;
+    i_lo = (r % a.tiles_per_head) * kTileM;
+    i_hi = min(i_lo + kTileM, a.S) - 1;
+  } else {
+    g_first = r * a.heads_box;
+    i_lo = 0;
+    i_hi = a.S - 1;
+  }
+  return true;
+}
+
+template <int D, bool kPair>
 __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_constant__ SdpaArgs a) {
-  constexpr int P = D / 64;
+  using G = Geom<D, kPair>;
+  constexpr int P = G::kPanels;
   extern __shared__ uint8_t smem_raw[];
-  auto& sm = *reinterpret_cast<SdpaSmem<D>*>(
+  auto& sm = *reinterpret_cast<SdpaSmem<D, kPair>*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const uint32_t lane = tid & 31;
   const int grp = blockIdx.y;  // b * Hkv + kv head
   const int rt = blockIdx.x;   // row tile within the group
+  const uint32_t rank = kPair ? cluster_rank() : 0u;
+  const bool leader = rank == 0;
   const int b = grp / a.Hkv;
   const int hkv = grp % a.Hkv;
   const int NK = a.M + a.S;    // key columns per query head
 
-  // Query rows of this tile: rows_box rows per head, heads_box heads.
-  int g_first, i_lo, i_hi;
-  if (a.tiles_per_head > 0) {
-    g_first = rt / a.tiles_per_head;
-    i_lo = (rt % a.tiles_per_head) * kTileM;
-    i_hi = min(i_lo + kTileM, a.S) - 1;
-  } else {
-    g_first = rt * a.heads_box;
-    i_lo = 0;
-    i_hi = a.S - 1;
-  }
-  const int rows_used = a.tiles_per_head > 0 ? kTileM : a.rows_box * a.heads_box;
+  int g_first = a.qg, i_lo = 0, i_hi = -1;
+  const bool has_rows = row_range(a, rt, g_first, i_lo, i_hi);
+  int pg = 0, p_lo = 0, p_hi = -1;
+  const bool peer_rows = kPair && row_range(a, rt ^ 1, pg, p_lo, p_hi);
+  // rows the Q box covers (the rest of the tile is zero-filled here)
+  const int box_rows = a.tiles_per_head > 0 ? kTileM : a.rows_box * a.heads_box;
 
   if (tid == 0) {
     bar_init(&sm.bar_q, 1);
-    for (int s = 0; s < ring_slots<D>(); ++s) {
+    for (int s = 0; s < G::kR; ++s) {
       bar_init(&sm.bar_full[s], 1);
       bar_init(&sm.bar_empty[s], 1);
     }
-    for (int x = 0; x < kSBufs; ++x) {
+    for (int x = 0; x < kSBufs1; ++x) {
       bar_init(&sm.bar_sfull[x], 1);
-      bar_init(&sm.bar_sread[x], kSoftmaxWarps / 2);  // the 8 warps of the team owning the tile
+      // the 8 warps of the team owning the tile, in every CTA of the pair
+      bar_init(&sm.bar_sread[x], G::kCtas * kSoftmaxWarps / 2);
     }
     for (int x = 0; x < kPBufs; ++x) {
-      bar_init(&sm.bar_pfull[x], kSoftmaxWarps / 2);
+      bar_init(&sm.bar_pfull[x], G::kCtas * kSoftmaxWarps / 2);
       bar_init(&sm.bar_pvdone[x], 1);
     }
     for (int x = 0; x < 2; ++x)
-      for (int w = 0; w < kNumWG; ++w) bar_init(&sm.bar_cs[x][w], 4);
+      for (int w = 0; w < kNumWG; ++w) sm.cs_count[x][w] = 0u;
     bar_init(&sm.bar_rowstat, kSoftmaxWarps);
     bar_init(&sm.bar_ofull, 1);
     bar_init(&sm.bar_drain[0], 1);
     bar_init(&sm.bar_drain[1], 1);
+    bar_init(&sm.bar_p1done, 1);
     sm.abort_flag = 0;
     fence_bar_init();
   }
   if (warp == 1) {
-    tmem_alloc(&sm.taddr, 512);
-    tmem_relinquish();
+    if constexpr (kPair) {
+      tmem_alloc_pair(&sm.taddr, 512);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(&sm.taddr, 512);
+      tmem_relinquish();
+    }
   }
   // Rows the Q box does not cover must still give finite logits.
-  if (rows_used < kTileM) {
-    const int words = (kTileM - rows_used) * 32;
+  if (box_rows < kTileM) {
+    const int words = (kTileM - box_rows) * 32;
     for (int p = 0; p < P; ++p)
       for (int x = tid; x < words; x += kThreads)
-        reinterpret_cast<uint32_t*>(sm.q[p] + rows_used * 128)[x] = 0u;
+        reinterpret_cast<uint32_t*>(sm.q[p] + box_rows * 128)[x] = 0u;
     fence_proxy_async_smem();
   }
-  // Classify key tiles against this CTA's rows.
+  // Classify key tiles against this CTA's rows (bits 0-1) and, on a pair, the
+  // other CTA's rows (bits 2-3).
   if (warp >= kFirstSoftmaxWarp) {
     const int sw = warp - kFirstSoftmaxWarp;
     const int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
-    const int lim_any = a.pos0 + i_hi;
-    const int lim_all = a.pos0 + i_lo;
     for (int ct = sw; ct < a.n_cache_tiles; ct += kSoftmaxWarps) {
-      bool any = false, all = true;
+      bool any0 = false, all0 = true, any1 = false, all1 = true;
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
         const int j = ct * kTileN + r * 32 + static_cast<int>(lane);
         const int pos = j < a.M ? __ldg(sp + j) : -1;
-        any |= pos >= 0 && pos <= lim_any;
-        all &= pos >= 0 && pos <= lim_all;
+        any0 |= pos >= 0 && pos <= a.pos0 + i_hi;
+        all0 &= pos >= 0 && pos <= a.pos0 + i_lo;
+        any1 |= pos >= 0 && pos <= a.pos0 + p_hi;
+        all1 &= pos >= 0 && pos <= a.pos0 + p_lo;
       }
-      any = __any_sync(0xffffffffu, any);
-      all = __all_sync(0xffffffffu, all);
-      if (lane == 0) sm.cls[ct] = any ? (all ? kClsFull : kClsPartial) : kClsSkip;
+      any0 = __any_sync(0xffffffffu, any0) && has_rows;
+      all0 = __all_sync(0xffffffffu, all0);
+      any1 = __any_sync(0xffffffffu, any1) && peer_rows;
+      all1 = __all_sync(0xffffffffu, all1);
+      const uint8_t c0 = any0 ? (all0 ? kClsFull : kClsPartial) : kClsSkip;
+      const uint8_t c1 = any1 ? (all1 ? kClsFull : kClsPartial) : kClsSkip;
+      if (lane == 0) sm.cls[ct] = static_cast<uint8_t>(c0 | (c1 << 2));
     }
     for (int c = sw; c < a.n_chunk_tiles; c += kSoftmaxWarps) {
       const int c0 = c * kTileN;
-      uint8_t cl = kClsPartial;
-      if (c0 > i_hi) cl = kClsSkip;
-      else if (c0 + kTileN - 1 <= i_lo && c0 + kTileN <= a.S) cl = kClsFull;
+      auto chunk_cls = [&](bool rows, int lo, int hi) -> uint8_t {
+        if (!rows || c0 > hi) return kClsSkip;
+        if (c0 + kTileN - 1 <= lo && c0 + kTileN <= a.S) return kClsFull;
+        return kClsPartial;
+      };
+      const uint8_t cl = static_cast<uint8_t>(chunk_cls(has_rows, i_lo, i_hi) |
+                                              (chunk_cls(peer_rows, p_lo, p_hi) << 2));
       if (lane == 0) sm.cls[a.n_cache_tiles + c] = cl;
     }
   }
   __syncthreads();
   if (warp == kFirstSoftmaxWarp) {
+    // tile list: the union over the pair, in order; masked here unless this
+    // CTA sees every key of the tile from every row
     const int total = a.n_cache_tiles + a.n_chunk_tiles;
     int n = 0;
     for (int base = 0; base < total; base += 32) {
       const int t = base + static_cast<int>(lane);
-      const uint8_t cl = t < total ? sm.cls[t] : kClsSkip;
-      const uint32_t m = __ballot_sync(0xffffffffu, cl != kClsSkip);
-      if (cl != kClsSkip) {
+      const uint8_t cl = t < total ? sm.cls[t] : 0;
+      const uint32_t m = __ballot_sync(0xffffffffu, cl != 0);
+      if (cl != 0) {
         const int pos = n + __popc(m & ((1u << lane) - 1u));
         uint16_t e = t < a.n_cache_tiles ? static_cast<uint16_t>(t)
                                          : static_cast<uint16_t>(kTileChunk | (t - a.n_cache_tiles));
-        if (cl == kClsPartial) e |= kTilePartial;
+        if ((cl & 3) != kClsFull) e |= kTilePartial;
         sm.tiles[pos] = e;
       }
       n += __popc(m);
@@ -216,12 +308,16 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
   }
   tc_fence_before_sync();
   __syncthreads();
+  // On a pair, both CTAs' barriers are initialised (and the zero-filled Q rows
+  // published) before any signal crosses between them.
+  if constexpr (kPair) cluster_sync_all();
   tc_fence_after_sync();
 
   const uint32_t tmem = sm.taddr;
   const uint32_t tS = tmem;                          // S buffer b: columns 128 b ..
   const uint32_t tP = tmem + 128 * kSBufs;           // P buffer p: columns 256 + 64 p ..
   const uint32_t tO = tP + kPCols * kPBufs;          // O accumulator: columns 384 ..
+  static_assert(128 * kSBufs + kPCols * kPBufs + 128 == 128 * kSBufs1, "TMEM layout");
   const int n_t = sm.n_tiles;
   volatile int* abort_flag = &sm.abort_flag;
 
@@ -235,120 +331,173 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         tma_prefetch_desc(&a.tm_kc);
         tma_prefetch_desc(&a.tm_vc);
       }
-      bar_expect_tx(&sm.bar_q, P * 128 * a.rows_box * a.heads_box);
-      for (int p = 0; p < P; ++p) tma_load_4d(sm.q[p], &a.tm_q, &sm.bar_q, 64 * p, i_lo, g_first, grp);
-      constexpr int RA = ring_a_slots<D>(), RB = ring_b_slots<D>();
-      int L[2] = {0, 0};  // loads issued per ring; ring r uses slots base_r + L % R_r
-      auto load = [&](bool is_v, int t) -> bool {
+      constexpr int RA = G::kRA, RB = G::kRB, R = G::kR;
+      const uint32_t q_bytes = P * 128 * box_rows;
+      if constexpr (kPair) {
+        const uint32_t bq = cluster_addr(&sm.bar_q, 0);
+        if (leader) bar_expect_tx(&sm.bar_q, 2 * q_bytes);
+        for (int p = 0; p < P; ++p)
+          tma_load_4d_pair(sm.q[p], &a.tm_q, bq, 64 * p, i_lo, g_first, grp);
+      } else {
+        bar_expect_tx(&sm.bar_q, q_bytes);
+        for (int p = 0; p < P; ++p) tma_load_4d(sm.q[p], &a.tm_q, &sm.bar_q, 64 * p, i_lo, g_first, grp);
+      }
+      int uses[R];  // loads issued into each slot so far
+#pragma unroll
+      for (int x = 0; x < R; ++x) uses[x] = 0;
+      auto load = [&](int s, bool is_v, int t) -> bool {
         const uint16_t e = sm.tiles[t];
         const bool chunk = (e & kTileChunk) != 0;
         const int row0 = (e & kTileIdxMask) * kTileN;
         const CUtensorMap* m =
             is_v ? (chunk ? &a.tm_vn : &a.tm_vc) : (chunk ? &a.tm_kn : &a.tm_kc);
-        const int r = is_v ? 1 : 0;
-        const int R = is_v ? RB : RA;
-        const int s = (is_v ? RA : 0) + L[r] % R;
-        if (L[r] >= R &&
-            !wait_bar(&sm.bar_empty[s], ((L[r] / R) - 1) & 1, abort_flag, kWaitLimitNs))
-          return false;
-        bar_expect_tx(&sm.bar_full[s], P * kTileN * 128);
-        for (int p = 0; p < P; ++p) tma_load_3d(sm.kv[s][p], m, &sm.bar_full[s], 64 * p, row0, grp);
-        ++L[r];
+        const int u = uses[s];
+        if (u > 0 && !wait_b<kPair>(&sm.bar_empty[s], (u - 1) & 1, abort_flag)) return false;
+        if constexpr (kPair) {
+          // this CTA's half: keys 64 rank .. of a K tile (both column panels),
+          // columns 64 rank .. of a V tile (all 128 keys)
+          const uint32_t bf = cluster_addr(&sm.bar_full[s], 0);
+          if (leader) bar_expect_tx(&sm.bar_full[s], 2 * G::kSlotBytes);
+          if (is_v) {
+            tma_load_3d_pair(sm.kv[s], m, bf, 64 * static_cast<int>(rank), row0, grp);
+          } else {
+            for (int p = 0; p < P; ++p)
+              tma_load_3d_pair(sm.kv[s] + p * G::kKPanelBytes, m, bf, 64 * p,
+                               row0 + (kTileN / 2) * static_cast<int>(rank), grp);
+          }
+        } else {
+          bar_expect_tx(&sm.bar_full[s], G::kSlotBytes);
+          for (int p = 0; p < P; ++p)
+            tma_load_3d(sm.kv[s] + p * G::kKPanelBytes, m, &sm.bar_full[s], 64 * p, row0, grp);
+        }
+        uses[s] = u + 1;
         return true;
       };
-      // pass 1: K_0..K_{n-1}; pass 2: K_t interleaved with V_{t-2}, then the last V's
+      // pass 1: K_0..K_{n-1} over all slots; pass 2: K_t (ring A) interleaved
+      // with V_{t-2} (ring B), then the last V's
       bool ok = true;
-      for (int t = 0; ok && t < n_t; ++t) ok = load(false, t);
+      for (int t = 0; ok && t < n_t; ++t) ok = load(t % R, false, t);
       for (int t = 0; ok && t < n_t; ++t) {
-        ok = load(false, t);
-        if (ok && t >= 2) ok = load(true, t - 2);
+        ok = load(t % RA, false, t);
+        if (ok && t >= 2) ok = load(RA + (t - 2) % RB, true, t - 2);
       }
-      for (int t = max(0, n_t - 2); ok && t < n_t; ++t) ok = load(true, t);
+      for (int t = max(0, n_t - 2); ok && t < n_t; ++t) ok = load(RA + t % RB, true, t);
       if (*abort_flag) {
-        // Let copies still in flight land before the CTA's shared memory goes away.
+        // Let copies still in flight land before the CTA's shared memory goes
+        // away: at most the latest load of each slot can be outstanding.  On a
+        // pair the copies are counted on the even CTA's barriers, so this CTA
+        // also gives them a fixed grace period.
         volatile int never = 0;
-        for (int x = max(0, L[0] - RA); x < L[0]; ++x)
-          wait_bar(&sm.bar_full[x % RA], (x / RA) & 1, &never, 100000000ull);
-        for (int x = max(0, L[1] - RB); x < L[1]; ++x)
-          wait_bar(&sm.bar_full[RA + x % RB], (x / RB) & 1, &never, 100000000ull);
+        if (leader)
+          for (int x = 0; x < R; ++x)
+            if (uses[x] > 0) wait_bar(&sm.bar_full[x], (uses[x] - 1) & 1, &never, 100000000ull);
+        const uint64_t t0 = global_timer_ns();
+        while (kPair && global_timer_ns() - t0 < 200000ull) {
+        }
       }
     }
   } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------- MMA issuers --
-    // Warp 1 issues every Q K^T (in tile order, so S buffers complete in
-    // order); warp 2 issues every P V and owns the O accumulator.  With two
+    // Pass 1: warps 1 and 2 issue the Q K^T of alternate tiles (each S buffer
+    // has one issuer, so its phases complete in order).  Pass 2: warp 1 issues
+    // every Q K^T, warp 2 every P V and owns the O accumulator.  With two
     // issuing threads the tensor pipe keeps working while one of them waits on
-    // a barrier after its commits.
-    if (lane == 0 && n_t > 0) {
-      constexpr uint32_t kIdescQK = idesc_bf16_f32(kTileM, kTileN, false);
-      constexpr uint32_t kIdescPV = idesc_bf16_f32(kTileM, D, true);
-      // Descriptors are built once; per MMA only the 14-bit start-address
-      // field advances, by compile-time immediates (bytes >> 4): a K-step of
-      // 16 bf16 is 32 B inside a 128-B swizzle row, a 64-column panel is
-      // 16 KB, a ring slot is P panels, 16 rows of V are 2 KB.
-      constexpr uint32_t kPanel = (kTileN * 128) >> 4;
-      constexpr uint32_t kSlot = P * kPanel;
-      constexpr int RA = ring_a_slots<D>(), RB = ring_b_slots<D>();
+    // a barrier or commits.  On a pair only the even CTA issues.
+    if (lane == 0 && n_t > 0 && leader) {
+      constexpr int kM = kPair ? 2 * kTileM : kTileM;
+      constexpr uint32_t kIdescQK = idesc_bf16_f32(kM, kTileN, false);
+      constexpr uint32_t kIdescPV = idesc_bf16_f32(kM, D, true);
+      // Descriptors: per MMA only the 14-bit start-address field advances
+      // (bytes >> 4): a K-step of 16 bf16 is 32 B inside a 128-B swizzle row, a
+      // 64-column panel is 16 KB for Q (8 KB for a pair's half K tile), a ring
+      // slot is kSlotBytes, 16 rows of V are 2 KB.  All eight are formed
+      // before the first MMA of a tile is issued.
+      constexpr uint32_t kQPanel = (kTileM * 128) >> 4;
+      constexpr uint32_t kKPanel = G::kKPanelBytes >> 4;
+      constexpr uint32_t kSlot = G::kSlotBytes >> 4;
+      constexpr int RA = G::kRA, RB = G::kRB;
       const bool is_qk = warp == 1;
-      bool ok = true;
-      if (is_qk) {
-        const uint64_t q_desc = sdesc_sw128(smem_addr(sm.q[0]), 16, 1024);
-        const uint64_t k_desc0 = sdesc_sw128(smem_addr(sm.kv[0][0]), 16, 1024);
-        ok = wait_bar(&sm.bar_q, 0, abort_flag, kWaitLimitNs);
-        for (int n = 0; ok && n < 2 * n_t; ++n) {
-          const int buf = n % kSBufs;
-          // buffer reuse: the softmax has loaded the S of tile n - 2
-          if (n >= kSBufs &&
-              !wait_bar(&sm.bar_sread[buf], ((n - kSBufs) / kSBufs) & 1, abort_flag, kWaitLimitNs)) {
-            ok = false;
-            break;
-          }
-          const int s = n % RA;  // ring A holds exactly the K tiles, in this order
-          if (!wait_bar(&sm.bar_full[s], (n / RA) & 1, abort_flag, kWaitLimitNs)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after_sync();
-          const uint64_t kd = k_desc0 + static_cast<uint64_t>(s) * kSlot;
-          const uint32_t d_tmem = tS + buf * 128;
+      const uint64_t q_desc = sdesc_sw128(smem_addr(sm.q[0]), 16, 1024);
+      const uint64_t k_desc0 = sdesc_sw128(smem_addr(sm.kv[0]), 16, 1024);
+      uint64_t qd[8];
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = kPanel * (kk / 4) + 2 * (kk % 4);
-            mma_ss(d_tmem, q_desc + off, kd + off, kIdescQK, kk > 0 ? 1u : 0u);
-          }
-          mma_commit(&sm.bar_sfull[buf]);
-          mma_commit(&sm.bar_empty[s]);
+      for (int kk = 0; kk < 8; ++kk) qd[kk] = q_desc + kQPanel * (kk / 4) + 2 * (kk % 4);
+      // S_n = Q K_t^T (tile t = n, or n - n_t in pass 2) into its S buffer
+      auto issue_qk = [&](int n) -> bool {
+        int buf, suse;
+        s_buffer(n, n_t, buf, suse);
+        // buffer reuse: the softmax has loaded the buffer's previous S
+        if (suse > 0 && !wait_b<kPair>(&sm.bar_sread[buf], (suse - 1) & 1, abort_flag))
+          return false;
+        int s, use;
+        if (n < n_t) {
+          s = n % (RA + RB);
+          use = n / (RA + RB);
+        } else {
+          s = (n - n_t) % RA;
+          use = pass1_uses(n_t, RA + RB, s) + (n - n_t) / RA;
         }
+        if (!wait_b<kPair>(&sm.bar_full[s], use & 1, abort_flag)) return false;
+        tc_fence_after_sync();
+        const uint64_t kd = k_desc0 + static_cast<uint64_t>(s) * kSlot;
+        const uint32_t d_tmem = tS + buf * 128;
+        if constexpr (D == 128) {
+          uint64_t bd[8];
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) bd[kk] = kd + kKPanel * (kk / 4) + 2 * (kk % 4);
+          mma_ss_x8<kPair>(d_tmem, qd, bd, kIdescQK, 0u);
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk)
+            mma_ss(d_tmem, qd[kk], kd + kKPanel * (kk / 4) + 2 * (kk % 4), kIdescQK, kk > 0 ? 1u : 0u);
+        }
+        commit_all<kPair>(&sm.bar_sfull[buf]);
+        commit_all<kPair>(&sm.bar_empty[s]);
+        return true;
+      };
+      bool ok = wait_b<kPair>(&sm.bar_q, 0, abort_flag);
+      if (is_qk) {
+        // pass 1: even tiles here, odd tiles on warp 2 (idle until pass 2)
+        for (int n = 0; ok && n < n_t; n += 2) ok = issue_qk(n);
+        // pass 2 reuses slots that warp 2 took in pass 1: start once it has
+        // waited for all of its pass-1 tiles, so that no full-barrier wait
+        // here runs two phases ahead
+        if (ok) ok = wait_b<kPair>(&sm.bar_p1done, 0, abort_flag);
+        for (int n = n_t; ok && n < 2 * n_t; ++n) ok = issue_qk(n);
       } else {
-        const uint64_t v_desc0 = sdesc_sw128(smem_addr(sm.kv[RA][0]), kTileN * 128, 1024);
+        for (int n = 1; ok && n < n_t; n += 2) ok = issue_qk(n);
+        bar_arrive(&sm.bar_p1done);
+        const uint64_t v_desc0 = sdesc_sw128(smem_addr(sm.kv[RA]), kTileN * 128, 1024);
         for (int t = 0; ok && t < n_t; ++t) {
           const int pb = t % kPBufs;
-          if (!wait_bar(&sm.bar_pfull[pb], (t / kPBufs) & 1, abort_flag, kWaitLimitNs)) {
+          if (!wait_b<kPair>(&sm.bar_pfull[pb], (t / kPBufs) & 1, abort_flag)) {
             ok = false;
             break;
           }
           const int vs = RA + t % RB;
-          if (!wait_bar(&sm.bar_full[vs], (t / RB) & 1, abort_flag, kWaitLimitNs)) {
+          const int use = pass1_uses(n_t, RA + RB, vs) + t / RB;
+          if (!wait_b<kPair>(&sm.bar_full[vs], use & 1, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after_sync();
           const uint64_t vd = v_desc0 + static_cast<uint64_t>(t % RB) * kSlot;
-          const uint32_t a_base = tP + kPCols * pb;
-          const uint32_t acc0 = t > 0 ? 1u : 0u;
-          // keys 16kk..16kk+15 sit as bf16 pairs in columns 8kk..8kk+7 of the P buffer
+          uint64_t bd[8];
 #pragma unroll
-          for (int kk = 0; kk < kTileN / 16; ++kk)
-            mma_ts(tO, a_base + 8 * kk, vd + 128 * kk, kIdescPV, kk > 0 ? 1u : acc0);
-          mma_commit(&sm.bar_empty[vs]);
-          mma_commit(&sm.bar_pvdone[pb]);
+          for (int kk = 0; kk < 8; ++kk) bd[kk] = vd + 128 * kk;
+          // keys 16kk..16kk+15 sit as bf16 pairs in columns 8kk..8kk+7 of the P buffer
+          mma_ts_x8<kPair>(tO, tP + kPCols * pb, bd, kIdescPV, t > 0 ? 1u : 0u);
+          commit_all<kPair>(&sm.bar_empty[vs]);
+          commit_all<kPair>(&sm.bar_pvdone[pb]);
         }
-        if (ok) mma_commit(&sm.bar_ofull);
+        if (ok) commit_all<kPair>(&sm.bar_ofull);
       }
       // No MMA of this thread may still be running when TMEM is freed.
-      mma_commit(&sm.bar_drain[is_qk ? 0 : 1]);
+      uint64_t* drain = &sm.bar_drain[is_qk ? 0 : 1];
+      if constexpr (kPair) mma_commit_pair(drain, 1);
+      else mma_commit(drain);
       volatile int never = 0;
-      wait_bar(&sm.bar_drain[is_qk ? 0 : 1], 0, &never, kWaitLimitNs);
+      wait_b<kPair>(drain, 0, &never);
     }
   } else {
     // ------------------------------------------- softmax / column sums --
@@ -364,14 +513,16 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     const int row = q4 * 32 + static_cast<int>(lane);
     // tile row -> (head within the group, chunk row i); false for padding rows
     auto row_info = [&](int r, int& gg, int& ii) -> bool {
+      gg = g_first;
+      ii = i_lo;
+      if (!has_rows) return false;
       if (a.tiles_per_head > 0) {
-        gg = g_first;
         ii = i_lo + r;
         return ii < a.S;
       }
       gg = g_first + r / a.rows_box;
       ii = r % a.rows_box;
-      return r < rows_used && ii < a.S && gg < a.qg;
+      return r < box_rows && ii < a.S && gg < a.qg;
     };
     int g, i;
     const bool valid = row_info(row, g, i);
@@ -397,9 +548,11 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     int warp_head[4];
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
-      int gw;
-      if (a.tiles_per_head > 0) gw = (i_lo + w * 32 < a.S) ? g_first : -1;
-      else gw = (w * 32 < rows_used) ? g_first + (w * 32) / a.rows_box : -1;
+      int gw = -1;
+      if (has_rows) {
+        if (a.tiles_per_head > 0) gw = (i_lo + w * 32 < a.S) ? g_first : -1;
+        else gw = (w * 32 < box_rows) ? g_first + (w * 32) / a.rows_box : -1;
+      }
       warp_head[w] = (gw >= 0 && gw < a.qg) ? gw : -1;
     }
     float m_run = -INFINITY, l_run = 0.f;
@@ -408,7 +561,8 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     bool have_lambda = false;
     int k2 = 0;  // pass-2 tiles this warp has processed (column-sum buffer phase)
     for (int n = team; ok && n < 2 * n_t; n += 2) {
-      const int buf = n % kSBufs;
+      int buf, suse;
+      s_buffer(n, n_t, buf, suse);
       const bool pass2 = n >= n_t;
       const int t = pass2 ? n - n_t : n;
       if (pass2 && !have_lambda) {
@@ -436,7 +590,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         }
         have_lambda = true;
       }
-      if (!wait_bar(&sm.bar_sfull[buf], (n / kSBufs) & 1, abort_flag, kWaitLimitNs)) {
+      if (!wait_b<kPair>(&sm.bar_sfull[buf], suse & 1, abort_flag)) {
         ok = false;
         break;
       }
@@ -462,7 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         }
         tc_fence_before_sync();
         __syncwarp();
-        if (lane == 0) bar_arrive(&sm.bar_sread[buf]);  // S buffer may be overwritten
+        if (lane == 0) arrive_issuer<kPair>(&sm.bar_sread[buf]);  // S buffer may be overwritten
         if (!partial) {
           float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
 #pragma unroll
@@ -485,15 +639,17 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           m_run = m_new;
         } else {
           uint64_t vis = 0ull;  // bit k: column col0 + k visible to this row
-          if (chunk) {
+          if (valid) {
+            if (chunk) {
 #pragma unroll
-            for (int k = 0; k < 64; ++k)
-              if (col0 + k <= i && col0 + k < a.S) vis |= 1ull << k;
-          } else {
-            for (int k = 0; k < 64; ++k) {
-              const int j = col0 + k;
-              const int pos = j < a.M ? __ldg(sp_base + j) : -1;
-              if (pos >= 0 && pos <= qpos) vis |= 1ull << k;
+              for (int k = 0; k < 64; ++k)
+                if (col0 + k <= i && col0 + k < a.S) vis |= 1ull << k;
+            } else {
+              for (int k = 0; k < 64; ++k) {
+                const int j = col0 + k;
+                const int pos = j < a.M ? __ldg(sp_base + j) : -1;
+                if (pos >= 0 && pos <= qpos) vis |= 1ull << k;
+              }
             }
           }
           float mx = -INFINITY;
@@ -518,26 +674,24 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         const int cb = k2 & 1;
         const int pbuf = t % kPBufs;
         const uint32_t p_base = tP + lane_addr + kPCols * pbuf + u * 32;
-#pragma unroll 1
+        // both 32-column halves of S are loaded before any is processed, so
+        // the S buffer is released at once
+        uint32_t rs[2][32];
+        tmem_ld_16x256b_x4x2_async(s_base, rs[0]);
+        tmem_ld_16x256b_x4x2_async(s_base + 32, rs[1]);
+        tmem_wait_ld(rs[0]);
+        tmem_regs_ready(rs[1]);
+        tc_fence_before_sync();
+        __syncwarp();
+        if (lane == 0) arrive_issuer<kPair>(&sm.bar_sread[buf]);
+#pragma unroll
         for (int h = 0; h < 2; ++h) {
-          const uint32_t s_addr = s_base + 32 * h;
           const int col0 = (e & kTileIdxMask) * kTileN + u * 64 + 32 * h;
           float pa[16], pb[16];  // rows lane/4 + {0, 8} and + {16, 24}
-          {
-            uint32_t r[32];
-            tmem_ld_16x256b_x4x2_async(s_addr, r);
-            tmem_wait_ld(r);
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-              pa[k] = __uint_as_float(r[k]);
-              pb[k] = __uint_as_float(r[16 + k]);
-            }
-          }
-          if (h == 1) {
-            // both halves of S are in registers: the S buffer may be overwritten
-            tc_fence_before_sync();
-            __syncwarp();
-            if (lane == 0) bar_arrive(&sm.bar_sread[buf]);
+          for (int k = 0; k < 16; ++k) {
+            pa[k] = __uint_as_float(rs[h][k]);
+            pb[k] = __uint_as_float(rs[h][16 + k]);
           }
           if (!partial) {
 #pragma unroll
@@ -570,8 +724,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           }
           if (h == 0 && t >= kPBufs) {
             // the P V of tile t - 2 must be done with this P buffer
-            if (!wait_bar(&sm.bar_pvdone[pbuf], ((t - kPBufs) / kPBufs) & 1, abort_flag,
-                          kWaitLimitNs)) {
+            if (!wait_b<kPair>(&sm.bar_pvdone[pbuf], ((t - kPBufs) / kPBufs) & 1, abort_flag)) {
               ok = false;
               break;
             }
@@ -584,13 +737,13 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
               pk[2 * k] = pack_bf16x2(pa[4 * k], pa[4 * k + 1]);
               pk[2 * k + 1] = pack_bf16x2(pa[4 * k + 2], pa[4 * k + 3]);
             }
-            tmem_st_16x128b_x4(p_base + 16 * h, pk);
+            tmem_st_16x128b_x4_async(p_base + 16 * h, pk);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               pk[2 * k] = pack_bf16x2(pb[4 * k], pb[4 * k + 1]);
               pk[2 * k + 1] = pack_bf16x2(pb[4 * k + 2], pb[4 * k + 3]);
             }
-            tmem_st_16x128b_x4(p_base + 16 * h + (16u << 16), pk);
+            tmem_st_16x128b_x4_async(p_base + 16 * h + (16u << 16), pk);
           }
           // column sums: 4 rows in-thread, then a reduce-scatter over lane bits
           // 4, 3, 2 leaves one column (summed over the warp's 32 rows) per lane
@@ -606,19 +759,25 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           sm.colsum[cb][wg][q4][32 * h + cl] = v[0];
         }
         if (!ok) break;
+        tmem_wait_st();
         tc_fence_before_sync();
         __syncwarp();
+        if (lane == 0) arrive_issuer<kPair>(&sm.bar_pfull[pbuf]);
+        // The last of the warpgroup's four warps to get here adds the four
+        // quarters' partial sums per query head and issues the reductions; the
+        // others go straight on to their next tile.  The counter only grows
+        // (four per tile), so "last" is old % 4 == 3.  Buffer cb is written
+        // again two tiles later, by a warp that has waited for the P V of the
+        // tile in between, which needed this warp's pfull arrival for that
+        // tile, which comes after the reads below in program order.
+        int last = 0;
         if (lane == 0) {
-          bar_arrive(&sm.bar_pfull[pbuf]);
-          bar_arrive(&sm.bar_cs[cb][wg]);
+          __threadfence_block();
+          last = (atomicAdd(&sm.cs_count[cb][wg], 1u) & 3u) == 3u;
+          __threadfence_block();
         }
-        if (!wait_bar(&sm.bar_cs[cb][wg], (k2 >> 1) & 1, abort_flag, kWaitLimitNs)) {
-          ok = false;
-          break;
-        }
-        // one warp of the warpgroup (a different one every tile) adds the four
-        // quarters' partial sums per query head and issues the reductions
-        if (q4 == (k2 & 3)) {
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (last) {
           const int colb = (e & kTileIdxMask) * kTileN + u * 64;
 #pragma unroll
           for (int hh = 0; hh < 2; ++hh) {
@@ -651,10 +810,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       if (lane == 0) bar_arrive(&sm.bar_rowstat);
     }
     // ------------------------------------------------------------ epilogue --
-    if (ok && n_t > 0 && wait_bar(&sm.bar_ofull, 0, abort_flag, kWaitLimitNs)) {
+    if (ok && n_t > 0 && wait_b<kPair>(&sm.bar_ofull, 0, abort_flag)) {
       tc_fence_after_sync();
       constexpr int kPart = D / kNumWG;  // O columns per warpgroup: 32 or 16
-      uint16_t* dst = a.out + (static_cast<size_t>(b * a.Hq + hq) * a.S + i) * D + wg * kPart;
       uint32_t pk[kPart / 2];
       if constexpr (kPart == 32) {
         uint32_t r[32];
@@ -670,6 +828,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           pk[x] = pack_bf16x2(__uint_as_float(r[2 * x]), __uint_as_float(r[2 * x + 1]));
       }
       if (valid) {
+        uint16_t* dst = a.out + (static_cast<size_t>(b * a.Hq + hq) * a.S + i) * D + wg * kPart;
         uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
         for (int x = 0; x < kPart / 8; ++x)
@@ -679,35 +838,50 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
   }
   tc_fence_before_sync();
   __syncthreads();
+  // On a pair, neither CTA frees TMEM or leaves (its shared memory holds
+  // barriers and operands the other one uses) before both are done.
+  if constexpr (kPair) cluster_sync_all();
   if (warp == 1) {
     __syncwarp();
-    tmem_dealloc(tmem, 512);
+    if constexpr (kPair) tmem_dealloc_pair(tmem, 512);
+    else tmem_dealloc(tmem, 512);
   }
   if (tid == 0 && sm.abort_flag) atomicOr(a.err, 1);
 }
 
-template <int D>
+template <int D, bool kPair>
 cudaError_t launch_d(const SdpaArgs& a, cudaStream_t stream) {
-  const size_t smem = sizeof(SdpaSmem<D>) + 1024;
+  const size_t smem = sizeof(SdpaSmem<D, kPair>) + 1024;
   static bool configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 64 && !configured[dev]) {
-    e = cudaFuncSetAttribute(sdpa_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem));
+    e = cudaFuncSetAttribute(sdpa_chunk_kernel<D, kPair>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  dim3 grid(a.n_row_tiles, a.B * a.Hkv);
-  sdpa_chunk_kernel<D><<<grid, kThreads, smem, stream>>>(a);
-  return cudaGetLastError();
+  const int ctas = kPair ? 2 * ((a.n_row_tiles + 1) / 2) : a.n_row_tiles;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas), static_cast<unsigned>(a.B * a.Hkv));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kPair ? 2 : 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, sdpa_chunk_kernel<D, kPair>, a);
 }
 
 }  // namespace
 
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream) {
-  return a.d == 64 ? launch_d<64>(a, stream) : launch_d<128>(a, stream);
+  return a.d == 64 ? launch_d<64, false>(a, stream) : launch_d<128, true>(a, stream);
 }
 
 }  // namespace h2o

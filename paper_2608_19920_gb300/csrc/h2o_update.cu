@@ -230,17 +230,6 @@ constexpr int kCThreads = 512;
 constexpr int kCWarps = kCThreads / 32;
 constexpr int kMaxSmemSlots = 24576;
 
-__device__ __forceinline__ void cluster_sync_all() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
-               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-
 // Exclusive prefix sum over the block of one value per thread.
 __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_tot,
                                                     uint32_t* total) {

@@ -42,15 +42,29 @@ __device__ __forceinline__ void bar_expect_tx(uint64_t* bar, uint32_t bytes) {
                : "memory");
 }
 
-__device__ __forceinline__ bool bar_try_wait(uint64_t* bar, uint32_t parity) {
+// One test of the phase; if it is not complete the thread is suspended in
+// hardware until it completes or `suspend_ns` pass, so a waiting warp takes no
+// issue slots from the warps that share its scheduler.
+__device__ __forceinline__ bool bar_try_wait(uint64_t* bar, uint32_t parity,
+                                             uint32_t suspend_ns = 0) {
   uint32_t done;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(done)
-      : "r"(smem_addr(bar)), "r"(parity)
-      : "memory");
+  if (suspend_ns == 0) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+  } else {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity), "r"(suspend_ns)
+        : "memory");
+  }
   return done != 0;
 }
 
@@ -68,6 +82,35 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatil
       return false;
     }
   }
+}
+
+// --------------------------------------------------------------- clusters --
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// shared::cluster address of the object at `p` (this CTA's shared memory) in
+// the CTA of the cluster with rank `cta`.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t cta) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(cta));
+  return r;
+}
+
+// Arrive on an mbarrier given by shared::cluster address (possibly in another
+// CTA of the cluster).  Default semantics (release at CTA scope): enough to
+// order this thread's tcgen05 operations (after tcgen05.fence::before_thread_sync)
+// before the waiter's, without waiting for its outstanding global writes the
+// way a cluster-scope release would.
+__device__ __forceinline__ void bar_arrive_remote(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 
 // -------------------------------------------------------------------- TMA --
@@ -90,6 +133,27 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
       "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_addr(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_addr(bar)), "r"(x), "r"(y), "r"(z), "r"(w)
+      : "memory");
+}
+
+// TMA loads of a CTA pair (.cta_group::2): the data lands in this CTA's shared
+// memory, the transaction bytes are counted on the mbarrier given by its
+// shared::cluster address, which may be in the other CTA of the pair.
+__device__ __forceinline__ void tma_load_3d_pair(void* dst, const CUtensorMap* map,
+                                                 uint32_t bar_cluster, int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d_pair(void* dst, const CUtensorMap* map,
+                                                 uint32_t bar_cluster, int x, int y, int z, int w) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y), "r"(z), "r"(w)
       : "memory");
 }
 
@@ -117,6 +181,24 @@ __device__ __forceinline__ void tc_fence_before_sync() {
 
 __device__ __forceinline__ void tc_fence_after_sync() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// CTA-pair TMEM management: one warp of EACH CTA of the pair issues these
+// together; the allocation is made at the same columns in both CTAs.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_addr(dst_smem)),
+               "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
 }
 
 // Instruction descriptor of tcgen05.mma kind::f16: bf16 x bf16 -> f32.
@@ -164,6 +246,100 @@ __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_
       "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+
+// CTA-pair MMAs (issued by one thread of the even CTA): M = 256, rows 0-127
+// from / into the even CTA, rows 128-255 from / into the odd one; B is split
+// along N, its first N/2 columns in the even CTA's shared memory and the rest
+// at the same offset in the odd CTA's.
+__device__ __forceinline__ void mma_ss_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_ts_pair(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives on the mbarrier at `bar`'s offset in every CTA of `cta_mask` once
+// every pair MMA issued so far by this thread has completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_addr(bar)),
+      "h"(cta_mask)
+      : "memory");
+}
+
+// Eight MMAs issued back to back from one asm block, so that no dependent
+// arithmetic separates them: the issuing thread only runs about one MMA ahead
+// of the tensor pipe, and every instruction between two MMAs leaves it idle.
+// The first MMA accumulates into D iff acc_first != 0, the rest always do.
+#define H2O_MMA8(KIND_A, A0, A1, A2, A3, A4, A5, A6, A7)                                  \
+  "{\n\t.reg .pred p0, p1;\n\t"                                                           \
+  "setp.ne.b32 p0, %2, 0;\n\t"                                                            \
+  "setp.eq.b32 p1, %2, %2;\n\t"                                                           \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A0 ", %4, %1, p0;\n\t"             \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A1 ", %5, %1, p1;\n\t"             \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A2 ", %6, %1, p1;\n\t"             \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A3 ", %7, %1, p1;\n\t"             \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A4 ", %8, %1, p1;\n\t"             \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A5 ", %9, %1, p1;\n\t"             \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A6 ", %10, %1, p1;\n\t"            \
+  "tcgen05.mma.cta_group::" KIND_A ".kind::f16 [%0], " A7 ", %11, %1, p1;\n\t}"
+
+// D (+)= sum_k A_k B_k^T over eight K-steps, A and B from shared memory.
+template <bool kPair>
+__device__ __forceinline__ void mma_ss_x8(uint32_t d_tmem, const uint64_t (&a)[8],
+                                          const uint64_t (&b)[8], uint32_t idesc,
+                                          uint32_t acc_first) {
+  if constexpr (kPair) {
+    asm volatile(H2O_MMA8("2", "%3", "%12", "%13", "%14", "%15", "%16", "%17", "%18")
+                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "l"(a[0]), "l"(b[0]), "l"(b[1]),
+                 "l"(b[2]), "l"(b[3]), "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]), "l"(a[1]),
+                 "l"(a[2]), "l"(a[3]), "l"(a[4]), "l"(a[5]), "l"(a[6]), "l"(a[7])
+                 : "memory");
+  } else {
+    asm volatile(H2O_MMA8("1", "%3", "%12", "%13", "%14", "%15", "%16", "%17", "%18")
+                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "l"(a[0]), "l"(b[0]), "l"(b[1]),
+                 "l"(b[2]), "l"(b[3]), "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]), "l"(a[1]),
+                 "l"(a[2]), "l"(a[3]), "l"(a[4]), "l"(a[5]), "l"(a[6]), "l"(a[7])
+                 : "memory");
+  }
+}
+
+// D (+)= sum_k A_k B_k over eight K-steps, A from TMEM (columns a_tmem + 8k),
+// B from shared memory.
+template <bool kPair>
+__device__ __forceinline__ void mma_ts_x8(uint32_t d_tmem, uint32_t a_tmem, const uint64_t (&b)[8],
+                                          uint32_t idesc, uint32_t acc_first) {
+  const uint32_t a1 = a_tmem + 8, a2 = a_tmem + 16, a3 = a_tmem + 24, a4 = a_tmem + 32,
+                 a5 = a_tmem + 40, a6 = a_tmem + 48, a7 = a_tmem + 56;
+  if constexpr (kPair) {
+    asm volatile(H2O_MMA8("2", "[%3]", "[%12]", "[%13]", "[%14]", "[%15]", "[%16]", "[%17]", "[%18]")
+                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "r"(a_tmem), "l"(b[0]), "l"(b[1]),
+                 "l"(b[2]), "l"(b[3]), "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]), "r"(a1),
+                 "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
+                 : "memory");
+  } else {
+    asm volatile(H2O_MMA8("1", "[%3]", "[%12]", "[%13]", "[%14]", "[%15]", "[%16]", "[%17]", "[%18]")
+                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "r"(a_tmem), "l"(b[0]), "l"(b[1]),
+                 "l"(b[2]), "l"(b[3]), "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]), "r"(a1),
+                 "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
+                 : "memory");
+  }
+}
+#undef H2O_MMA8
 
 // Arrives on `bar` once every MMA issued so far by this thread has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
@@ -310,6 +486,29 @@ __device__ __forceinline__ void tmem_ld_16x256b_x4x2_async(uint32_t taddr, uint3
 
 __device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+
+// tcgen05.st of 16x128b.x4 without waiting for completion; the source
+// registers may be reused at once, but the stored columns are only visible to
+// later tcgen05 operations after tmem_wait_st().
+__device__ __forceinline__ void tmem_st_16x128b_x4_async(uint32_t taddr, const uint32_t (&r)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.16x128b.x4.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Compiler-only barrier on 32 registers loaded by an async tcgen05.ld whose
+// completion an earlier tmem_wait_ld() (which waits for all of this thread's
+// loads) has already covered: keeps their reads after that wait.
+__device__ __forceinline__ void tmem_regs_ready(uint32_t (&r)[32]) {
+  asm volatile(""
                : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
                :
                : "memory");

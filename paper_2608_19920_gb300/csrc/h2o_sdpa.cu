@@ -30,10 +30,10 @@
 //    the other waits on a barrier; warps 3-18 form four softmax
 //    warpgroups in two teams that take alternate tiles; the two warpgroups of a
 //    team own key columns 0-63 and 64-127 of their tiles.
-//  * TMEM holds two fp32 S buffers, two bf16 P buffers and the O accumulator.
-//    An S buffer is released as soon as the softmax has loaded it, so Q K^T of
-//    later tiles never waits for P V; P is written as bf16 pairs into a P
-//    buffer and consumed by the P V MMA directly from TMEM.
+//  * TMEM: pass 1 uses four fp32 S buffers; pass 2 three S buffers and the O
+//    accumulator.  In pass 2 the bf16 P of a tile is written over the S
+//    columns it came from (each warpgroup over its own), and the P V MMA reads
+//    it there, so storing P never waits for an earlier P V.
 //  * Column sums use the fp32 P (not the bf16 copy fed to the MMA).  Pass 2
 //    reads S in TMEM's 16x256b layout, where a thread holds 4 rows x 8
 //    columns: it adds its 4 rows, a 3-step warp reduce-scatter leaves one
@@ -64,14 +64,18 @@ constexpr uint16_t kTilePartial = 0x4000;
 constexpr uint16_t kTileIdxMask = 0x3FFF;
 constexpr uint8_t kClsSkip = 0, kClsFull = 1, kClsPartial = 2;
 // TMEM (512 columns).  Pass 1 needs no P or O: four S buffers (fp32, 128
-// columns each).  Pass 2: S buffers 0 and 1, two P buffers (bf16 pairs, 64
-// columns each) over the columns of S buffer 2, and the O accumulator over
-// those of S buffer 3.  An S buffer is free again as soon as the softmax has
-// loaded it; a P buffer when the P V that read it has completed.
+// columns each), each free again as soon as the softmax has loaded it.
+// Pass 2: three S buffers and the O accumulator (columns 384..).  The softmax
+// loads a tile's S, then writes the bf16 P of warpgroup u's 64 keys as pairs
+// into columns 64u .. 64u+31 of the same buffer (columns only that warpgroup
+// loaded), where the P V MMA reads it; the buffer is free again when that P V
+// has completed.  So writing P never waits for an earlier P V.
 constexpr int kSBufs1 = 4;
-constexpr int kSBufs = 2;
-constexpr int kPBufs = 2;
-constexpr int kPCols = kTileN / 2;
+constexpr int kSBufs2 = 3;
+
+__device__ __forceinline__ int pass1_buffer_uses(int n_t, int b) {
+  return n_t > b ? (n_t - 1 - b) / kSBufs1 + 1 : 0;
+}
 
 // S buffer of step n (pass-1 tile n < n_t, pass-2 tile n - n_t) and how many
 // times that buffer was filled before.
@@ -80,8 +84,8 @@ __device__ __forceinline__ void s_buffer(int n, int n_t, int& buf, int& use) {
     buf = n % kSBufs1;
     use = n / kSBufs1;
   } else {
-    buf = (n - n_t) % kSBufs;
-    use = (n_t > buf ? (n_t - 1 - buf) / kSBufs1 + 1 : 0) + (n - n_t) / kSBufs;
+    buf = (n - n_t) % kSBufs2;
+    use = pass1_buffer_uses(n_t, buf) + (n - n_t) / kSBufs2;
   }
 }
 
@@ -120,7 +124,7 @@ struct __align__(1024) SdpaSmem {
   float rowstat[kNumWG][kTileM][2];
   uint64_t bar_q;
   uint64_t bar_full[G::kR], bar_empty[G::kR];
-  uint64_t bar_sfull[kSBufs1], bar_sread[kSBufs1], bar_pfull[kPBufs], bar_pvdone[kPBufs];
+  uint64_t bar_sfull[kSBufs1], bar_sread[kSBufs1], bar_pfull[kSBufs2], bar_pvdone[kSBufs2];
   uint64_t bar_rowstat, bar_ofull, bar_drain[2], bar_p1done;
   uint32_t cs_count[2][kNumWG];  // column-sum partials deposited (4 per tile)
   uint32_t taddr;
@@ -218,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       // the 8 warps of the team owning the tile, in every CTA of the pair
       bar_init(&sm.bar_sread[x], G::kCtas * kSoftmaxWarps / 2);
     }
-    for (int x = 0; x < kPBufs; ++x) {
+    for (int x = 0; x < kSBufs2; ++x) {
       bar_init(&sm.bar_pfull[x], G::kCtas * kSoftmaxWarps / 2);
       bar_init(&sm.bar_pvdone[x], 1);
     }
@@ -315,9 +319,8 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
 
   const uint32_t tmem = sm.taddr;
   const uint32_t tS = tmem;                          // S buffer b: columns 128 b ..
-  const uint32_t tP = tmem + 128 * kSBufs;           // P buffer p: columns 256 + 64 p ..
-  const uint32_t tO = tP + kPCols * kPBufs;          // O accumulator: columns 384 ..
-  static_assert(128 * kSBufs + kPCols * kPBufs + 128 == 128 * kSBufs1, "TMEM layout");
+  const uint32_t tO = tmem + 128 * kSBufs2;          // O accumulator: columns 384 ..
+  static_assert(128 * kSBufs2 + 128 == 128 * kSBufs1, "TMEM layout");
   const int n_t = sm.n_tiles;
   volatile int* abort_flag = &sm.abort_flag;
 
@@ -426,9 +429,15 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       auto issue_qk = [&](int n) -> bool {
         int buf, suse;
         s_buffer(n, n_t, buf, suse);
-        // buffer reuse: the softmax has loaded the buffer's previous S
-        if (suse > 0 && !wait_b<kPair>(&sm.bar_sread[buf], (suse - 1) & 1, abort_flag))
-          return false;
+        // buffer reuse: a pass-1 S is released when the softmax has loaded
+        // it, a pass-2 one when the P V that read its P has completed
+        if (suse > 0) {
+          const int c1 = pass1_buffer_uses(n_t, buf);
+          const bool ok_wait =
+              suse <= c1 ? wait_b<kPair>(&sm.bar_sread[buf], (suse - 1) & 1, abort_flag)
+                         : wait_b<kPair>(&sm.bar_pvdone[buf], (suse - 1 - c1) & 1, abort_flag);
+          if (!ok_wait) return false;
+        }
         int s, use;
         if (n < n_t) {
           s = n % (RA + RB);
@@ -469,8 +478,8 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         bar_arrive(&sm.bar_p1done);
         const uint64_t v_desc0 = sdesc_sw128(smem_addr(sm.kv[RA]), kTileN * 128, 1024);
         for (int t = 0; ok && t < n_t; ++t) {
-          const int pb = t % kPBufs;
-          if (!wait_b<kPair>(&sm.bar_pfull[pb], (t / kPBufs) & 1, abort_flag)) {
+          const int pb = t % kSBufs2;  // the S buffer of pass-2 tile t holds its P
+          if (!wait_b<kPair>(&sm.bar_pfull[pb], (t / kSBufs2) & 1, abort_flag)) {
             ok = false;
             break;
           }
@@ -485,8 +494,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           uint64_t bd[8];
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) bd[kk] = vd + 128 * kk;
-          // keys 16kk..16kk+15 sit as bf16 pairs in columns 8kk..8kk+7 of the P buffer
-          mma_ts_x8<kPair>(tO, tP + kPCols * pb, bd, kIdescPV, t > 0 ? 1u : 0u);
+          // keys 0-63 (16 per K-step) as bf16 pairs in columns 0-31 of the
+          // buffer, keys 64-127 in columns 64-95
+          mma_ts_x8<kPair>(tO, tS + 128 * pb, tS + 128 * pb + 64, bd, kIdescPV, t > 0 ? 1u : 0u);
           commit_all<kPair>(&sm.bar_empty[vs]);
           commit_all<kPair>(&sm.bar_pvdone[pb]);
         }
@@ -672,18 +682,14 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         // pass 2 (16x256b layout), in two halves of 32 columns: P in fp32,
         // bf16 copy to a TMEM P buffer for P V, column sums of the fp32 P
         const int cb = k2 & 1;
-        const int pbuf = t % kPBufs;
-        const uint32_t p_base = tP + lane_addr + kPCols * pbuf + u * 32;
-        // both 32-column halves of S are loaded before any is processed, so
-        // the S buffer is released at once
+        // P goes over this warpgroup's own S columns: 64 keys -> 32 columns
+        const uint32_t p_base = s_base;
+        // both 32-column halves of S are loaded before P overwrites the first
         uint32_t rs[2][32];
         tmem_ld_16x256b_x4x2_async(s_base, rs[0]);
         tmem_ld_16x256b_x4x2_async(s_base + 32, rs[1]);
         tmem_wait_ld(rs[0]);
         tmem_regs_ready(rs[1]);
-        tc_fence_before_sync();
-        __syncwarp();
-        if (lane == 0) arrive_issuer<kPair>(&sm.bar_sread[buf]);
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int col0 = (e & kTileIdxMask) * kTileN + u * 64 + 32 * h;
@@ -722,14 +728,6 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
               }
             }
           }
-          if (h == 0 && t >= kPBufs) {
-            // the P V of tile t - 2 must be done with this P buffer
-            if (!wait_b<kPair>(&sm.bar_pvdone[pbuf], ((t - kPBufs) / kPBufs) & 1, abort_flag)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after_sync();
-          }
           {
             uint32_t pk[8];
 #pragma unroll
@@ -762,7 +760,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         tmem_wait_st();
         tc_fence_before_sync();
         __syncwarp();
-        if (lane == 0) arrive_issuer<kPair>(&sm.bar_pfull[pbuf]);
+        if (lane == 0) arrive_issuer<kPair>(&sm.bar_pfull[buf]);
         // The last of the warpgroup's four warps to get here adds the four
         // quarters' partial sums per query head and issues the reductions; the
         // others go straight on to their next tile.  The counter only grows

@@ -318,13 +318,14 @@ __device__ __forceinline__ void mma_ss_x8(uint32_t d_tmem, const uint64_t (&a)[8
   }
 }
 
-// D (+)= sum_k A_k B_k over eight K-steps, A from TMEM (columns a_tmem + 8k),
-// B from shared memory.
+// D (+)= sum_k A_k B_k over eight K-steps, A from TMEM (K-steps 0-3 at
+// columns a_lo + 8k, K-steps 4-7 at a_hi + 8(k - 4)), B from shared memory.
 template <bool kPair>
-__device__ __forceinline__ void mma_ts_x8(uint32_t d_tmem, uint32_t a_tmem, const uint64_t (&b)[8],
-                                          uint32_t idesc, uint32_t acc_first) {
-  const uint32_t a1 = a_tmem + 8, a2 = a_tmem + 16, a3 = a_tmem + 24, a4 = a_tmem + 32,
-                 a5 = a_tmem + 40, a6 = a_tmem + 48, a7 = a_tmem + 56;
+__device__ __forceinline__ void mma_ts_x8(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi,
+                                          const uint64_t (&b)[8], uint32_t idesc,
+                                          uint32_t acc_first) {
+  const uint32_t a_tmem = a_lo, a1 = a_lo + 8, a2 = a_lo + 16, a3 = a_lo + 24, a4 = a_hi,
+                 a5 = a_hi + 8, a6 = a_hi + 16, a7 = a_hi + 24;
   if constexpr (kPair) {
     asm volatile(H2O_MMA8("2", "[%3]", "[%12]", "[%13]", "[%14]", "[%15]", "[%16]", "[%17]", "[%18]")
                  ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "r"(a_tmem), "l"(b[0]), "l"(b[1]),

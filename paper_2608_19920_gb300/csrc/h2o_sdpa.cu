@@ -682,22 +682,24 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         // pass 2 (16x256b layout), in two halves of 32 columns: P in fp32,
         // bf16 copy to a TMEM P buffer for P V, column sums of the fp32 P
         const int cb = k2 & 1;
-        // P goes over this warpgroup's own S columns: 64 keys -> 32 columns
+        // P goes over this warpgroup's own S columns: its 64 keys as bf16
+        // pairs in columns 0-31 of the group's range, which hold the S of half
+        // 0; half 0 is loaded before any P is stored, half 1 (columns 32-63)
+        // is never overwritten.
         const uint32_t p_base = s_base;
-        // both 32-column halves of S are loaded before P overwrites the first
-        uint32_t rs[2][32];
-        tmem_ld_16x256b_x4x2_async(s_base, rs[0]);
-        tmem_ld_16x256b_x4x2_async(s_base + 32, rs[1]);
-        tmem_wait_ld(rs[0]);
-        tmem_regs_ready(rs[1]);
-#pragma unroll
+#pragma unroll 1
         for (int h = 0; h < 2; ++h) {
           const int col0 = (e & kTileIdxMask) * kTileN + u * 64 + 32 * h;
           float pa[16], pb[16];  // rows lane/4 + {0, 8} and + {16, 24}
+          {
+            uint32_t r[32];
+            tmem_ld_16x256b_x4x2_async(s_base + 32 * h, r);
+            tmem_wait_ld(r);
 #pragma unroll
-          for (int k = 0; k < 16; ++k) {
-            pa[k] = __uint_as_float(rs[h][k]);
-            pb[k] = __uint_as_float(rs[h][16 + k]);
+            for (int k = 0; k < 16; ++k) {
+              pa[k] = __uint_as_float(r[k]);
+              pb[k] = __uint_as_float(r[16 + k]);
+            }
           }
           if (!partial) {
 #pragma unroll
@@ -769,13 +771,10 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         // tile in between, which needed this warp's pfull arrival for that
         // tile, which comes after the reads below in program order.
         int last = 0;
-        if (lane == 0) {
-          __threadfence_block();
-          last = (atomicAdd(&sm.cs_count[cb][wg], 1u) & 3u) == 3u;
-          __threadfence_block();
-        }
+        if (lane == 0) last = (atomic_add_acq_rel_cta(&sm.cs_count[cb][wg], 1u) & 3u) == 3u;
         last = __shfl_sync(0xffffffffu, last, 0);
         if (last) {
+          __syncwarp();
           const int colb = (e & kTileIdxMask) * kTileN + u * 64;
 #pragma unroll
           for (int hh = 0; hh < 2; ++hh) {

@@ -505,14 +505,16 @@ __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// Compiler-only barrier on 32 registers loaded by an async tcgen05.ld whose
-// completion an earlier tmem_wait_ld() (which waits for all of this thread's
-// loads) has already covered: keeps their reads after that wait.
-__device__ __forceinline__ void tmem_regs_ready(uint32_t (&r)[32]) {
-  asm volatile(""
-               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
-               :
+// Shared-memory atomic add with acquire-release semantics at CTA scope:
+// writes before it (by this thread, or ordered before it by a warp or block
+// barrier) are visible to a thread whose later atomic reads its result.
+__device__ __forceinline__ uint32_t atomic_add_acq_rel_cta(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], %2;"
+               : "=r"(old)
+               : "r"(smem_addr(p)), "r"(v)
                : "memory");
+  return old;
 }
 
 // Packs two floats into bf16x2 (round to nearest even): `lo` in bits 0-15.

@@ -19,6 +19,7 @@ over ranks and rank 0 prints.
 from __future__ import annotations
 
 import argparse
+import datetime
 import json
 import math
 import os
@@ -70,8 +71,9 @@ def peaks():
 
 # ---------------------------------------------------------------- clocks --
 class ClockSampler:
-    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi clocks / throttle reasons, sampled every 20 ms; only samples
+    whose timestamps fall inside [mark_start, mark_end] are summarised."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -79,25 +81,44 @@ class ClockSampler:
         self.gpu = gpu_index
         self.proc = None
         self.file = None
+        self.t_start = self.t_end = None
 
     def __enter__(self):
         try:
             self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=self.file, stderr=subprocess.DEVNULL)
+            # sampling must be running before the timed region starts
+            deadline = time.time() + 5.0
+            while time.time() < deadline and os.path.getsize(self.file.name) == 0:
+                time.sleep(0.02)
         except (OSError, FileNotFoundError):
             self.proc = None
         return self
 
+    def mark_start(self):
+        self.t_start = time.time()
+
+    def mark_end(self):
+        self.t_end = time.time()
+
     def __exit__(self, *exc):
         if self.proc is not None:
+            time.sleep(0.05)
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
+
+    @staticmethod
+    def _stamp(x):
+        try:
+            return datetime.datetime.strptime(x, "%Y/%m/%d %H:%M:%S.%f").timestamp()
+        except ValueError:
+            return None
 
     def summary(self):
         if self.proc is None or self.file is None:
@@ -107,23 +128,41 @@ class ClockSampler:
         with open(self.file.name) as f:
             for line in f:
                 parts = [x.strip() for x in line.split(",")]
-                if len(parts) >= 9:
+                if len(parts) >= 10:
                     rows.append(parts)
         os.unlink(self.file.name)
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        inside = []
+        if self.t_start is not None and self.t_end is not None:
+            for r in rows:
+                t = self._stamp(r[0])
+                if t is not None and self.t_start <= t <= self.t_end:
+                    inside.append(r)
+        note = None
+        if not inside:
+            # timed region shorter than the sampling period: nearest sample
+            mid = 0.5 * ((self.t_start or 0.0) + (self.t_end or 0.0))
+            inside = [min(rows, key=lambda r: abs((self._stamp(r[0]) or 0.0) - mid))]
+            note = "no sample inside the timed region; nearest sample used"
 
         def num(x):
             try:
                 return float(x)
             except ValueError:
                 return None
-        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
-        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        sm = [num(r[2]) for r in inside if num(r[2]) is not None]
+        mx = [num(r[3]) for r in inside if num(r[3]) is not None]
+        pw = [num(r[4]) for r in inside if num(r[4]) is not None]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
-        return {"sm_mhz": statistics.median(sm) if sm else None,
-                "sm_max_mhz": max(mx) if mx else None, "samples": len(rows), "reasons": reasons}
+        reasons = sorted({names[i] for r in inside for i in range(4) if r[6 + i].lower() == "active"})
+        out = {"sm_mhz": statistics.median(sm) if sm else None,
+               "sm_max_mhz": max(mx) if mx else None,
+               "power_w": statistics.median(pw) if pw else None,
+               "samples": len(inside) if note is None else 0, "reasons": reasons}
+        if note:
+            out["note"] = note
+        return out
 
 
 # ------------------------------------------------------------ distributed --
@@ -278,11 +317,13 @@ def run_ours(args, w):
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
+        clk.mark_start()
         t0.record(stream)
         for s in range(args.steps):
             one_step(record=(s == args.steps - 1))
         t1.record(stream)
         torch.cuda.synchronize()
+        clk.mark_end()
     elapsed_ms = t0.elapsed_time(t1)
     barrier(world)
     elapsed_ms = max_over_ranks(elapsed_ms, world)
@@ -314,11 +355,15 @@ def run_ours(args, w):
         "gpu_launches": args.steps * (2 * len(plan)),
         "clocks": clocks,
     }
+    # the chunk SDPA is timed on its own (launch after launch, L2 flushed in
+    # between): its denominator is the burst peak; the sustained one is given
+    # alongside
     line["roofline"] = {
-        "bound": "tensor", "kernel": "sdpa_chunk_kernel<128> (steady-state chunk)",
-        "achieved": kern["alg_tflops"], "peak": pk["bf16_sus"], "unit": "TFLOP/s",
-        "frac": kern["alg_tflops"] / pk["bf16_sus"], "traffic": args.traffic,
-        "peak_source": f"{pk['source']} bf16 dense, sustained",
+        "bound": "tensor", "kernel": "sdpa_chunk_kernel<128,pair> (steady-state chunk)",
+        "achieved": kern["alg_tflops"], "peak": pk["bf16"], "unit": "TFLOP/s",
+        "frac": kern["alg_tflops"] / pk["bf16"], "traffic": args.traffic,
+        "peak_source": f"{pk['source']} bf16 dense, burst",
+        "frac_of_sustained": kern["alg_tflops"] / pk["bf16_sus"],
         "avg_launch_us": kern["avg_us"], "flops_per_launch": kern["flops"],
         "executed_tflops": kern["alg_tflops"] * kern["exec_ratio"],
     }
@@ -341,9 +386,14 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
     out = torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=q.device)
     inc = torch.empty((w.B, w.Hq, w.M + e - p), dtype=torch.float32, device=q.device)
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
+    clean = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
     times = []
     for _ in range(reps + 2):
-        flush.zero_()  # evict the previous launch's data from L2
+        # Evict the previous launch's data from L2 by writing a buffer twice
+        # its size, then read another one so that the write-back of those
+        # dirty lines happens here, not inside the timed launch.
+        flush.zero_()
+        clean.sum()
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
@@ -414,7 +464,7 @@ def run_e2e(w, layer, plan, outs, dev, args, world):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama8b_32k", choices=sorted(wl.WORKLOADS))

@@ -20,11 +20,16 @@
 //     writes slot_pos, scores, evict_idx; whole warps copy the K and V rows of
 //     the evicted slots with 16-byte vector loads and stores.
 //
-// Two variants.  When the keys of one (b, kv head) fit in shared memory and
-// S > 1, a cluster of C CTAs handles the (b, kv head): every CTA computes the
-// keys into shared memory and runs the same deterministic selection, a cluster
+// Two variants.  When the keys and accumulated scores of one (b, kv head)
+// fit in shared memory and S > 1, a cluster of C CTAs handles the (b, kv
+// head): every CTA computes keys and scores into shared memory (each thread
+// owns a contiguous run of slots and issues all loads of a batch before the
+// first sum), runs the same deterministic selection (one packed scan of the
+// counts below and equal to the threshold gives every slot's rank), a cluster
 // barrier separates all reads of the old state from the writes, CTA 0 writes
-// scores / slot_pos / evict_idx, and the C CTAs share the row copies.
+// scores / slot_pos / evict_idx, and the C CTAs share the row copies with
+// several 16-byte loads in flight per thread.  The whole update is latency
+// bound (a few MB per chunk), so the design minimises dependent round trips.
 // Otherwise one CTA per (b, kv head) recomputes keys from global memory on
 // every pass (S = 1 takes the argmin path).
 #include "h2o_internal.h"
@@ -228,7 +233,10 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
 // ----------------------------------------------------- cluster variant --
 constexpr int kCThreads = 512;
 constexpr int kCWarps = kCThreads / 32;
-constexpr int kMaxSmemSlots = 24576;
+// dynamic shared memory of the cluster variant: keys and scores of the M
+// slots, scores and evicted slots of the S new tokens (M < 25600 < 65536,
+// which the packed 16-bit counts of phase 3 need)
+constexpr size_t kMaxClusterSmem = 200 * 1024;
 
 // Exclusive prefix sum over the block of one value per thread.
 __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_tot,
@@ -258,6 +266,11 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_t
   return base + incl - v;
 }
 
+// Loads of up to kMaxQg query heads are issued before their sum is formed.
+constexpr int kMaxQg = 8;
+// Slots a thread handles per batch of loads in phase 1.
+constexpr int kBatch = 8;
+
 __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const UpdateArgs a, int C) {
   extern __shared__ uint32_t dyn[];
   __shared__ uint32_t hist[256];
@@ -267,28 +280,91 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   const int rank = static_cast<int>(cluster_rank());
   const int grp = blockIdx.x / C;
   const int b = grp / a.Hkv, h = grp % a.Hkv;
-  const int M = a.M, S = a.S;
+  const int M = a.M, S = a.S, NK = M + S, qg = a.qg;
   float* sc = a.scores + static_cast<size_t>(grp) * M;
   int* sp = a.slot_pos + static_cast<size_t>(grp) * M;
-  const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * a.qg) * (M + S);
+  const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK;
   const int thr = a.pos0 + S - a.W;
-  uint32_t* keys = dyn;                                   // [M]
-  int* elist = reinterpret_cast<int*>(dyn + M);           // [S] evicted slot of rank c
+  uint32_t* keys = dyn;                                          // [M]
+  float* accs = reinterpret_cast<float*>(dyn + M);               // [M] accumulated scores
+  float* nscore = reinterpret_cast<float*>(dyn + 2 * M);         // [S] score of new token c
+  int* elist = reinterpret_cast<int*>(dyn + 2 * M + S);          // [S] evicted slot of rank c
 
-  for (int j = tid; j < M; j += kCThreads) {
-    float acc;
-    keys[j] = slot_key(a, sc, sp, inc, j, thr, &acc);
+  // Thread t owns slots [t R, t R + R) in slot order.
+  const int R = (M + kCThreads - 1) / kCThreads;
+  const int j0 = min(M, tid * R), j1 = min(M, j0 + R);
+  // 16-byte loads need every row start (grp M, head rows of NK) and j0 aligned
+  const bool vec = R % 4 == 0 && M % 4 == 0 && NK % 4 == 0 && qg <= kMaxQg;
+
+  // Phase 1: acc_j = scores_j + (inc_0j + inc_1j + ...), fp32, heads in order
+  // (Eq. 3), and the selection key of every slot; each batch issues all of
+  // its loads before the first sum.
+  for (int jb = j0; jb < j1; jb += kBatch) {
+    const int n = min(kBatch, j1 - jb);
+    float sv[kBatch], tv[kBatch];
+    int pv[kBatch];
+    if (vec && n == kBatch) {
+      float4 s4[2], i4[kMaxQg][2];
+      int4 p4[2];
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        s4[q] = *reinterpret_cast<const float4*>(sc + jb + 4 * q);
+        p4[q] = *reinterpret_cast<const int4*>(sp + jb + 4 * q);
+      }
+#pragma unroll
+      for (int g = 0; g < kMaxQg; ++g)
+        if (g < qg)
+#pragma unroll
+          for (int q = 0; q < 2; ++q)
+            i4[g][q] = __ldg(reinterpret_cast<const float4*>(inc + static_cast<size_t>(g) * NK + jb) + q);
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        sv[4 * q] = s4[q].x; sv[4 * q + 1] = s4[q].y; sv[4 * q + 2] = s4[q].z; sv[4 * q + 3] = s4[q].w;
+        pv[4 * q] = p4[q].x; pv[4 * q + 1] = p4[q].y; pv[4 * q + 2] = p4[q].z; pv[4 * q + 3] = p4[q].w;
+        tv[4 * q] = i4[0][q].x; tv[4 * q + 1] = i4[0][q].y;
+        tv[4 * q + 2] = i4[0][q].z; tv[4 * q + 3] = i4[0][q].w;
+      }
+#pragma unroll
+      for (int g = 1; g < kMaxQg; ++g)
+        if (g < qg)
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            tv[4 * q] = __fadd_rn(tv[4 * q], i4[g][q].x);
+            tv[4 * q + 1] = __fadd_rn(tv[4 * q + 1], i4[g][q].y);
+            tv[4 * q + 2] = __fadd_rn(tv[4 * q + 2], i4[g][q].z);
+            tv[4 * q + 3] = __fadd_rn(tv[4 * q + 3], i4[g][q].w);
+          }
+    } else {
+      for (int k = 0; k < n; ++k) {
+        sv[k] = sc[jb + k];
+        pv[k] = sp[jb + k];
+        tv[k] = group_sum(inc, NK, qg, jb + k);
+      }
+    }
+    for (int k = 0; k < n; ++k) {
+      const float acc = __fadd_rn(sv[k], tv[k]);
+      const int pos = pv[k];
+      uint32_t key;
+      if (pos >= thr) key = kProtected;
+      else if (pos < 0) key = 0u;
+      else key = min(__float_as_uint(acc) + 1u, kProtected - 1u);
+      keys[jb + k] = key;
+      accs[jb + k] = acc;
+    }
   }
+  // scores of the new tokens: their own columns M + c, summed over the group
+  for (int c = tid; c < S; c += kCThreads) nscore[c] = group_sum(inc + M, NK, qg, c);
   // Every CTA of the cluster has read the old state before CTA 0 rewrites it.
   cluster_sync_all();
 
-  // radix select: the S-th smallest key T, and how many keys equal to T are taken
+  // Phase 2: radix select of the S-th smallest key T, and how many keys equal
+  // to T are taken (the lowest slots first).
   uint32_t prefix = 0, mask = 0, kth = static_cast<uint32_t>(S);
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
     for (int x = tid; x < 256; x += kCThreads) hist[x] = 0u;
     __syncthreads();
-    for (int j = tid; j < M; j += kCThreads) {
+    for (int j = j0; j < j1; ++j) {
       const uint32_t key = keys[j];
       if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
     }
@@ -328,64 +404,92 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   }
   const uint32_t T = prefix, take_eq = kth;
 
-  // ranks in slot order: thread t owns slots [t*R, t*R + R)
-  const int R = (M + kCThreads - 1) / kCThreads;
-  const int j0 = min(M, tid * R), j1 = min(M, j0 + R);
-  uint32_t n_eq = 0;
-  for (int j = j0; j < j1; ++j) n_eq += keys[j] == T;
-  uint32_t tot;
-  uint32_t eq_run = block_excl_scan(n_eq, warp_tot, &tot);
-  uint32_t n_sel = 0;
-  {
-    uint32_t e = eq_run;
-    for (int j = j0; j < j1; ++j) {
-      const uint32_t key = keys[j];
-      const bool eq = key == T;
-      n_sel += key < T || (eq && e < take_eq);
-      e += eq;
-    }
+  // Phase 3: one scan of (keys < T, keys == T) per thread, packed in 16-bit
+  // halves (M < 65536), gives each slot's eviction rank: the slots below T
+  // before it plus the taken slots equal to T before it.
+  uint32_t n_lt = 0, n_eq = 0;
+  for (int j = j0; j < j1; ++j) {
+    n_lt += keys[j] < T;
+    n_eq += keys[j] == T;
   }
-  uint32_t c = block_excl_scan(n_sel, warp_tot, &tot);
+  uint32_t tot;
+  const uint32_t before = block_excl_scan(n_lt | (n_eq << 16), warp_tot, &tot);
+  uint32_t lt_b = before & 0xFFFFu, eq_b = before >> 16;
+
+  // Phase 4: evicted slots get ranks 0..S-1; CTA 0 writes the new state.
   for (int j = j0; j < j1; ++j) {
     const uint32_t key = keys[j];
     const bool eq = key == T;
-    const bool sel = (key < T || (eq && eq_run < take_eq)) && c < static_cast<uint32_t>(S);
-    eq_run += eq;
+    const bool sel0 = key < T || (eq && eq_b < take_eq);
+    const uint32_t c = lt_b + min(eq_b, take_eq);
+    const bool sel = sel0 && c < static_cast<uint32_t>(S);
+    lt_b += key < T;
+    eq_b += eq;
     if (sel) {
       elist[c] = j;
       if (rank == 0) {
-        sc[j] = group_sum(inc + M, M + S, a.qg, static_cast<int>(c));
         sp[j] = a.pos0 + static_cast<int>(c);
         if (a.evict_idx) a.evict_idx[static_cast<size_t>(grp) * S + c] = j;
+        accs[j] = nscore[c];
       }
-      ++c;
-    } else if (rank == 0) {
-      sc[j] = __fadd_rn(sc[j], group_sum(inc, M + S, a.qg, j));
+    }
+  }
+  if (rank == 0) {
+    if (vec) {
+      for (int j = j0; j < j1; j += 4)
+        *reinterpret_cast<float4*>(sc + j) = *reinterpret_cast<const float4*>(accs + j);
+    } else {
+      for (int j = j0; j < j1; ++j) sc[j] = accs[j];
     }
   }
   __syncthreads();
-  // this CTA's share of the K/V row copies: ranks c = rank (mod C)
-  const int n_sel_tot = min(static_cast<int>(tot), S);
-  for (int cc = rank + C * warp; cc < n_sel_tot; cc += C * kCWarps)
-    copy_row(a, grp, cc, elist[cc], lane);
+
+  // Phase 5: this CTA's share of the K/V row copies (ranks c = rank mod C),
+  // 16-byte pieces, four loads in flight per thread before their stores.
+  const int n_sel = min(static_cast<int>((tot & 0xFFFFu) + min(tot >> 16, take_eq)), S);
+  const int rows = n_sel > rank ? (n_sel - 1 - rank) / C + 1 : 0;
+  const int vecs = a.d / 8;  // 16-byte pieces per row
+  const int pieces = rows * 2 * vecs;
+  for (int x0 = tid; x0 < pieces; x0 += 4 * kCThreads) {
+    uint4 v[4];
+    uint4* dst[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int x = x0 + u * kCThreads;
+      dst[u] = nullptr;
+      if (x < pieces) {
+        const int piece = x % vecs;
+        const int rv = x / vecs;           // row index * 2 + (0 = K, 1 = V)
+        const int cc = rank + C * (rv >> 1);
+        const bool is_v = rv & 1;
+        const uint16_t* src = (is_v ? a.v_new : a.k_new) + (static_cast<size_t>(grp) * S + cc) * a.d;
+        uint16_t* d = (is_v ? a.v_cache : a.k_cache) + (static_cast<size_t>(grp) * M + elist[cc]) * a.d;
+        v[u] = __ldg(reinterpret_cast<const uint4*>(src) + piece);
+        dst[u] = reinterpret_cast<uint4*>(d) + piece;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (dst[u]) *dst[u] = v[u];
+  }
 }
 
 }  // namespace
 
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
-  const bool smem_path = a.S > 1 && a.M <= kMaxSmemSlots;
+  const size_t smem = (2 * static_cast<size_t>(a.M) + 2 * static_cast<size_t>(a.S)) * sizeof(uint32_t);
+  const bool smem_path = a.S > 1 && smem <= kMaxClusterSmem;
   if (!smem_path) {
     update_kernel<<<a.B * a.Hkv, kUpdThreads, 0, stream>>>(a);
     return cudaGetLastError();
   }
-  const size_t smem = (static_cast<size_t>(a.M) + a.S) * sizeof(uint32_t);
   static bool configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 64 && !configured[dev]) {
     e = cudaFuncSetAttribute(update_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>((kMaxSmemSlots * 2) * sizeof(uint32_t)));
+                             static_cast<int>(kMaxClusterSmem));
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }

@@ -59,6 +59,13 @@ def step_flops(w: wl.Workload):
     return prefill, chunks
 
 
+# dram__bytes_read.sum + dram__bytes_write.sum of one steady-state llama8b_32k
+# chunk launch of the current SDPA kernel, from the ncu capture summarised in
+# profiles/sdpa_chunk_kernel_llama8b_32k.md; None whenever the kernel has
+# changed since that capture.
+SDPA_DRAM_BYTES = 23.9695e6
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -470,7 +477,7 @@ def main():
     ap.add_argument("--workload", default="llama8b_32k", choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
-    ap.add_argument("--traffic", type=float, default=None,
+    ap.add_argument("--traffic", type=float, default=SDPA_DRAM_BYTES,
                     help="DRAM bytes per launch of the dominant kernel from an ncu capture")
     ap.add_argument("--ref-budget", type=float, default=20.0)
     ap.add_argument("--mode", default="step", choices=["step", "kernel"],

@@ -30,6 +30,13 @@ Readings where the paper is silent (each is also listed in the design notes):
   the c-th smallest evicted slot index receives the chunk's c-th token.
 * The new slot's score is the summed weight its own column received in this
   chunk (Eq. 3 sums over s >= t(j), and the chunk's queries are s >= t(j)).
+* Policy variants of §3.1.1 (``policy``): ``"h2o"`` ranks occupied slots by
+  their score; ``"h2o_norm"`` by the normalized score, score / (t - t(j)) with
+  t = P + S the number of tokens processed once the chunk is in (the stored
+  scores stay unnormalized); ``"h2o_orig"`` ranks the slots of KV head h by the
+  score summed over the batch (ascending b) and evicts the same slots in every
+  batch entry, whose positions are read from batch entry 0 (they are identical
+  across the batch when every update used this policy since a reset).
 * Scores accumulate in one of two precisions: ``"fp64"`` (the oracle's own
   trajectory) or ``"fp32"``, which adds, in float32, the q_g query heads in
   ascending order (t = inc_0; t = t + inc_g) and then ``scores + t``; that is
@@ -46,7 +53,7 @@ import math
 import numpy as np
 
 __all__ = ["sdpa_chunk", "update", "run_sequence", "SequenceState", "lse_merge",
-           "chunk_bounds"]
+           "chunk_bounds", "POLICIES"]
 
 
 def _token_positions(slot_pos_bh: np.ndarray, pos0: int, S: int) -> np.ndarray:
@@ -111,14 +118,20 @@ def lse_merge(l1, l2):
     return np.maximum(l1, l2) + np.log1p(np.exp(-np.abs(l1 - l2)))
 
 
+POLICIES = ("h2o", "h2o_norm", "h2o_orig")
+
+
 def update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0: int,
-           recent_window: int, precision: str = "fp32"):
+           recent_window: int, precision: str = "fp32", policy: str = "h2o"):
     """H2O score accumulation, eviction and K/V write (§3.1.1 Eq. 3, §3.2, §A.1.1).
 
-    Inputs are not modified.  Returns a dict with new ``scores`` (float32 or
-    float64), ``slot_pos``, ``k_cache``, ``v_cache`` and ``evict_idx``
-    (B, H_kv, S) int32: slot receiving token pos0 + c, ascending in c.
+    ``policy`` selects the ranking of §3.1.1 (see the module notes).  Inputs
+    are not modified.  Returns a dict with new ``scores`` (float32 or float64),
+    ``slot_pos``, ``k_cache``, ``v_cache`` and ``evict_idx`` (B, H_kv, S)
+    int32: slot receiving token pos0 + c, ascending in c.
     """
+    if policy not in POLICIES:
+        raise ValueError(f"unknown policy {policy!r}")
     B, Hkv, M = slot_pos.shape
     Bq, Hq, N = score_inc.shape
     S = N - M
@@ -134,30 +147,50 @@ def update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0: in
     out_k = np.array(k_cache, copy=True)
     out_v = np.array(v_cache, copy=True)
     evict = np.zeros((B, Hkv, S), np.int32)
+    acc = np.zeros((B, Hkv, M), ft)
+    new = np.zeros((B, Hkv, S), ft)
     for b in range(B):
         for h in range(Hkv):
             # group sum over the q_g query heads of KV head h, ascending order
             t = inc[b, h * qg].copy()
             for g in range(1, qg):
                 t = t + inc[b, h * qg + g]
-            acc = out_scores[b, h] + t[:M]          # Eq. 3: accumulate this chunk
-            new = t[M:]                              # scores of the chunk's own tokens
+            acc[b, h] = out_scores[b, h] + t[:M]    # Eq. 3: accumulate this chunk
+            new[b, h] = t[M:]                        # scores of the chunk's own tokens
+
+    def choose(rank_score, pos):
+        """S smallest candidates under (empty first, rank_score, slot)."""
+        cand = np.nonzero(pos < pos0 + S - W)[0]    # the recent window is protected
+        if cand.size < S:
+            raise ValueError("fewer eviction candidates than chunk tokens")
+        occupied = pos[cand] >= 0
+        rank0 = occupied.astype(np.int64)                   # 0 = empty: ranks first
+        rank1 = np.where(occupied, rank_score[cand], 0)     # empties tie, broken by slot
+        order = np.lexsort((cand, rank1, rank0))
+        return np.sort(cand[order[:S]])
+
+    for h in range(Hkv):
+        if policy == "h2o_orig":
+            tot = acc[0, h].copy()
+            for b in range(1, B):
+                tot = tot + acc[b, h]
+            shared = choose(tot, out_pos[0, h])
+        for b in range(B):
             pos = out_pos[b, h]
-            cand = np.nonzero(pos < pos0 + S - W)[0]  # recent window is protected
-            if cand.size < S:
-                raise ValueError("fewer eviction candidates than chunk tokens")
-            occupied = pos[cand] >= 0
-            rank0 = occupied.astype(np.int64)               # 0 = empty: ranks first
-            rank1 = np.where(occupied, acc[cand], 0)        # empties tie, broken by slot
-            order = np.lexsort((cand, rank1, rank0))
-            chosen = np.sort(cand[order[:S]])
+            if policy == "h2o":
+                chosen = choose(acc[b, h], pos)
+            elif policy == "h2o_norm":
+                age = np.maximum(pos0 + S - pos.astype(np.int64), 1).astype(ft)
+                chosen = choose(acc[b, h] / age, pos)
+            else:
+                chosen = shared
             evict[b, h] = chosen
-            out_scores[b, h] = acc
+            out_scores[b, h] = acc[b, h]
             for c, e in enumerate(chosen):            # scatter along the slot axis
                 out_k[b, h, e] = k_new[b, h, c]
                 out_v[b, h, e] = v_new[b, h, c]
                 out_pos[b, h, e] = pos0 + c
-                out_scores[b, h, e] = new[c]
+                out_scores[b, h, e] = new[b, h, c]
     return dict(scores=out_scores, slot_pos=out_pos, k_cache=out_k, v_cache=out_v,
                 evict_idx=evict)
 
@@ -184,7 +217,8 @@ def chunk_bounds(T: int, M: int, S: int, prefill: int | None = None):
 
 
 def run_sequence(q, k, v, M: int, S: int, W: int, prefill: int | None = None,
-                 scale: float | None = None, precision: str = "fp64", on_step=None):
+                 scale: float | None = None, precision: str = "fp64", on_step=None,
+                 policy: str = "h2o"):
     """Sparse-attention pass over whole sequences: prefill, then chunks of S.
 
     q (B,H_q,T,d), k/v (B,H_kv,T,d).  Returns (out (B,H_q,T,d), final state).
@@ -199,7 +233,7 @@ def run_sequence(q, k, v, M: int, S: int, W: int, prefill: int | None = None,
                                st.slot_pos, p, scale)
         out[:, :, p:e] = o
         res = update(st.scores, st.slot_pos, inc, k[:, :, p:e], v[:, :, p:e],
-                     st.k_cache, st.v_cache, p, W, precision)
+                     st.k_cache, st.v_cache, p, W, precision, policy)
         before = (st.scores, st.slot_pos, st.k_cache, st.v_cache)
         st.scores, st.slot_pos = res["scores"], res["slot_pos"]
         st.k_cache, st.v_cache = res["k_cache"], res["v_cache"]

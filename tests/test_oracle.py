@@ -10,6 +10,7 @@
   overwrites everything, §3.3).
 """
 import itertools
+from fractions import Fraction
 import json
 import math
 import os
@@ -325,3 +326,126 @@ def test_row_subset_matches_full_chunk():
     np.testing.assert_allclose(o2, out[:, :, rows], atol=1e-14)
     np.testing.assert_allclose(l2, lse[:, :, rows], atol=1e-14)
     np.testing.assert_allclose(inc2.sum(axis=-1), len(rows), rtol=1e-12)
+
+
+# ------------------------------------------------- policy variants (§3.1.1) --
+def _brute_force_evict_keyed(key_of, pos, pos0, S, W):
+    """S-subset of candidates with the smallest key sum (empty slot = -1; keys are
+    exact fractions), ties by the lexicographically smallest subset."""
+    cand = [j for j in range(len(pos)) if pos[j] < pos0 + S - W]
+    key = {j: (Fraction(-1) if pos[j] < 0 else key_of(j)) for j in cand}
+    best = None
+    for sub in itertools.combinations(cand, S):
+        s = sum(key[j] for j in sub)
+        if best is None or (s, sub) < best:
+            best = (s, sub)
+    return list(best[1])
+
+
+def _policy_case(seed, B=1):
+    rng = np.random.default_rng(500 + seed)
+    M = int(rng.integers(2, 9))
+    S = int(rng.integers(1, M + 1))
+    W = int(rng.integers(0, S + 2)) if rng.random() < 0.7 else 0
+    if M - max(0, W - S) < S:
+        W = S
+    qg, d, pos0 = 2, 4, 50
+    n_empty = int(rng.integers(0, M + 1)) if rng.random() < 0.4 else 0
+    st = _state(rng, B, 1, M, d, pos0, n_empty=n_empty, int_scores=True)
+    for r in range(max(0, W - S)):
+        st["slot_pos"][:, 0, r] = pos0 - 1 - r
+    st["slot_pos"][1:] = st["slot_pos"][0]        # one set of positions for the batch
+    st["scores"][st["slot_pos"] < 0] = 0
+    inc = rng.integers(0, 3, size=(B, qg, M + S)).astype(np.float32)
+    for b in range(B):
+        inc[b, :, :M][:, st["slot_pos"][b, 0] < 0] = 0
+    _, kn, vn = _rand_seq(rng, B, qg, 1, S, d)
+    return st, inc, kn, vn, M, S, W, pos0
+
+
+@pytest.mark.parametrize("precision", ["fp32", "fp64"])
+@pytest.mark.parametrize("seed", range(30))
+def test_norm_policy_matches_brute_force(seed, precision):
+    """h2o_norm ranks occupied slots by score / (t - t(j)), t = P + S (§3.1.1)."""
+    st, inc, kn, vn, M, S, W, pos0 = _policy_case(seed)
+    res = update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+                 pos0, W, precision, "h2o_norm")
+    acc = st["scores"][0, 0] + inc[0].sum(axis=0)[:M]
+    pos = st["slot_pos"][0, 0]
+    expect = _brute_force_evict_keyed(
+        lambda j: Fraction(int(acc[j])) / (pos0 + S - int(pos[j])), pos, pos0, S, W)
+    assert list(res["evict_idx"][0, 0]) == expect
+    # stored scores stay unnormalized: Eq. 3 for kept slots, own column for new ones
+    kept = np.setdiff1d(np.arange(M), expect)
+    np.testing.assert_array_equal(res["scores"][0, 0, kept], acc[kept])
+    for c, e in enumerate(expect):
+        assert res["slot_pos"][0, 0, e] == pos0 + c
+        assert res["scores"][0, 0, e] == inc[0, :, M + c].sum()
+
+
+def test_norm_policy_evicts_the_older_of_two_equal_scores():
+    rng = np.random.default_rng(9)
+    M, S, W, pos0, d = 3, 1, 0, 100, 4
+    st = _state(rng, 1, 1, M, d, pos0)
+    st["slot_pos"][0, 0] = [90, 10, 95]        # ages 11, 91, 6 at t = 101
+    st["scores"][0, 0] = [4.0, 4.0, 1.0]       # normalized: 0.364, 0.044, 0.167
+    inc = np.zeros((1, 1, M + S), np.float32)
+    _, kn, vn = _rand_seq(rng, 1, 1, 1, S, d)
+    r_h2o = update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+                   pos0, W, "fp32", "h2o")
+    r_norm = update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+                    pos0, W, "fp32", "h2o_norm")
+    assert list(r_h2o["evict_idx"][0, 0]) == [2]       # smallest raw score
+    assert list(r_norm["evict_idx"][0, 0]) == [1]      # long-resident, rarely used
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_orig_policy_for_one_batch_entry_is_h2o(seed):
+    st, inc, kn, vn, M, S, W, pos0 = _policy_case(seed)
+    a = update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+               pos0, W, "fp32", "h2o")
+    b = update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+               pos0, W, "fp32", "h2o_orig")
+    for key in a:
+        np.testing.assert_array_equal(a[key], b[key])
+
+
+@pytest.mark.parametrize("seed", range(30))
+def test_orig_policy_matches_brute_force(seed):
+    """h2o_orig: one selection per KV head from the scores summed over b."""
+    B = 2 + seed % 2
+    st, inc, kn, vn, M, S, W, pos0 = _policy_case(seed, B=B)
+    res = update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+                 pos0, W, "fp32", "h2o_orig")
+    acc = st["scores"][:, 0] + inc.sum(axis=1)[:, :M]          # (B, M), small integers
+    tot = acc.sum(axis=0)
+    expect = _brute_force_evict_keyed(lambda j: Fraction(int(tot[j])), st["slot_pos"][0, 0],
+                                      pos0, S, W)
+    for b in range(B):
+        assert list(res["evict_idx"][b, 0]) == expect
+        for c, e in enumerate(expect):
+            assert res["slot_pos"][b, 0, e] == pos0 + c
+            np.testing.assert_array_equal(res["k_cache"][b, 0, e], kn[b, 0, c])
+            assert res["scores"][b, 0, e] == inc[b, :, M + c].sum()
+    np.testing.assert_array_equal(res["slot_pos"][0], res["slot_pos"][-1])
+
+
+@pytest.mark.parametrize("policy", ["h2o_norm", "h2o_orig"])
+def test_run_invariants_for_policies(policy):
+    """Whole runs with the variants keep the cache invariants (and h2o_orig keeps one
+    set of positions across the batch)."""
+    w = wl.WORKLOADS["tiny"].replace(T=360, S=24, W=16, M=96, B=2)
+    q, k, v = wl.batch_tokens(w, 0, w.T)
+    steps = []
+    out, st = run_sequence(q, k, v, w.M, w.S, w.W, precision="fp32", policy=policy,
+                           on_step=lambda i, pe, before, res: steps.append((pe, res)))
+    for (p, e), res in steps[1:]:
+        pos = res["slot_pos"]
+        assert (pos < e).all() and (pos >= 0).all()
+        for b in range(w.B):
+            for h in range(w.Hkv):
+                assert len(set(pos[b, h].tolist())) == w.M          # no token twice
+                assert set(range(e - w.W, e)) <= set(pos[b, h].tolist())  # recent window
+        if policy == "h2o_orig":
+            assert (pos == pos[0:1]).all()
+    assert np.isfinite(out).all()

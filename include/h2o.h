@@ -141,6 +141,35 @@ H2O_API int h2o_update(const h2o_dims_t* dims, int64_t pos0, float* scores, int3
                h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget, int32_t recent_window,
                int32_t* evict_idx, void* stream);
 
+/* Eviction policies of §3.1.1 (h2o_update_policy). */
+enum {
+  H2O_POLICY_H2O = 0,  /* rank by the H2O score acc_j (what h2o_update does) */
+  H2O_POLICY_NORM = 1, /* rank by the normalized score acc_j / (t - slot_pos_j),
+                          t = pos0 + S the tokens processed once the chunk is
+                          in; the division is float32, rounded to nearest, of
+                          acc_j by the nearest float32 to t - slot_pos_j.  The
+                          stored scores stay the unnormalized acc_j. */
+  H2O_POLICY_ORIG = 2  /* one selection per KV head h shared by every batch
+                          entry, ranked by sum_b acc_{b,h,j} (float32, ascending
+                          b); candidates, empties and the recent window are read
+                          from slot_pos[0, h, :], which must be identical across
+                          b (it stays so when every update of the cache since
+                          h2o_cache_reset used this policy).  Each batch entry
+                          writes its own rows, scores and positions. */
+};
+
+/*
+ * h2o_update with an explicit eviction policy (§3.1.1: the paper's h2o,
+ * h2o_norm and h2o_orig).  Same arguments, layouts, ordering and errors as
+ * h2o_update; `policy` is one of H2O_POLICY_* (H2O_ERR_ARG otherwise).
+ * h2o_update(...) is h2o_update_policy(..., H2O_POLICY_H2O, ...).
+ */
+H2O_API int h2o_update_policy(const h2o_dims_t* dims, int64_t pos0, float* scores,
+                              int32_t* slot_pos, const float* score_inc, const h2o_bf16* k_new,
+                              const h2o_bf16* v_new, h2o_bf16* k_cache, h2o_bf16* v_cache,
+                              int32_t budget, int32_t recent_window, int32_t policy,
+                              int32_t* evict_idx, void* stream);
+
 /* Empties a cache before a new sequence: slot_pos (B, Hkv, M) int32 := -1 and
  * scores (B, Hkv, M) f32 := 0, enqueued on `stream` (the K/V buffers need no
  * clearing: empty slots are never attended and are overwritten first).  This

@@ -20,8 +20,12 @@ H2O_DEVERR_TIMEOUT = 1
 H2O_DEVERR_CANDIDATES = 2
 
 # Every symbol include/h2o.h declares.
-EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_cache_reset",
-           "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors", "h2o_version")
+EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_update_policy",
+           "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
+           "h2o_version")
+
+# Eviction policies of h2o_update_policy (H2O_POLICY_* in include/h2o.h).
+POLICY = {"h2o": 0, "h2o_norm": 1, "h2o_orig": 2}
 
 
 class H2ODims(ctypes.Structure):
@@ -57,10 +61,13 @@ def load(path: str = LIB_PATH):
     lib.h2o_sdpa_chunk.argtypes = [dims_p, i64, f32, vp, vp, vp, vp, vp, vp, vp, vp, vp,
                                    ctypes.c_size_t, vp]
     lib.h2o_update.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, vp]
+    lib.h2o_update_policy.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, i32, i32, i32,
+                                      vp, vp]
     lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_status_string.argtypes = [ctypes.c_int]
     lib.h2o_status_string.restype = ctypes.c_char_p
-    for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_cache_reset",
+    for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_update_policy",
+               "h2o_cache_reset",
                "h2o_last_cuda_error",
                "h2o_device_errors", "h2o_version"):
         getattr(lib, fn).restype = ctypes.c_int
@@ -146,12 +153,14 @@ def h2o_sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale
 
 
 def h2o_update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0: int,
-               recent_window: int, evict_idx=None, budget: int | None = None, stream=None):
+               recent_window: int, evict_idx=None, budget: int | None = None, stream=None,
+               policy: str = "h2o"):
     """H2O score accumulation, eviction and K/V write, in place (see include/h2o.h).
 
     scores (B,Hkv,M) f32, slot_pos (B,Hkv,M) int32, score_inc (B,Hq,M+S) f32,
     k_new/v_new (B,Hkv,S,d) bf16, k_cache/v_cache (B,Hkv,M,d) bf16,
-    evict_idx (B,Hkv,S) int32 or None.  Returns evict_idx.
+    evict_idx (B,Hkv,S) int32 or None.  ``policy`` "h2o" calls h2o_update,
+    "h2o_norm" / "h2o_orig" call h2o_update_policy.  Returns evict_idx.
     """
     lib = load()
     dev = scores.device
@@ -168,12 +177,30 @@ def h2o_update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0
     if evict_idx is not None:
         _expect(evict_idx, "evict_idx", (B, Hkv, S), torch.int32, dev)
     dims = H2ODims(B, Hq, Hkv, d, S, M)
-    st = lib.h2o_update(ctypes.byref(dims), int(pos0), _ptr(scores), _ptr(slot_pos),
-                        _ptr(score_inc), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache),
-                        int(M if budget is None else budget), int(recent_window), _ptr(evict_idx),
-                        _stream(stream))
-    _check("h2o_update", st)
+    args = (ctypes.byref(dims), int(pos0), _ptr(scores), _ptr(slot_pos), _ptr(score_inc),
+            _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache),
+            int(M if budget is None else budget), int(recent_window))
+    if policy == "h2o":
+        st = lib.h2o_update(*args, _ptr(evict_idx), _stream(stream))
+        _check("h2o_update", st)
+    else:
+        if policy not in POLICY:
+            raise ValueError(f"unknown policy {policy!r}")
+        st = lib.h2o_update_policy(*args, POLICY[policy], _ptr(evict_idx), _stream(stream))
+        _check("h2o_update_policy", st)
     return evict_idx
+
+
+def h2o_update_policy(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0: int,
+                      recent_window: int, policy: str, evict_idx=None, budget: int | None = None,
+                      stream=None):
+    """h2o_update with an explicit eviction policy of §3.1.1: "h2o", "h2o_norm"
+    or "h2o_orig" (see include/h2o.h).  Returns evict_idx."""
+    if policy not in POLICY:
+        raise ValueError(f"unknown policy {policy!r}")
+    return h2o_update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0,
+                      recent_window, evict_idx=evict_idx, budget=budget, stream=stream,
+                      policy=policy)
 
 
 def h2o_cache_reset(slot_pos, scores, stream=None):

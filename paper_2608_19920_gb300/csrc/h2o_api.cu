@@ -221,6 +221,14 @@ int h2o_update(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slo
                const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
                h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget, int32_t recent_window,
                int32_t* evict_idx, void* stream) {
+  return h2o_update_policy(dims, pos0, scores, slot_pos, score_inc, k_new, v_new, k_cache,
+                           v_cache, budget, recent_window, H2O_POLICY_H2O, evict_idx, stream);
+}
+
+int h2o_update_policy(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+                      const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
+                      h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget,
+                      int32_t recent_window, int32_t policy, int32_t* evict_idx, void* stream) {
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
@@ -231,6 +239,8 @@ int h2o_update(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slo
       (evict_idx && misaligned(evict_idx)))
     return H2O_ERR_ALIGN;
   if (budget != D.M) return H2O_ERR_ARG;
+  if (policy != H2O_POLICY_H2O && policy != H2O_POLICY_NORM && policy != H2O_POLICY_ORIG)
+    return H2O_ERR_ARG;
   if (D.M < 1 || D.S > D.M) return H2O_ERR_SHAPE;
   if (recent_window < 0 || recent_window > D.M) return H2O_ERR_ARG;
   if (D.M - std::max(0, recent_window - D.S) < D.S) return H2O_ERR_ARG;
@@ -244,6 +254,7 @@ int h2o_update(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slo
   a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = D.Hq / D.Hkv;
   a.pos0 = static_cast<int>(pos0);
   a.W = recent_window;
+  a.policy = policy;
   const cudaError_t e = launch_update(a, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e);
   return H2O_OK;

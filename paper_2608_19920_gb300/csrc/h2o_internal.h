@@ -6,6 +6,8 @@
 
 #include <cstdint>
 
+#include "../../include/h2o.h"
+
 namespace h2o {
 
 constexpr int kTileM = 128;        // query rows per CTA (tcgen05 M)
@@ -47,6 +49,7 @@ struct UpdateArgs {
   int B, Hq, Hkv, d, S, M, qg;
   int pos0;
   int W;
+  int policy;              // H2O_POLICY_*
 };
 
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);

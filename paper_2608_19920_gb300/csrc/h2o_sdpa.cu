@@ -191,8 +191,11 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
   using G = Geom<D, kPair>;
   constexpr int P = G::kPanels;
   extern __shared__ uint8_t smem_raw[];
+  // 1024-byte aligned (128-byte swizzle atoms).  Offsetting the shared array
+  // itself, rather than an integer copy of its address, keeps the pointer in
+  // the shared state space, so accesses through `sm` compile to shared loads.
   auto& sm = *reinterpret_cast<SdpaSmem<D, kPair>*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+      smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const uint32_t lane = tid & 31;

@@ -56,14 +56,33 @@ __device__ __forceinline__ float group_sum(const float* inc, int stride, int qg,
   return t;
 }
 
-__device__ __forceinline__ uint32_t slot_key(const UpdateArgs& a, const float* sc, const int* sp,
-                                             const float* inc, int j, int thr, float* acc_out) {
-  const int pos = sp[j];
-  const float acc = __fadd_rn(sc[j], group_sum(inc, a.M + a.S, a.qg, j));
-  *acc_out = acc;
+// Selection key of a slot (step 2 above).  The rank value is the score for
+// h2o and h2o_orig (the caller passes the batch sum) and, for h2o_norm, the
+// score over the slot's age t - t(j), t = pos0 + S (fp32, rounded to nearest).
+__device__ __forceinline__ uint32_t make_key(float acc, int pos, int thr, int policy, int t_now) {
   if (pos >= thr) return kProtected;
   if (pos < 0) return 0u;
-  return min(__float_as_uint(acc) + 1u, kProtected - 1u);
+  const float r = policy == H2O_POLICY_NORM ? __fdiv_rn(acc, __int2float_rn(t_now - pos)) : acc;
+  return min(__float_as_uint(r) + 1u, kProtected - 1u);
+}
+
+// Eq. 3 for slot j of (b, h): scores + the group's summed weights.
+__device__ __forceinline__ float slot_acc(const UpdateArgs& a, int b, int h, int j) {
+  const size_t grp = static_cast<size_t>(b) * a.Hkv + h;
+  const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * a.qg) * (a.M + a.S);
+  return __fadd_rn(a.scores[grp * a.M + j], group_sum(inc, a.M + a.S, a.qg, j));
+}
+
+// Key of slot j for the selection of (b, h) (h2o_orig: of KV head h, b = 0);
+// *acc_out receives the score of (b, h).
+__device__ __forceinline__ uint32_t slot_key(const UpdateArgs& a, int b, int h, int j, int thr,
+                                             float* acc_out) {
+  const int pos = a.slot_pos[(static_cast<size_t>(b) * a.Hkv + h) * a.M + j];
+  float acc = slot_acc(a, b, h, j);
+  *acc_out = acc;
+  if (a.policy == H2O_POLICY_ORIG)
+    for (int bb = 1; bb < a.B; ++bb) acc = __fadd_rn(acc, slot_acc(a, bb, h, j));
+  return make_key(acc, pos, thr, a.policy, a.pos0 + a.S);
 }
 
 // Exclusive block scan of one bit per thread; returns the prefix, total in *tot.
@@ -97,11 +116,11 @@ __device__ __forceinline__ void copy_row(const UpdateArgs& a, int grp, int c, in
 __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs a) {
   __shared__ UpdSmem sm;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int grp = blockIdx.x;
-  const int b = grp / a.Hkv, h = grp % a.Hkv;
-  float* sc = a.scores + static_cast<size_t>(grp) * a.M;
-  int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
-  const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * a.qg) * (a.M + a.S);
+  // one (b, h) per CTA; h2o_orig: one KV head per CTA, for every b
+  const bool orig = a.policy == H2O_POLICY_ORIG;
+  const int b = orig ? 0 : static_cast<int>(blockIdx.x) / a.Hkv;
+  const int h = orig ? static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x) % a.Hkv;
+  const int nb = orig ? a.B : 1;  // batch entries whose state this CTA writes
   const int thr = a.pos0 + a.S - a.W;  // slots holding positions >= thr are protected
   const int M = a.M, S = a.S;
 
@@ -111,7 +130,7 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
     unsigned long long best = ~0ull;
     for (int j = tid; j < M; j += kUpdThreads) {
       float acc;
-      const uint32_t key = slot_key(a, sc, sp, inc, j, thr, &acc);
+      const uint32_t key = slot_key(a, b, h, j, thr, &acc);
       const unsigned long long k64 = (static_cast<unsigned long long>(key) << 32) | static_cast<uint32_t>(j);
       best = k64 < best ? k64 : best;
     }
@@ -147,7 +166,7 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
       __syncthreads();
       for (int j = tid; j < M; j += kUpdThreads) {
         float acc;
-        const uint32_t key = slot_key(a, sc, sp, inc, j, thr, &acc);
+        const uint32_t key = slot_key(a, b, h, j, thr, &acc);
         if ((key & mask) == prefix) atomicAdd(&sm.hist[(key >> shift) & 255u], 1u);
       }
       __syncthreads();
@@ -197,7 +216,7 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
   for (int base = 0; base < M; base += kUpdThreads) {
     const int j = base + tid;
     float acc = 0.f;
-    const uint32_t key = j < M ? slot_key(a, sc, sp, inc, j, thr, &acc) : kProtected;
+    const uint32_t key = j < M ? slot_key(a, b, h, j, thr, &acc) : kProtected;
     const bool lt = key < T;
     const bool eq = j < M && key == T;
     uint32_t eq_tot;
@@ -208,12 +227,18 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
     const uint32_t c = sel_base + block_scan_bit(sel0, sm.warp_tot2, &sel_tot);
     const bool sel = sel0 && c < static_cast<uint32_t>(S);
     if (j < M) {
-      if (sel) {
-        sc[j] = group_sum(inc + M, M + S, a.qg, static_cast<int>(c));  // the new token's own column
-        sp[j] = a.pos0 + static_cast<int>(c);
-        if (a.evict_idx) a.evict_idx[static_cast<size_t>(grp) * S + c] = j;
-      } else {
-        sc[j] = acc;
+      for (int bi = 0; bi < nb; ++bi) {
+        const int bb = b + bi;
+        const size_t g = static_cast<size_t>(bb) * a.Hkv + h;
+        const float* inc = a.score_inc + static_cast<size_t>(bb * a.Hq + h * a.qg) * (M + S);
+        if (sel) {
+          // the new token's own column
+          a.scores[g * M + j] = group_sum(inc + M, M + S, a.qg, static_cast<int>(c));
+          a.slot_pos[g * M + j] = a.pos0 + static_cast<int>(c);
+          if (a.evict_idx) a.evict_idx[g * S + c] = j;
+        } else {
+          a.scores[g * M + j] = bi == 0 ? acc : slot_acc(a, bb, h, j);
+        }
       }
     }
     // warp-cooperative K/V copies of this warp's evicted slots
@@ -223,7 +248,7 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
       m &= m - 1;
       const int cc = __shfl_sync(0xffffffffu, static_cast<int>(c), src_lane);
       const int jj = __shfl_sync(0xffffffffu, j, src_lane);
-      copy_row(a, grp, cc, jj, lane);
+      for (int bi = 0; bi < nb; ++bi) copy_row(a, (b + bi) * a.Hkv + h, cc, jj, lane);
     }
     eq_base += eq_tot;
     sel_base += sel_tot;
@@ -266,8 +291,8 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_t
   return base + incl - v;
 }
 
-// Loads of up to kMaxQg query heads are issued before their sum is formed.
-constexpr int kMaxQg = 8;
+// Loads of up to kQgBatch query heads are in flight before their sums.
+constexpr int kQgBatch = 4;
 // Slots a thread handles per batch of loads in phase 1.
 constexpr int kBatch = 8;
 
@@ -278,82 +303,100 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   __shared__ uint32_t bcast[4];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rank = static_cast<int>(cluster_rank());
-  const int grp = blockIdx.x / C;
-  const int b = grp / a.Hkv, h = grp % a.Hkv;
+  // one (b, h) per cluster; h2o_orig: one KV head per cluster, for every b
+  const bool orig = a.policy == H2O_POLICY_ORIG;
+  const int gidx = static_cast<int>(blockIdx.x) / C;
+  const int b0 = orig ? 0 : gidx / a.Hkv, h = orig ? gidx : gidx % a.Hkv;
+  const int nb = orig ? a.B : 1;  // batch entries whose state this cluster writes
   const int M = a.M, S = a.S, NK = M + S, qg = a.qg;
-  float* sc = a.scores + static_cast<size_t>(grp) * M;
-  int* sp = a.slot_pos + static_cast<size_t>(grp) * M;
-  const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK;
   const int thr = a.pos0 + S - a.W;
   uint32_t* keys = dyn;                                          // [M]
-  float* accs = reinterpret_cast<float*>(dyn + M);               // [M] accumulated scores
+  float* accs = reinterpret_cast<float*>(dyn + M);               // [M] scores of (b0, h)
   float* nscore = reinterpret_cast<float*>(dyn + 2 * M);         // [S] score of new token c
   int* elist = reinterpret_cast<int*>(dyn + 2 * M + S);          // [S] evicted slot of rank c
+  auto scores_of = [&](int b) { return a.scores + (static_cast<size_t>(b) * a.Hkv + h) * M; };
+  auto pos_of = [&](int b) { return a.slot_pos + (static_cast<size_t>(b) * a.Hkv + h) * M; };
+  auto inc_of = [&](int b) { return a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK; };
 
   // Thread t owns slots [t R, t R + R) in slot order.
   const int R = (M + kCThreads - 1) / kCThreads;
   const int j0 = min(M, tid * R), j1 = min(M, j0 + R);
-  // 16-byte loads need every row start (grp M, head rows of NK) and j0 aligned
-  const bool vec = R % 4 == 0 && M % 4 == 0 && NK % 4 == 0 && qg <= kMaxQg;
+  // 16-byte loads need every row start (b, h rows of M and NK) and j0 aligned
+  const bool vec = R % 4 == 0 && M % 4 == 0 && NK % 4 == 0;
 
-  // Phase 1: acc_j = scores_j + (inc_0j + inc_1j + ...), fp32, heads in order
-  // (Eq. 3), and the selection key of every slot; each batch issues all of
-  // its loads before the first sum.
-  for (int jb = j0; jb < j1; jb += kBatch) {
-    const int n = min(kBatch, j1 - jb);
+  // acc_j = scores_j + (inc_0j + inc_1j + ...) of batch entry b for the n
+  // slots from jb, fp32, heads in order (Eq. 3); tot_j := acc_j (first) or
+  // tot_j + acc_j.  Loads of up to four heads are in flight before their sums.
+  auto add_acc = [&](int b, int jb, int n, float (&tot)[kBatch], bool first) {
+    const float* sc = scores_of(b);
+    const float* inc = inc_of(b);
     float sv[kBatch], tv[kBatch];
-    int pv[kBatch];
     if (vec && n == kBatch) {
-      float4 s4[2], i4[kMaxQg][2];
-      int4 p4[2];
+      float4 s4[2];
 #pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        s4[q] = *reinterpret_cast<const float4*>(sc + jb + 4 * q);
-        p4[q] = *reinterpret_cast<const int4*>(sp + jb + 4 * q);
+      for (int q = 0; q < 2; ++q) s4[q] = *reinterpret_cast<const float4*>(sc + jb + 4 * q);
+      for (int g0 = 0; g0 < qg; g0 += kQgBatch) {
+        float4 i4[kQgBatch][2];
+#pragma unroll
+        for (int gg = 0; gg < kQgBatch; ++gg)
+          if (g0 + gg < qg)
+#pragma unroll
+            for (int q = 0; q < 2; ++q)
+              i4[gg][q] = __ldg(reinterpret_cast<const float4*>(
+                                    inc + static_cast<size_t>(g0 + gg) * NK + jb) + q);
+#pragma unroll
+        for (int gg = 0; gg < kQgBatch; ++gg)
+          if (g0 + gg < qg)
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const float x[4] = {i4[gg][q].x, i4[gg][q].y, i4[gg][q].z, i4[gg][q].w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e)
+                tv[4 * q + e] = (g0 + gg == 0) ? x[e] : __fadd_rn(tv[4 * q + e], x[e]);
+            }
       }
-#pragma unroll
-      for (int g = 0; g < kMaxQg; ++g)
-        if (g < qg)
-#pragma unroll
-          for (int q = 0; q < 2; ++q)
-            i4[g][q] = __ldg(reinterpret_cast<const float4*>(inc + static_cast<size_t>(g) * NK + jb) + q);
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
         sv[4 * q] = s4[q].x; sv[4 * q + 1] = s4[q].y; sv[4 * q + 2] = s4[q].z; sv[4 * q + 3] = s4[q].w;
-        pv[4 * q] = p4[q].x; pv[4 * q + 1] = p4[q].y; pv[4 * q + 2] = p4[q].z; pv[4 * q + 3] = p4[q].w;
-        tv[4 * q] = i4[0][q].x; tv[4 * q + 1] = i4[0][q].y;
-        tv[4 * q + 2] = i4[0][q].z; tv[4 * q + 3] = i4[0][q].w;
       }
-#pragma unroll
-      for (int g = 1; g < kMaxQg; ++g)
-        if (g < qg)
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            tv[4 * q] = __fadd_rn(tv[4 * q], i4[g][q].x);
-            tv[4 * q + 1] = __fadd_rn(tv[4 * q + 1], i4[g][q].y);
-            tv[4 * q + 2] = __fadd_rn(tv[4 * q + 2], i4[g][q].z);
-            tv[4 * q + 3] = __fadd_rn(tv[4 * q + 3], i4[g][q].w);
-          }
     } else {
       for (int k = 0; k < n; ++k) {
         sv[k] = sc[jb + k];
-        pv[k] = sp[jb + k];
         tv[k] = group_sum(inc, NK, qg, jb + k);
       }
     }
+#pragma unroll
+    for (int k = 0; k < kBatch; ++k)
+      if (k < n) {
+        const float acc = __fadd_rn(sv[k], tv[k]);
+        tot[k] = first ? acc : __fadd_rn(tot[k], acc);
+      }
+  };
+
+  // Phase 1: scores and selection keys of every slot (positions of b0).
+  for (int jb = j0; jb < j1; jb += kBatch) {
+    const int n = min(kBatch, j1 - jb);
+    float tot[kBatch];
+    int pv[kBatch];
+    const int* sp = pos_of(b0);
+    if (vec && n == kBatch) {
+      const int4 p0 = *reinterpret_cast<const int4*>(sp + jb);
+      const int4 p1 = *reinterpret_cast<const int4*>(sp + jb + 4);
+      pv[0] = p0.x; pv[1] = p0.y; pv[2] = p0.z; pv[3] = p0.w;
+      pv[4] = p1.x; pv[5] = p1.y; pv[6] = p1.z; pv[7] = p1.w;
+    } else {
+      for (int k = 0; k < n; ++k) pv[k] = sp[jb + k];
+    }
+    // h2o_orig sums the batch entries in ascending b
+    for (int bi = 0; bi < nb; ++bi) add_acc(b0 + bi, jb, n, tot, bi == 0);
     for (int k = 0; k < n; ++k) {
-      const float acc = __fadd_rn(sv[k], tv[k]);
-      const int pos = pv[k];
-      uint32_t key;
-      if (pos >= thr) key = kProtected;
-      else if (pos < 0) key = 0u;
-      else key = min(__float_as_uint(acc) + 1u, kProtected - 1u);
-      keys[jb + k] = key;
-      accs[jb + k] = acc;
+      keys[jb + k] = make_key(tot[k], pv[k], thr, a.policy, a.pos0 + S);
+      if (!orig) accs[jb + k] = tot[k];
     }
   }
   // scores of the new tokens: their own columns M + c, summed over the group
-  for (int c = tid; c < S; c += kCThreads) nscore[c] = group_sum(inc + M, NK, qg, c);
+  if (!orig)
+    for (int c = tid; c < S; c += kCThreads) nscore[c] = group_sum(inc_of(b0) + M, NK, qg, c);
   // Every CTA of the cluster has read the old state before CTA 0 rewrites it.
   cluster_sync_all();
 
@@ -414,27 +457,40 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   }
   uint32_t tot;
   const uint32_t before = block_excl_scan(n_lt | (n_eq << 16), warp_tot, &tot);
-  uint32_t lt_b = before & 0xFFFFu, eq_b = before >> 16;
 
-  // Phase 4: evicted slots get ranks 0..S-1; CTA 0 writes the new state.
-  for (int j = j0; j < j1; ++j) {
-    const uint32_t key = keys[j];
-    const bool eq = key == T;
-    const bool sel0 = key < T || (eq && eq_b < take_eq);
-    const uint32_t c = lt_b + min(eq_b, take_eq);
-    const bool sel = sel0 && c < static_cast<uint32_t>(S);
-    lt_b += key < T;
-    eq_b += eq;
-    if (sel) {
-      elist[c] = j;
+  // Phase 4: evicted slots get ranks 0..S-1; CTA 0 writes the new state of
+  // every batch entry the cluster owns.
+  {
+    uint32_t lt_b = before & 0xFFFFu, eq_b = before >> 16;
+    for (int j = j0; j < j1; ++j) {
+      const uint32_t key = keys[j];
+      const bool eq = key == T;
+      const bool sel0 = key < T || (eq && eq_b < take_eq);
+      const uint32_t c = lt_b + min(eq_b, take_eq);
+      const bool sel = sel0 && c < static_cast<uint32_t>(S);
+      lt_b += key < T;
+      eq_b += eq;
+      if (sel) elist[c] = j;
       if (rank == 0) {
-        sp[j] = a.pos0 + static_cast<int>(c);
-        if (a.evict_idx) a.evict_idx[static_cast<size_t>(grp) * S + c] = j;
-        accs[j] = nscore[c];
+        for (int bi = 0; bi < nb; ++bi) {
+          const int b = b0 + bi;
+          const size_t g = static_cast<size_t>(b) * a.Hkv + h;
+          if (sel) {
+            pos_of(b)[j] = a.pos0 + static_cast<int>(c);
+            if (a.evict_idx) a.evict_idx[g * S + c] = j;
+          }
+          if (orig) {
+            scores_of(b)[j] = sel ? group_sum(inc_of(b) + M, NK, qg, static_cast<int>(c))
+                                  : slot_acc(a, b, h, j);
+          } else if (sel) {
+            accs[j] = nscore[c];
+          }
+        }
       }
     }
   }
-  if (rank == 0) {
+  if (rank == 0 && !orig) {
+    float* sc = scores_of(b0);
     if (vec) {
       for (int j = j0; j < j1; j += 4)
         *reinterpret_cast<float4*>(sc + j) = *reinterpret_cast<const float4*>(accs + j);
@@ -444,12 +500,14 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   }
   __syncthreads();
 
-  // Phase 5: this CTA's share of the K/V row copies (ranks c = rank mod C),
-  // 16-byte pieces, four loads in flight per thread before their stores.
+  // Phase 5: this CTA's share of the K/V row copies (ranks c = rank mod C) of
+  // every batch entry the cluster owns, 16-byte pieces, four loads in flight
+  // per thread before their stores.
   const int n_sel = min(static_cast<int>((tot & 0xFFFFu) + min(tot >> 16, take_eq)), S);
   const int rows = n_sel > rank ? (n_sel - 1 - rank) / C + 1 : 0;
   const int vecs = a.d / 8;  // 16-byte pieces per row
-  const int pieces = rows * 2 * vecs;
+  const int per_b = rows * 2 * vecs;
+  const int pieces = nb * per_b;
   for (int x0 = tid; x0 < pieces; x0 += 4 * kCThreads) {
     uint4 v[4];
     uint4* dst[4];
@@ -458,12 +516,15 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
       const int x = x0 + u * kCThreads;
       dst[u] = nullptr;
       if (x < pieces) {
-        const int piece = x % vecs;
-        const int rv = x / vecs;           // row index * 2 + (0 = K, 1 = V)
+        const int b = b0 + x / per_b;
+        const int xr = x % per_b;
+        const int piece = xr % vecs;
+        const int rv = xr / vecs;          // row index * 2 + (0 = K, 1 = V)
         const int cc = rank + C * (rv >> 1);
         const bool is_v = rv & 1;
-        const uint16_t* src = (is_v ? a.v_new : a.k_new) + (static_cast<size_t>(grp) * S + cc) * a.d;
-        uint16_t* d = (is_v ? a.v_cache : a.k_cache) + (static_cast<size_t>(grp) * M + elist[cc]) * a.d;
+        const size_t g = static_cast<size_t>(b) * a.Hkv + h;
+        const uint16_t* src = (is_v ? a.v_new : a.k_new) + (g * S + cc) * a.d;
+        uint16_t* d = (is_v ? a.v_cache : a.k_cache) + (g * M + elist[cc]) * a.d;
         v[u] = __ldg(reinterpret_cast<const uint4*>(src) + piece);
         dst[u] = reinterpret_cast<uint4*>(d) + piece;
       }
@@ -480,7 +541,8 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
   const size_t smem = (2 * static_cast<size_t>(a.M) + 2 * static_cast<size_t>(a.S)) * sizeof(uint32_t);
   const bool smem_path = a.S > 1 && smem <= kMaxClusterSmem;
   if (!smem_path) {
-    update_kernel<<<a.B * a.Hkv, kUpdThreads, 0, stream>>>(a);
+    const int groups = a.policy == H2O_POLICY_ORIG ? a.Hkv : a.B * a.Hkv;
+    update_kernel<<<groups, kUpdThreads, 0, stream>>>(a);
     return cudaGetLastError();
   }
   static bool configured[64] = {};
@@ -496,7 +558,8 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
   int C = (a.S + 63) / 64;
   C = C < 1 ? 1 : (C > 8 ? 8 : C);
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(a.B * a.Hkv * C));
+  const int groups = a.policy == H2O_POLICY_ORIG ? a.Hkv : a.B * a.Hkv;
+  cfg.gridDim = dim3(static_cast<unsigned>(groups * C));
   cfg.blockDim = dim3(kCThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;

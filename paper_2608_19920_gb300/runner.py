@@ -27,8 +27,11 @@ class H2OLayer:
     """Device-resident H2O cache state of one layer: M slots per (b, KV head)."""
 
     def __init__(self, B: int, Hq: int, Hkv: int, d: int, M: int, S: int, W: int,
-                 device="cuda", scale: float = 0.0, keep_evictions: bool = True):
+                 device="cuda", scale: float = 0.0, keep_evictions: bool = True,
+                 policy: str = "h2o"):
+        """``policy``: eviction rule of §3.1.1, "h2o", "h2o_norm" or "h2o_orig"."""
         self.B, self.Hq, self.Hkv, self.d, self.M, self.S, self.W = B, Hq, Hkv, d, M, S, W
+        self.policy = policy
         self.scale = scale
         dev = torch.device(device)
         self.k_cache = torch.zeros((B, Hkv, M, d), dtype=torch.bfloat16, device=dev)
@@ -62,5 +65,6 @@ class H2OLayer:
         out, inc = lib.h2o_sdpa_chunk(q, self.k_cache, self.v_cache, k_new, v_new, self.slot_pos,
                                       pos0, self.scale, out=out, score_inc=inc, stream=stream)
         lib.h2o_update(self.scores, self.slot_pos, inc, k_new, v_new, self.k_cache, self.v_cache,
-                       pos0, self.W, evict_idx=ev if self.keep_evictions else None, stream=stream)
+                       pos0, self.W, evict_idx=ev if self.keep_evictions else None, stream=stream,
+                       policy=self.policy)
         return out, inc, ev

@@ -83,6 +83,21 @@ def test_update_argument_checks(lib):
     assert _upd(lib, _dims(M=0, S=1), budget=0) == SHAPE
 
 
+def _upd_policy(lib, dims, policy, budget=256, W=32, pos0=256):
+    vp = ctypes.c_void_p
+    return lib.h2o_update_policy(ctypes.byref(dims), pos0, *[vp(0x1000)] * 7, budget, W, policy,
+                                 None, None)
+
+
+def test_update_policy_argument_checks(lib):
+    """Unknown policy codes are rejected on the host; the other checks are shared."""
+    assert _upd_policy(lib, _dims(), 3) == ARG
+    assert _upd_policy(lib, _dims(), -1) == ARG
+    assert _upd_policy(lib, _dims(), 1, budget=255) == ARG
+    assert _upd_policy(lib, _dims(S=300), 2) == SHAPE
+    assert [b.POLICY[p] for p in ("h2o", "h2o_norm", "h2o_orig")] == [0, 1, 2]
+
+
 def test_binding_refuses_to_run_without_the_library(tmp_path):
     saved = b._lib
     try:

@@ -15,7 +15,8 @@ import torch
 
 from oracle import sdpa_chunk as ref_sdpa
 from oracle import update as ref_update
-from paper_2608_19920_gb300 import H2OLayer, build, h2o_device_errors, h2o_sdpa_chunk, h2o_update
+from paper_2608_19920_gb300 import (H2OLayer, build, h2o_device_errors, h2o_sdpa_chunk, h2o_update,
+                                   h2o_update_policy)
 from paper_2608_19920_gb300 import workloads as wl
 from paper_2608_19920_gb300.runner import chunk_bounds
 
@@ -169,6 +170,73 @@ def test_update_is_bit_exact(dev, case):
                                   ref["scores"].astype(np.float32).view(np.uint32))
     np.testing.assert_array_equal(f32(g_k), ref["k_cache"])
     np.testing.assert_array_equal(f32(g_v), ref["v_cache"])
+
+
+POLICY_CASES = [
+    # B, Hq, Hkv, d, S, M, W, n_empty, int_scores
+    (2, 8, 2, 128, 20, 300, 50, 17, True),      # cluster path, ties
+    (1, 8, 2, 128, 512, 4096, 512, 0, False),   # the Llama-3-8B-shaped chunk
+    (3, 4, 2, 64, 1, 500, 64, 0, False),        # S = 1: argmin path
+    (2, 4, 1, 64, 40, 26000, 100, 0, False),    # keys beyond the cluster variant's shared memory
+    (4, 32, 8, 128, 256, 2048, 256, 0, False),  # batched workload shape
+]
+
+
+@pytest.mark.parametrize("case", POLICY_CASES, ids=lambda c: "x".join(map(str, c)))
+@pytest.mark.parametrize("policy", ["h2o_norm", "h2o_orig"])
+def test_update_policy_is_bit_exact(dev, policy, case):
+    """h2o_update_policy against the oracle's policies of §3.1.1, bit for bit."""
+    B, Hq, Hkv, d, S, M, W, n_empty, int_scores = case
+    st, inc, kn, vn, pos0 = _update_inputs(case, hash((policy,) + case) % 2**32)
+    if policy == "h2o_orig":     # one set of positions across the batch
+        st["slot_pos"][1:] = st["slot_pos"][0]
+    g_scores = torch.from_numpy(st["scores"]).to(dev)
+    g_pos = torch.from_numpy(st["slot_pos"]).to(dev)
+    g_k = bf(st["k_cache"], dev)
+    g_v = bf(st["v_cache"], dev)
+    ev = torch.full((B, Hkv, S), -7, dtype=torch.int32, device=dev)
+    h2o_update_policy(g_scores, g_pos, torch.from_numpy(inc).to(dev), bf(kn, dev), bf(vn, dev),
+                      g_k, g_v, pos0, W, policy, evict_idx=ev)
+    torch.cuda.synchronize()
+    assert h2o_device_errors() == 0
+    ref = ref_update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+                     pos0, W, "fp32", policy)
+    np.testing.assert_array_equal(ev.cpu().numpy(), ref["evict_idx"])
+    np.testing.assert_array_equal(g_pos.cpu().numpy(), ref["slot_pos"])
+    np.testing.assert_array_equal(g_scores.cpu().numpy().view(np.uint32),
+                                  ref["scores"].astype(np.float32).view(np.uint32))
+    np.testing.assert_array_equal(f32(g_k), ref["k_cache"])
+    np.testing.assert_array_equal(f32(g_v), ref["v_cache"])
+    # the variant changes the victims on these inputs (not a silent h2o)
+    plain = ref_update(st["scores"], st["slot_pos"], inc, kn, vn, st["k_cache"], st["v_cache"],
+                       pos0, W, "fp32", "h2o")
+    if S >= 20 and (B > 1 or policy == "h2o_norm"):
+        assert not np.array_equal(plain["evict_idx"], ref["evict_idx"])
+
+
+@pytest.mark.parametrize("policy", ["h2o_norm", "h2o_orig"])
+def test_tiny_workload_policy_teacher_forced(dev, policy):
+    """A whole tiny sequence (B = 2) with each variant: the GPU chunk step against
+    the oracle's, from the GPU's own cache state, at every chunk."""
+    w = wl.WORKLOADS["tiny"].replace(B=2)
+    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, policy=policy)
+    layer.reset()
+    for i, (p, e) in enumerate(chunk_bounds(w.T, w.M, w.S)):
+        q, k, v = wl.batch_tokens(w, p, e)
+        before = dict(scores=layer.scores.cpu().numpy(), slot_pos=layer.slot_pos.cpu().numpy(),
+                      k_cache=f32(layer.k_cache), v_cache=f32(layer.v_cache))
+        out, inc, ev = layer.step(bf(q, dev), bf(k, dev), bf(v, dev), p)
+        torch.cuda.synchronize()
+        ref = ref_update(before["scores"], before["slot_pos"], inc.cpu().numpy(), k, v,
+                         before["k_cache"], before["v_cache"], p, w.W, "fp32", policy)
+        np.testing.assert_array_equal(layer.slot_pos.cpu().numpy(), ref["slot_pos"])
+        np.testing.assert_array_equal(layer.scores.cpu().numpy().view(np.uint32),
+                                      ref["scores"].astype(np.float32).view(np.uint32))
+        np.testing.assert_array_equal(f32(layer.k_cache), ref["k_cache"])
+    assert h2o_device_errors() == 0
+    if policy == "h2o_orig":
+        pos = layer.slot_pos.cpu().numpy()
+        assert (pos == pos[0:1]).all()
 
 
 def test_update_twice_in_a_row_without_evict_idx(dev):

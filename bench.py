@@ -63,7 +63,7 @@ def step_flops(w: wl.Workload):
 # chunk launch of the current SDPA kernel, from the ncu capture summarised in
 # profiles/sdpa_chunk_kernel_llama8b_32k.md; None whenever the kernel has
 # changed since that capture.
-SDPA_DRAM_BYTES = 23.9695e6
+SDPA_DRAM_BYTES = None
 
 
 def peaks():
@@ -359,21 +359,33 @@ def run_ours(args, w):
         "tflops": alg_tflops,
         "tflops_frac_of_peak": alg_tflops / pk["bf16_sus"],
         "chunk_step_ms_median": statistics.median(chunk_step_ms) if chunk_step_ms else None,
-        "gpu_launches": args.steps * (2 * len(plan)),
+        "gpu_launches": args.steps * sum(launches_per_chunk(e - p, w.M) for p, e in plan),
         "clocks": clocks,
     }
     # the chunk SDPA is timed on its own (launch after launch, L2 flushed in
     # between): its denominator is the burst peak; the sustained one is given
     # alongside
-    line["roofline"] = {
-        "bound": "tensor", "kernel": "sdpa_chunk_kernel<128,pair> (steady-state chunk)",
-        "achieved": kern["alg_tflops"], "peak": pk["bf16"], "unit": "TFLOP/s",
-        "frac": kern["alg_tflops"] / pk["bf16"], "traffic": args.traffic,
-        "peak_source": f"{pk['source']} bf16 dense, burst",
-        "frac_of_sustained": kern["alg_tflops"] / pk["bf16_sus"],
-        "avg_launch_us": kern["avg_us"], "flops_per_launch": kern["flops"],
-        "executed_tflops": kern["alg_tflops"] * kern["exec_ratio"],
-    }
+    traffic = args.traffic if args.traffic is not None else (
+        SDPA_DRAM_BYTES if w.name == "llama8b_32k" else None)
+    if w.S == 1:
+        # decode: K and V read once per step, HBM bound
+        line["roofline"] = {
+            "bound": "hbm", "kernel": "decode_split_kernel + decode_combine_kernel (one step)",
+            "achieved": kern["gbs"], "peak": pk["hbm"], "unit": "GB/s",
+            "frac": kern["gbs"] / pk["hbm"], "traffic": traffic,
+            "peak_source": f"{pk['source']} HBM copy bandwidth",
+            "avg_launch_us": kern["avg_us"], "bytes_per_launch": kern["bytes"],
+        }
+    else:
+        line["roofline"] = {
+            "bound": "tensor", "kernel": "sdpa_chunk_kernel<128,pair> (steady-state chunk)",
+            "achieved": kern["alg_tflops"], "peak": pk["bf16"], "unit": "TFLOP/s",
+            "frac": kern["alg_tflops"] / pk["bf16"], "traffic": traffic,
+            "peak_source": f"{pk['source']} bf16 dense, burst",
+            "frac_of_sustained": kern["alg_tflops"] / pk["bf16_sus"],
+            "avg_launch_us": kern["avg_us"], "flops_per_launch": kern["flops"],
+            "executed_tflops": kern["alg_tflops"] * kern["exec_ratio"],
+        }
     if args.e2e:
         line["e2e"] = run_e2e(w, layer, plan, outs, dev, args, world)
     if args.cpu_baseline and rank == 0 and world == 1:
@@ -391,7 +403,7 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
     p, e = plan[idx]
     q, k, v = inputs[idx]
     out = torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=q.device)
-    inc = torch.empty((w.B, w.Hq, w.M + e - p), dtype=torch.float32, device=q.device)
+    inc, _, ws = layer._buf(e - p)
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
     clean = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
     times = []
@@ -405,7 +417,7 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
         h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out=out,
-                       score_inc=inc)
+                       score_inc=inc, workspace=ws)
         b.record(stream)
         torch.cuda.synchronize()
         times.append(a.elapsed_time(b))
@@ -413,8 +425,20 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
     avg_ms = sum(times) / len(times)
     flops = chunk_flops(w.B, w.Hq, w.d, e - p, w.M)
     exec_flops = executed_mma_flops(w, e - p)
+    kv_bytes = decode_kv_bytes(w)
     return dict(avg_us=avg_ms * 1e3, flops=flops, alg_tflops=flops / (avg_ms / 1e3) / 1e12,
-                exec_ratio=exec_flops / flops)
+                exec_ratio=exec_flops / flops, bytes=kv_bytes, gbs=kv_bytes / (avg_ms / 1e3) / 1e9)
+
+
+def decode_kv_bytes(w):
+    """Algorithmic bytes of one decode step: every cache K and V row read once."""
+    return 2.0 * w.B * w.Hkv * w.M * w.d * 2
+
+
+def launches_per_chunk(S, M):
+    """Kernels of this library one chunk launches: the SDPA (split + combine
+    when S = 1 and a cache exists) and the update."""
+    return 3 if S == 1 and M > 0 else 2
 
 
 def executed_mma_flops(w, S):
@@ -477,7 +501,7 @@ def main():
     ap.add_argument("--workload", default="llama8b_32k", choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
-    ap.add_argument("--traffic", type=float, default=SDPA_DRAM_BYTES,
+    ap.add_argument("--traffic", type=float, default=None,
                     help="DRAM bytes per launch of the dominant kernel from an ncu capture")
     ap.add_argument("--ref-budget", type=float, default=20.0)
     ap.add_argument("--mode", default="step", choices=["step", "kernel"],

@@ -123,7 +123,8 @@ def h2o_sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale
 
     q (B,Hq,S,d) bf16; k_cache/v_cache (B,Hkv,M,d) bf16; k_new/v_new (B,Hkv,S,d)
     bf16; slot_pos (B,Hkv,M) int32.  Returns (out (B,Hq,S,d) bf16,
-    score_inc (B,Hq,M+S) f32).
+    score_inc (B,Hq,M+S) f32).  ``workspace`` (a device buffer of at least
+    h2o_workspace_size bytes) is allocated here when it is needed and not given.
     """
     lib = load()
     dev = q.device
@@ -144,6 +145,10 @@ def h2o_sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale
     _expect(out, "out", (B, Hq, S, d), bf, dev)
     _expect(score_inc, "score_inc", (B, Hq, M + S), torch.float32, dev)
     dims = H2ODims(B, Hq, Hkv, d, S, M)
+    if workspace is None:
+        n = h2o_workspace_size(dims)
+        if n:
+            workspace = torch.empty(n, dtype=torch.uint8, device=dev)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     st = lib.h2o_sdpa_chunk(ctypes.byref(dims), int(pos0), float(scale), _ptr(q), _ptr(k_cache),
                             _ptr(v_cache), _ptr(k_new), _ptr(v_new), _ptr(slot_pos), _ptr(out),

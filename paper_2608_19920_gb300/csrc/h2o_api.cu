@@ -139,7 +139,10 @@ int h2o_workspace_size(const h2o_dims_t* dims, size_t* bytes) {
   const int st = check_dims(dims);
   if (st != H2O_OK) return st;
   if (!bytes) return H2O_ERR_NULL;
-  *bytes = 0;
+  int split_len = 0, n_split = 0;
+  size_t ws = 0;
+  const h2o_dims_t& D = *dims;
+  *bytes = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws) ? ws : 0;
   return H2O_OK;
 }
 
@@ -147,8 +150,6 @@ int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, co
                    const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
                    const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out,
                    float* score_inc, void* workspace, size_t workspace_bytes, void* stream) {
-  (void)workspace;
-  (void)workspace_bytes;
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
@@ -160,16 +161,38 @@ int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, co
     return H2O_ERR_ALIGN;
   if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
   if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
+  const int qg = D.Hq / D.Hkv;
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
+  int split_len = 0, n_split = 0;
+  size_t ws_need = 0;
+  const bool decode = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
+  if (decode && (!workspace || workspace_bytes < ws_need)) return H2O_ERR_WORKSPACE;
+  if (decode && misaligned(workspace)) return H2O_ERR_ALIGN;
   DeviceInfo* di = nullptr;
   if ((st = current_device(&di)) != H2O_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  if (decode) {
+    // one query token per sequence: split-K kernels (h2o_decode.cu)
+    DecodeArgs a;
+    a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
+    a.slot_pos = slot_pos; a.out = out; a.score_inc = score_inc;
+    a.part = static_cast<float*>(workspace);
+    a.err = di->err_word;
+    a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.M = D.M; a.qg = qg;
+    a.pos0 = static_cast<int>(pos0);
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.split_len = split_len;
+    a.n_split = n_split;
+    const cudaError_t e = launch_decode(a, s);
+    return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+  }
   if ((st = get_encoder()) != H2O_OK) return st;
 
-  const int qg = D.Hq / D.Hkv;
   SdpaArgs a;
   std::memset(&a, 0, sizeof(a));
   a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = qg;
   a.pos0 = static_cast<int>(pos0);
-  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
   a.scale_log2 = scale * 1.4426950408889634f;
   if (D.S > kTileM) {
     a.rows_box = kTileM;
@@ -208,7 +231,6 @@ int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, co
       if ((st = encode(&a.tm_vc, v_cache, 3, dc, bv)) != H2O_OK) return st;
     }
   }
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   const size_t inc_bytes = static_cast<size_t>(G) * qg * (static_cast<size_t>(D.M) + D.S) * sizeof(float);
   cudaError_t e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
   if (e != cudaSuccess) return cuda_fail(e);

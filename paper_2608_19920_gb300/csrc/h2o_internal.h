@@ -52,7 +52,38 @@ struct UpdateArgs {
   int policy;              // H2O_POLICY_*
 };
 
+// S = 1 (one query token per sequence): split-K decode kernels.
+constexpr int kDecodeMaxQg = 8;         // larger GQA groups take the chunk kernel
+constexpr int kDecodeMaxSplitLen = 2048;
+constexpr int kDecodeMinSplitLen = 256;
+constexpr int kDecodeTargetCtas = 608;  // 4 x 152 SMs
+
+struct DecodeArgs {
+  const uint16_t* q;        // (B, Hq, 1, d)
+  const uint16_t* k_cache;  // (B, Hkv, M, d)
+  const uint16_t* v_cache;
+  const uint16_t* k_new;    // (B, Hkv, 1, d)
+  const uint16_t* v_new;
+  const int32_t* slot_pos;  // (B, Hkv, M)
+  uint16_t* out;            // (B, Hq, 1, d) bf16
+  float* score_inc;         // (B, Hq, M + 1): logits (log2 units), then weights
+  float* part;              // (B, Hq, n_split, 2 + d): max, sum, unnormalised output
+  int* err;
+  int B, Hq, Hkv, d, M, qg;
+  int pos0;
+  float scale_log2;
+  int split_len;            // cache slots per split (multiple of 64)
+  int n_split;              // ceil(M / split_len); the last split also takes the new token
+};
+
+// Split of the M cache slots for the decode kernels (a function of the sizes
+// only, so that h2o_workspace_size and h2o_sdpa_chunk agree).  Returns false
+// when the decode kernels do not apply (S != 1, M == 0 or q_g too large).
+bool decode_plan(int B, int Hq, int Hkv, int d, int S, int M, int* split_len, int* n_split,
+                 size_t* ws_bytes);
+
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);
 
 }  // namespace h2o

@@ -31,7 +31,7 @@
 // several 16-byte loads in flight per thread.  The whole update is latency
 // bound (a few MB per chunk), so the design minimises dependent round trips.
 // Otherwise one CTA per (b, kv head) recomputes keys from global memory on
-// every pass (S = 1 takes the argmin path).
+// every pass.  S = 1 has a kernel of its own (update_decode_kernel).
 #include "h2o_internal.h"
 #include "sm100.cuh"
 
@@ -46,7 +46,6 @@ struct UpdSmem {
   uint32_t hist[256];
   uint32_t warp_tot[kUpdWarps];
   uint32_t warp_tot2[kUpdWarps];
-  unsigned long long warp_min[kUpdWarps];
   uint32_t bcast[4];
 };
 
@@ -126,39 +125,7 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
 
   uint32_t T = 0;         // threshold key
   uint32_t take_eq = 0;   // keys equal to T that are evicted (lowest slots first)
-  if (S == 1) {
-    unsigned long long best = ~0ull;
-    for (int j = tid; j < M; j += kUpdThreads) {
-      float acc;
-      const uint32_t key = slot_key(a, b, h, j, thr, &acc);
-      const unsigned long long k64 = (static_cast<unsigned long long>(key) << 32) | static_cast<uint32_t>(j);
-      best = k64 < best ? k64 : best;
-    }
-    for (int o = 16; o > 0; o >>= 1) {
-      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
-      best = other < best ? other : best;
-    }
-    if (lane == 0) sm.warp_min[warp] = best;
-    __syncthreads();
-    if (warp == 0) {
-      best = sm.warp_min[lane];
-      for (int o = 16; o > 0; o >>= 1) {
-        const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
-        best = other < best ? other : best;
-      }
-      if (lane == 0) {
-        sm.bcast[0] = static_cast<uint32_t>(best >> 32);
-        sm.bcast[1] = 1u;
-      }
-    }
-    __syncthreads();
-    T = sm.bcast[0];
-    if (T == kProtected) {  // every slot is inside the recent window
-      if (tid == 0) atomicOr(a.err, 2);
-      return;
-    }
-    take_eq = 1;  // the argmin slot is the first slot with key T
-  } else {
+  {
     uint32_t prefix = 0, mask = 0, kth = static_cast<uint32_t>(S);
     for (int pass = 0; pass < 4; ++pass) {
       const int shift = 24 - 8 * pass;
@@ -535,11 +502,159 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   }
 }
 
+// ------------------------------------------------------ S = 1 (decode) --
+// The selection is an argmin over (key, slot), so nothing is kept per slot:
+// a cluster of C CTAs per (b, kv head) (h2o_orig: per kv head, every b) splits
+// the M slots into C contiguous ranges.  Each thread computes acc_j for its
+// slots with all loads of a batch in flight (the score_inc rows, M + 1 long,
+// are not 16-byte aligned, so loads are 4-byte and coalesced), writes acc_j
+// back to scores and keeps the smallest (key << 32 | j).  The CTA minima meet
+// in CTA 0's shared memory; after a cluster barrier (which also orders every
+// score write before the ones below) CTA 0 writes the evicted slot: the new
+// token's score, position, evict_idx and its K and V rows.
+constexpr int kDThreads = 512;
+constexpr int kDBatch = 6;  // slots per thread per batch of loads
+
+__global__ void __launch_bounds__(kDThreads, 2) update_decode_kernel(const UpdateArgs a, int C) {
+  __shared__ unsigned long long wmin[kDThreads / 32];
+  __shared__ unsigned long long cmin[8];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rank = static_cast<int>(cluster_rank());
+  const bool orig = a.policy == H2O_POLICY_ORIG;
+  const int gidx = static_cast<int>(blockIdx.x) / C;
+  const int b0 = orig ? 0 : gidx / a.Hkv, h = orig ? gidx : gidx % a.Hkv;
+  const int nb = orig ? a.B : 1;
+  const int M = a.M, NK = M + 1, qg = a.qg;
+  const int thr = a.pos0 + 1 - a.W;
+  const int t_now = a.pos0 + 1;
+  const int per = (M + C - 1) / C;
+  const int jlo = min(M, rank * per), jhi = min(M, jlo + per);
+  const int32_t* pos_b0 = a.slot_pos + (static_cast<size_t>(b0) * a.Hkv + h) * M;
+
+  unsigned long long best = ~0ull;
+  for (int base = jlo + tid; base < jhi; base += kDThreads * kDBatch) {
+    int pos[kDBatch];
+    float kacc[kDBatch];
+#pragma unroll
+    for (int u = 0; u < kDBatch; ++u) {
+      const int j = base + u * kDThreads;
+      pos[u] = j < jhi ? pos_b0[j] : 0;
+    }
+    for (int bi = 0; bi < nb; ++bi) {
+      const int b = b0 + bi;
+      float* sc = a.scores + (static_cast<size_t>(b) * a.Hkv + h) * M;
+      const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK;
+      float t[kDBatch], old[kDBatch];
+#pragma unroll
+      for (int u = 0; u < kDBatch; ++u) {
+        const int j = base + u * kDThreads;
+        old[u] = j < jhi ? sc[j] : 0.f;
+        t[u] = j < jhi ? __ldg(inc + j) : 0.f;
+      }
+      for (int g = 1; g < qg; ++g) {
+        float x[kDBatch];
+#pragma unroll
+        for (int u = 0; u < kDBatch; ++u) {
+          const int j = base + u * kDThreads;
+          x[u] = j < jhi ? __ldg(inc + static_cast<size_t>(g) * NK + j) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < kDBatch; ++u) t[u] = __fadd_rn(t[u], x[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < kDBatch; ++u) {
+        const int j = base + u * kDThreads;
+        const float acc = __fadd_rn(old[u], t[u]);
+        if (j < jhi) sc[j] = acc;
+        kacc[u] = bi == 0 ? acc : __fadd_rn(kacc[u], acc);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kDBatch; ++u) {
+      const int j = base + u * kDThreads;
+      if (j < jhi) {
+        const uint32_t key = make_key(kacc[u], pos[u], thr, a.policy, t_now);
+        const unsigned long long k64 =
+            (static_cast<unsigned long long>(key) << 32) | static_cast<uint32_t>(j);
+        best = k64 < best ? k64 : best;
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+    best = other < best ? other : best;
+  }
+  if (lane == 0) wmin[warp] = best;
+  __syncthreads();
+  if (warp == 0) {
+    best = lane < kDThreads / 32 ? wmin[lane] : ~0ull;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+      best = other < best ? other : best;
+    }
+    if (lane == 0) {
+      const uint32_t dst = cluster_addr(&cmin[rank], 0);
+      asm volatile("st.shared::cluster.u64 [%0], %1;" ::"r"(dst), "l"(best) : "memory");
+    }
+  }
+  // every CTA's minimum has landed in CTA 0, and every acc write is ordered
+  // before CTA 0's writes below
+  cluster_sync_all();
+  if (rank != 0) return;
+  if (warp == 0) {
+    best = lane < C ? cmin[lane] : ~0ull;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+      best = other < best ? other : best;
+    }
+    if (lane == 0) wmin[0] = best;
+  }
+  __syncthreads();
+  best = wmin[0];
+  if (static_cast<uint32_t>(best >> 32) == kProtected) {  // every slot inside the window
+    if (tid == 0) atomicOr(a.err, 2);
+    return;
+  }
+  const int e = static_cast<int>(best & 0xFFFFFFFFu);
+  for (int bi = warp; bi < nb; bi += kDThreads / 32) {
+    const int b = b0 + bi;
+    const int grp = b * a.Hkv + h;
+    if (lane == 0) {
+      const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK;
+      a.scores[static_cast<size_t>(grp) * M + e] = group_sum(inc, NK, qg, M);
+      a.slot_pos[static_cast<size_t>(grp) * M + e] = a.pos0;
+      if (a.evict_idx) a.evict_idx[grp] = e;
+    }
+    copy_row(a, grp, 0, e, lane);
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
   const size_t smem = (2 * static_cast<size_t>(a.M) + 2 * static_cast<size_t>(a.S)) * sizeof(uint32_t);
   const bool smem_path = a.S > 1 && smem <= kMaxClusterSmem;
+  if (a.S == 1) {
+    int C = a.M / 8192;
+    C = C < 1 ? 1 : (C > 8 ? 8 : C);
+    const int groups = a.policy == H2O_POLICY_ORIG ? a.Hkv : a.B * a.Hkv;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(groups * C));
+    cfg.blockDim = dim3(kDThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = static_cast<unsigned>(C);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, update_decode_kernel, a, C);
+  }
   if (!smem_path) {
     const int groups = a.policy == H2O_POLICY_ORIG ? a.Hkv : a.B * a.Hkv;
     update_kernel<<<groups, kUpdThreads, 0, stream>>>(a);

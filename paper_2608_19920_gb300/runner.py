@@ -40,6 +40,7 @@ class H2OLayer:
         self.scores = torch.zeros((B, Hkv, M), dtype=torch.float32, device=dev)
         self._inc = {}
         self._evict = {}
+        self._ws = {}
         self.keep_evictions = keep_evictions
         self.device = dev
 
@@ -53,7 +54,9 @@ class H2OLayer:
                                        device=self.device)
             self._evict[s] = torch.empty((self.B, self.Hkv, s), dtype=torch.int32,
                                          device=self.device)
-        return self._inc[s], self._evict[s]
+            n = lib.h2o_workspace_size(lib.H2ODims(self.B, self.Hq, self.Hkv, self.d, s, self.M))
+            self._ws[s] = torch.empty(n, dtype=torch.uint8, device=self.device) if n else None
+        return self._inc[s], self._evict[s], self._ws[s]
 
     def step(self, q, k_new, v_new, pos0: int, out=None, stream=None):
         """One chunk: attend (writes out, score_inc), then update the cache in place.
@@ -61,9 +64,10 @@ class H2OLayer:
         Returns (out, score_inc, evict_idx); the last two are reused buffers.
         """
         s = q.shape[2]
-        inc, ev = self._buf(s)
+        inc, ev, ws = self._buf(s)
         out, inc = lib.h2o_sdpa_chunk(q, self.k_cache, self.v_cache, k_new, v_new, self.slot_pos,
-                                      pos0, self.scale, out=out, score_inc=inc, stream=stream)
+                                      pos0, self.scale, out=out, score_inc=inc, workspace=ws,
+                                      stream=stream)
         lib.h2o_update(self.scores, self.slot_pos, inc, k_new, v_new, self.k_cache, self.v_cache,
                        pos0, self.W, evict_idx=ev if self.keep_evictions else None, stream=stream,
                        policy=self.policy)

@@ -12,7 +12,7 @@ from paper_2608_19920_gb300 import build as build_mod
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "h2o.h")
 
-OK, NULL, SHAPE, ALIGN, UNSUP, ARG = 0, -1, -2, -3, -4, -6
+OK, NULL, SHAPE, ALIGN, UNSUP, WORKSPACE, ARG = 0, -1, -2, -3, -4, -5, -6
 
 
 @pytest.fixture(scope="module")
@@ -63,6 +63,30 @@ def test_sdpa_argument_checks(lib):
     n = ctypes.c_size_t(7)
     assert lib.h2o_workspace_size(ctypes.byref(_dims()), ctypes.byref(n)) == OK and n.value == 0
     assert lib.h2o_workspace_size(ctypes.byref(_dims(d=32)), ctypes.byref(n)) == UNSUP
+
+
+def test_decode_workspace(lib):
+    """S = 1 with a cache takes the split-K decode kernels, whose per-split
+    partials (max, sum, d outputs per query head) live in the caller's workspace."""
+    n = ctypes.c_size_t(0)
+    dims = _dims(B=8, Hq=32, Hkv=8, d=128, S=1, M=65536)
+    assert lib.h2o_workspace_size(ctypes.byref(dims), ctypes.byref(n)) == OK
+    # 64 (b, kv head) groups x 65536 slots over 608 CTAs -> splits of 2048 slots
+    assert n.value == 8 * 32 * (65536 // 2048) * (2 + 128) * 4
+    small = _dims(B=1, Hq=4, Hkv=2, d=64, S=1, M=100)
+    assert lib.h2o_workspace_size(ctypes.byref(small), ctypes.byref(n)) == OK
+    assert n.value == 1 * 4 * 1 * (2 + 64) * 4
+    # no cache, or a GQA group above 8: the chunk kernel, no workspace
+    for d_ in (_dims(S=1, M=0), _dims(Hq=16, Hkv=1, S=1, M=100)):
+        assert lib.h2o_workspace_size(ctypes.byref(d_), ctypes.byref(n)) == OK and n.value == 0
+    # a missing or short workspace is refused before anything runs
+    vp = ctypes.c_void_p
+    ptrs = [vp(0x1000)] * 8
+    assert lib.h2o_sdpa_chunk(ctypes.byref(small), 100, 0.0, *ptrs, None, 0, None) == WORKSPACE
+    assert lib.h2o_sdpa_chunk(ctypes.byref(small), 100, 0.0, *ptrs, vp(0x2000), 4 * 66 * 4 - 1,
+                              None) == WORKSPACE
+    assert lib.h2o_sdpa_chunk(ctypes.byref(small), 100, 0.0, *ptrs, vp(0x2004), 4 * 66 * 4,
+                              None) == ALIGN
 
 
 def _upd(lib, dims, budget=256, W=32, pos0=256, ptrs=None, evict=None):

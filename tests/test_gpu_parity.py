@@ -106,6 +106,51 @@ def test_sdpa_chunk_matches_oracle(dev, case):
     np.testing.assert_allclose(inc.sum(-1).cpu().numpy(), S, rtol=1e-4)
 
 
+DECODE_CASES = [
+    # B, Hq, Hkv, d, M, n_empty, n_future, pos0, empty block [lo, hi)
+    (1, 4, 1, 128, 1, 0, 0, 5, None),            # a single cache slot
+    (2, 8, 2, 128, 63, 0, 0, 100, None),         # less than one 64-key tile
+    (1, 5, 1, 128, 64, 0, 0, 70, None),          # q_g = 5 (the 8-head variant)
+    (2, 16, 2, 128, 1000, 37, 20, 2000, None),   # q_g = 8, empty and future slots
+    (2, 4, 4, 128, 5000, 600, 0, 6000, None),    # q_g = 1, 20 splits with a ragged last one
+    (1, 8, 2, 64, 3000, 0, 0, 5000, (256, 768)), # d = 64; whole splits see no key
+    (1, 32, 2, 64, 200, 0, 0, 300, None),        # q_g = 16: the chunk kernel takes S = 1
+    (8, 32, 8, 128, 4096, 0, 0, 4200, None),     # the decode workload's shape, M = 4096
+]
+
+
+@pytest.mark.parametrize("case", DECODE_CASES, ids=lambda c: "x".join(map(str, c[:8])))
+def test_decode_step_matches_oracle(dev, case):
+    """S = 1: the split-K decode kernels (split + combine) against the oracle."""
+    B, Hq, Hkv, d, M, n_empty, n_future, pos0, block = case
+    rng = np.random.default_rng(hash(case) % 2**32)
+    st = wl.random_state(rng, B, Hkv, M, d, pos0=pos0, n_empty=n_empty)
+    for b in range(B):
+        for h in range(Hkv):
+            occ = np.nonzero(st["slot_pos"][b, h] >= 0)[0]
+            st["slot_pos"][b, h, occ[:min(n_future, len(occ))]] = pos0 + 1 + np.arange(
+                min(n_future, len(occ)))  # not visible to the token at pos0
+    if block is not None:
+        st["slot_pos"][:, :, block[0]:block[1]] = -1
+    q = wl.round_bf16(rng.standard_normal((B, Hq, 1, d), dtype=np.float32))
+    kn = wl.round_bf16(rng.standard_normal((B, Hkv, 1, d), dtype=np.float32))
+    vn = wl.round_bf16(rng.standard_normal((B, Hkv, 1, d), dtype=np.float32))
+    for rep in range(2):  # the same workspace twice in a row
+        out, inc = h2o_sdpa_chunk(bf(q, dev), bf(st["k_cache"], dev), bf(st["v_cache"], dev),
+                                  bf(kn, dev), bf(vn, dev),
+                                  torch.from_numpy(st["slot_pos"]).to(dev), pos0)
+        torch.cuda.synchronize()
+        assert h2o_device_errors() == 0
+        ref_out, ref_inc, _ = ref_sdpa(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"],
+                                       pos0)
+        check_sdpa(out, inc, ref_out, ref_inc)
+        np.testing.assert_allclose(inc.sum(-1).cpu().numpy(), 1.0, rtol=1e-4)
+        # masked slots get exactly zero weight
+        hidden = (st["slot_pos"] < 0) | (st["slot_pos"] > pos0)
+        g_hidden = np.repeat(hidden, Hq // Hkv, axis=1)
+        assert (inc[:, :, :M].cpu().numpy()[g_hidden] == 0).all()
+
+
 def test_softmax_scale_argument(dev):
     rng = np.random.default_rng(11)
     B, Hq, Hkv, d, S, M, pos0 = 1, 4, 2, 64, 40, 200, 300
@@ -132,6 +177,9 @@ UPDATE_CASES = [
     (1, 2, 1, 64, 5, 2000, 100, 1500, True),   # many empty slots and ties
     (1, 2, 1, 64, 33, 1030, 0, 0, True),       # M not a multiple of the block size
     (4, 32, 8, 128, 256, 2048, 256, 0, False), # batched workload shape
+    (2, 8, 2, 128, 1, 16384, 64, 0, False),    # S = 1, clusters of 2
+    (1, 4, 2, 64, 1, 65536, 64, 3, True),      # S = 1, clusters of 8, ties and empties
+    (2, 8, 2, 64, 1, 9000, 0, 0, True),        # S = 1, no recent window, ragged ranges
 ]
 
 
@@ -179,6 +227,7 @@ POLICY_CASES = [
     (3, 4, 2, 64, 1, 500, 64, 0, False),        # S = 1: argmin path
     (2, 4, 1, 64, 40, 26000, 100, 0, False),    # keys beyond the cluster variant's shared memory
     (4, 32, 8, 128, 256, 2048, 256, 0, False),  # batched workload shape
+    (3, 12, 3, 64, 1, 40000, 64, 0, False),     # S = 1, clusters of 4 (h2o_orig: 3 b each)
 ]
 
 

@@ -505,13 +505,15 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
 // ------------------------------------------------------ S = 1 (decode) --
 // The selection is an argmin over (key, slot), so nothing is kept per slot:
 // a cluster of C CTAs per (b, kv head) (h2o_orig: per kv head, every b) splits
-// the M slots into C contiguous ranges.  Each thread computes acc_j for its
-// slots with all loads of a batch in flight (the score_inc rows, M + 1 long,
-// are not 16-byte aligned, so loads are 4-byte and coalesced), writes acc_j
-// back to scores and keeps the smallest (key << 32 | j).  The CTA minima meet
-// in CTA 0's shared memory; after a cluster barrier (which also orders every
-// score write before the ones below) CTA 0 writes the evicted slot: the new
-// token's score, position, evict_idx and its K and V rows.
+// the M slots into C contiguous ranges.  Pass 1: each thread computes acc_j
+// and the key of its slots with all loads of a batch in flight (the score_inc
+// rows, M + 1 long, are not 16-byte aligned, so loads are 4-byte and
+// coalesced) and keeps the smallest (key << 32 | j).  Every CTA sends its
+// minimum to every CTA of the cluster; after a cluster barrier all know the
+// evicted slot.  Pass 2 (nothing is written before it, so a (b, h) without a
+// candidate stays unchanged): each CTA recomputes and writes acc_j of its
+// range, and the CTA holding the evicted slot writes the new token's score,
+// position, evict_idx and K/V rows there.
 constexpr int kDThreads = 512;
 constexpr int kDBatch = 6;  // slots per thread per batch of loads
 
@@ -531,6 +533,33 @@ __global__ void __launch_bounds__(kDThreads, 2) update_decode_kernel(const Updat
   const int jlo = min(M, rank * per), jhi = min(M, jlo + per);
   const int32_t* pos_b0 = a.slot_pos + (static_cast<size_t>(b0) * a.Hkv + h) * M;
 
+  // acc_j (Eq. 3) of batch entry b for the slots base + u * kDThreads, heads
+  // of the group added in ascending order, no fused multiply-add
+  auto batch_acc = [&](int b, int base, float (&acc)[kDBatch]) {
+    const float* sc = a.scores + (static_cast<size_t>(b) * a.Hkv + h) * M;
+    const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK;
+    float t[kDBatch], old[kDBatch];
+#pragma unroll
+    for (int u = 0; u < kDBatch; ++u) {
+      const int j = base + u * kDThreads;
+      old[u] = j < jhi ? sc[j] : 0.f;
+      t[u] = j < jhi ? __ldg(inc + j) : 0.f;
+    }
+    for (int g = 1; g < qg; ++g) {
+      float x[kDBatch];
+#pragma unroll
+      for (int u = 0; u < kDBatch; ++u) {
+        const int j = base + u * kDThreads;
+        x[u] = j < jhi ? __ldg(inc + static_cast<size_t>(g) * NK + j) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < kDBatch; ++u) t[u] = __fadd_rn(t[u], x[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < kDBatch; ++u) acc[u] = __fadd_rn(old[u], t[u]);
+  };
+
+  // ---- pass 1: the smallest (key, slot) of this CTA's range
   unsigned long long best = ~0ull;
   for (int base = jlo + tid; base < jhi; base += kDThreads * kDBatch) {
     int pos[kDBatch];
@@ -541,33 +570,10 @@ __global__ void __launch_bounds__(kDThreads, 2) update_decode_kernel(const Updat
       pos[u] = j < jhi ? pos_b0[j] : 0;
     }
     for (int bi = 0; bi < nb; ++bi) {
-      const int b = b0 + bi;
-      float* sc = a.scores + (static_cast<size_t>(b) * a.Hkv + h) * M;
-      const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK;
-      float t[kDBatch], old[kDBatch];
+      float acc[kDBatch];
+      batch_acc(b0 + bi, base, acc);
 #pragma unroll
-      for (int u = 0; u < kDBatch; ++u) {
-        const int j = base + u * kDThreads;
-        old[u] = j < jhi ? sc[j] : 0.f;
-        t[u] = j < jhi ? __ldg(inc + j) : 0.f;
-      }
-      for (int g = 1; g < qg; ++g) {
-        float x[kDBatch];
-#pragma unroll
-        for (int u = 0; u < kDBatch; ++u) {
-          const int j = base + u * kDThreads;
-          x[u] = j < jhi ? __ldg(inc + static_cast<size_t>(g) * NK + j) : 0.f;
-        }
-#pragma unroll
-        for (int u = 0; u < kDBatch; ++u) t[u] = __fadd_rn(t[u], x[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < kDBatch; ++u) {
-        const int j = base + u * kDThreads;
-        const float acc = __fadd_rn(old[u], t[u]);
-        if (j < jhi) sc[j] = acc;
-        kacc[u] = bi == 0 ? acc : __fadd_rn(kacc[u], acc);
-      }
+      for (int u = 0; u < kDBatch; ++u) kacc[u] = bi == 0 ? acc[u] : __fadd_rn(kacc[u], acc[u]);
     }
 #pragma unroll
     for (int u = 0; u < kDBatch; ++u) {
@@ -594,31 +600,35 @@ __global__ void __launch_bounds__(kDThreads, 2) update_decode_kernel(const Updat
       const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
       best = other < best ? other : best;
     }
-    if (lane == 0) {
-      const uint32_t dst = cluster_addr(&cmin[rank], 0);
+    // this CTA's minimum into slot `rank` of every CTA of the cluster
+    if (lane < C) {
+      const uint32_t dst = cluster_addr(&cmin[rank], static_cast<uint32_t>(lane));
       asm volatile("st.shared::cluster.u64 [%0], %1;" ::"r"(dst), "l"(best) : "memory");
     }
   }
-  // every CTA's minimum has landed in CTA 0, and every acc write is ordered
-  // before CTA 0's writes below
   cluster_sync_all();
-  if (rank != 0) return;
-  if (warp == 0) {
-    best = lane < C ? cmin[lane] : ~0ull;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
-      best = other < best ? other : best;
-    }
-    if (lane == 0) wmin[0] = best;
-  }
-  __syncthreads();
-  best = wmin[0];
+  best = ~0ull;
+  for (int r = 0; r < C; ++r) best = cmin[r] < best ? cmin[r] : best;
   if (static_cast<uint32_t>(best >> 32) == kProtected) {  // every slot inside the window
-    if (tid == 0) atomicOr(a.err, 2);
+    if (rank == 0 && tid == 0) atomicOr(a.err, 2);
     return;
   }
   const int e = static_cast<int>(best & 0xFFFFFFFFu);
+
+  // ---- pass 2: write acc_j of this range; the evicted slot takes the new token
+  for (int base = jlo + tid; base < jhi; base += kDThreads * kDBatch) {
+    for (int bi = 0; bi < nb; ++bi) {
+      float acc[kDBatch];
+      batch_acc(b0 + bi, base, acc);
+      float* sc = a.scores + (static_cast<size_t>(b0 + bi) * a.Hkv + h) * M;
+#pragma unroll
+      for (int u = 0; u < kDBatch; ++u) {
+        const int j = base + u * kDThreads;
+        if (j < jhi && j != e) sc[j] = acc[u];
+      }
+    }
+  }
+  if (e < jlo || e >= jhi) return;
   for (int bi = warp; bi < nb; bi += kDThreads / 32) {
     const int b = b0 + bi;
     const int grp = b * a.Hkv + h;

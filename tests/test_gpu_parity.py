@@ -324,6 +324,25 @@ def test_update_reports_too_few_candidates_and_leaves_state(dev):
     assert h2o_device_errors() == 0
 
 
+@pytest.mark.parametrize("M", [16, 20000])
+def test_decode_update_reports_too_few_candidates_and_leaves_state(dev, M):
+    """S = 1 (cluster argmin kernel): every slot inside the window."""
+    B, Hq, Hkv, d, W = 2, 4, 2, 64, 8
+    pos0 = 100
+    sp = np.full((B, Hkv, M), pos0 - 1, np.int32)
+    g_pos = torch.from_numpy(sp).to(dev)
+    sc = np.random.default_rng(3).random((B, Hkv, M), dtype=np.float32)
+    g_scores = torch.from_numpy(sc).to(dev)
+    g_k = torch.zeros((B, Hkv, M, d), dtype=torch.bfloat16, device=dev)
+    kn = torch.ones((B, Hkv, 1, d), dtype=torch.bfloat16, device=dev)
+    h2o_update(g_scores, g_pos, torch.ones((B, Hq, M + 1), device=dev), kn, kn, g_k,
+               torch.zeros_like(g_k), pos0, W)
+    assert h2o_device_errors() == 2
+    assert (g_pos.cpu().numpy() == sp).all() and g_k.abs().sum().item() == 0
+    np.testing.assert_array_equal(g_scores.cpu().numpy(), sc)
+    assert h2o_device_errors() == 0
+
+
 def _teacher_forced_step(layer, q, kn, vn, p, W):
     """Runs one GPU step and checks it against the oracle started from the GPU's state."""
     before = dict(k=f32(layer.k_cache), v=f32(layer.v_cache), pos=layer.slot_pos.cpu().numpy(),

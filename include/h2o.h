@@ -108,6 +108,31 @@ H2O_API int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_s
                    void* stream);
 
 /*
+ * h2o_sdpa_chunk for one query token per sequence (dims->S == 1, M >= 1,
+ * Hq / Hkv <= 8), with no workspace argument: it allocates nothing.  The
+ * paper has no counterpart; this entry point exists for callers that cannot
+ * allocate device memory around the call.
+ *
+ * Its scratch (the per-split partial max, sum and output of every query head,
+ * h2o_workspace_size(dims) bytes) is a fixed device array of 8 MiB inside the
+ * library, one per device; dims needing more are rejected with
+ * H2O_ERR_WORKSPACE and nothing runs.  Other sizes outside the decode case
+ * give H2O_ERR_UNSUPPORTED.  Arguments, outputs and the other errors are
+ * those of h2o_sdpa_chunk.
+ *
+ *  - The first call on a device looks up the array's address on that device
+ *    (with the device current); make that first call before any stream capture.
+ *  - Every call on a device shares the one array: calls whose kernels overlap
+ *    on the GPU (different streams, no ordering between them) race on it.
+ *    Nothing in it needs to start at zero; each call writes every entry it
+ *    reads.
+ */
+H2O_API int h2o_sdpa_decode_static(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                   const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
+                   h2o_bf16* out, float* score_inc, void* stream);
+
+/*
  * H2O cache update after h2o_sdpa_chunk (§3.1.1 Eq. 3 and the eviction rule
  * that follows it; scatter of §3.2 / §A.1.1).  Per (b, kv head h):
  *

@@ -20,7 +20,8 @@ H2O_DEVERR_TIMEOUT = 1
 H2O_DEVERR_CANDIDATES = 2
 
 # Every symbol include/h2o.h declares.
-EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_update_policy",
+EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
+           "h2o_update_policy",
            "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
            "h2o_version")
 
@@ -60,13 +61,15 @@ def load(path: str = LIB_PATH):
     lib.h2o_workspace_size.argtypes = [dims_p, ctypes.POINTER(ctypes.c_size_t)]
     lib.h2o_sdpa_chunk.argtypes = [dims_p, i64, f32, vp, vp, vp, vp, vp, vp, vp, vp, vp,
                                    ctypes.c_size_t, vp]
+    lib.h2o_sdpa_decode_static.argtypes = [dims_p, i64, f32, vp, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.h2o_update.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, vp]
     lib.h2o_update_policy.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, i32, i32, i32,
                                       vp, vp]
     lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_status_string.argtypes = [ctypes.c_int]
     lib.h2o_status_string.restype = ctypes.c_char_p
-    for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_update", "h2o_update_policy",
+    for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
+               "h2o_update_policy",
                "h2o_cache_reset",
                "h2o_last_cuda_error",
                "h2o_device_errors", "h2o_version"):
@@ -154,6 +157,37 @@ def h2o_sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale
                             _ptr(v_cache), _ptr(k_new), _ptr(v_new), _ptr(slot_pos), _ptr(out),
                             _ptr(score_inc), _ptr(workspace), ws_bytes, _stream(stream))
     _check("h2o_sdpa_chunk", st)
+    return out, score_inc
+
+
+def h2o_sdpa_decode_static(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int,
+                           scale: float = 0.0, out=None, score_inc=None, stream=None):
+    """h2o_sdpa_chunk for S = 1 on the library's fixed scratch (see include/h2o.h):
+    the call itself allocates nothing on the device (``out`` and ``score_inc``
+    are allocated here only when not given)."""
+    lib = load()
+    dev = q.device
+    B, Hq, S, d = q.shape
+    Hkv = k_new.shape[1]
+    M = k_cache.shape[2]
+    bf = torch.bfloat16
+    _expect(q, "q", (B, Hq, S, d), bf, dev)
+    _expect(k_cache, "k_cache", (B, Hkv, M, d), bf, dev)
+    _expect(v_cache, "v_cache", (B, Hkv, M, d), bf, dev)
+    _expect(k_new, "k_new", (B, Hkv, S, d), bf, dev)
+    _expect(v_new, "v_new", (B, Hkv, S, d), bf, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    if out is None:
+        out = torch.empty((B, Hq, S, d), dtype=bf, device=dev)
+    if score_inc is None:
+        score_inc = torch.empty((B, Hq, M + S), dtype=torch.float32, device=dev)
+    _expect(out, "out", (B, Hq, S, d), bf, dev)
+    _expect(score_inc, "score_inc", (B, Hq, M + S), torch.float32, dev)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    st = lib.h2o_sdpa_decode_static(ctypes.byref(dims), int(pos0), float(scale), _ptr(q),
+                                    _ptr(k_cache), _ptr(v_cache), _ptr(k_new), _ptr(v_new),
+                                    _ptr(slot_pos), _ptr(out), _ptr(score_inc), _stream(stream))
+    _check("h2o_sdpa_decode_static", st)
     return out, score_inc
 
 

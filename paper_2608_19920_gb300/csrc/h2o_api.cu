@@ -61,6 +61,14 @@ int current_device(DeviceInfo** out) {
   return H2O_OK;
 }
 
+// Address of the decode kernels' fixed scratch on each device, resolved once.
+struct StaticScratch {
+  std::once_flag once;
+  cudaError_t status = cudaSuccess;
+  void* ptr = nullptr;
+};
+StaticScratch g_static_scratch[kMaxDevices];
+
 int get_encoder() {
   std::call_once(g_encode_once, [] {
     cudaDriverEntryPointQueryResult q;
@@ -237,6 +245,49 @@ int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, co
   e = launch_sdpa(a, s);
   if (e != cudaSuccess) return cuda_fail(e);
   return H2O_OK;
+}
+
+int h2o_sdpa_decode_static(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                           const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                           const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
+                           h2o_bf16* out, float* score_inc, void* stream) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (!q || !k_cache || !v_cache || !k_new || !v_new || !slot_pos || !out || !score_inc)
+    return H2O_ERR_NULL;
+  if (misaligned(q) || misaligned(k_cache) || misaligned(v_cache) || misaligned(k_new) ||
+      misaligned(v_new) || misaligned(slot_pos) || misaligned(out) || misaligned(score_inc))
+    return H2O_ERR_ALIGN;
+  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
+  int split_len = 0, n_split = 0;
+  size_t ws_need = 0;
+  if (!decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need))
+    return H2O_ERR_UNSUPPORTED;
+  if (ws_need > kDecodeStaticScratchBytes) return H2O_ERR_WORKSPACE;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  StaticScratch& ss = g_static_scratch[dev];  // dev < kMaxDevices: current_device checked it
+  std::call_once(ss.once, [&ss] { ss.status = decode_static_scratch(&ss.ptr); });
+  if (ss.status != cudaSuccess) return cuda_fail(ss.status);
+
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
+  DecodeArgs a;
+  a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
+  a.slot_pos = slot_pos; a.out = out; a.score_inc = score_inc;
+  a.part = static_cast<float*>(ss.ptr);
+  a.err = di->err_word;
+  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.M = D.M; a.qg = D.Hq / D.Hkv;
+  a.pos0 = static_cast<int>(pos0);
+  a.scale_log2 = scale * 1.4426950408889634f;
+  a.split_len = split_len;
+  a.n_split = n_split;
+  e = launch_decode(a, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
 }
 
 int h2o_update(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,

@@ -469,6 +469,15 @@ bool decode_plan(int B, int Hq, int Hkv, int d, int S, int M, int* split_len, in
   return true;
 }
 
+// The per-split partials of h2o_sdpa_decode_static live here instead of in a
+// caller's workspace.  Every entry a call reads was written earlier in the
+// same call, so nothing needs clearing between calls.
+static __device__ __align__(256) unsigned char g_decode_static_scratch[kDecodeStaticScratchBytes];
+
+cudaError_t decode_static_scratch(void** ptr) {
+  return cudaGetSymbolAddress(ptr, g_decode_static_scratch);
+}
+
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   return a.d == 128 ? launch_d<128>(a, stream) : launch_d<64>(a, stream);
 }

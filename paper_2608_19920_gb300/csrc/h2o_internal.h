@@ -82,6 +82,12 @@ struct DecodeArgs {
 bool decode_plan(int B, int Hq, int Hkv, int d, int S, int M, int* split_len, int* n_split,
                  size_t* ws_bytes);
 
+// Fixed scratch of h2o_sdpa_decode_static (a file-scope device array in
+// h2o_decode.cu, shared by every call on a device): its size and its address
+// on the current device.
+constexpr size_t kDecodeStaticScratchBytes = size_t(8) << 20;
+cudaError_t decode_static_scratch(void** ptr);
+
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);

@@ -28,6 +28,7 @@
 // Bytes per step: K and V once (the algorithmic 2 B d per slot each), plus
 // the score_inc row written as logits, read and written again as weights.
 #include <algorithm>
+#include <cstdint>
 
 #include "h2o_internal.h"
 #include "sm100.cuh"
@@ -52,7 +53,8 @@ struct DecGeom {
 
 struct alignas(16) DecHead {  // 16-byte size: the logits after it are read as float4
   uint64_t full[kDecStages];
-  float red[kDecWarps][kDecodeMaxQg];
+  float red[kDecWarps][kDecodeMaxQg];   // per-warp maxima
+  float red2[kDecWarps][kDecodeMaxQg];  // per-warp sums
   int abort;
 };
 
@@ -113,6 +115,45 @@ __device__ __forceinline__ int scatter_head(uint32_t lane) {
   return QG == 8 ? static_cast<int>(lane & 7u) : static_cast<int>((lane >> 1) & 3u);
 }
 
+// One (b, kv head, split) work item.
+struct DecItem {
+  int grp, s, j0, n_cache, n_loc, n_tiles;
+  bool last;
+};
+
+template <int D>
+__device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int it) {
+  DecItem x;
+  x.grp = it / a.n_split;
+  x.s = it % a.n_split;
+  x.j0 = x.s * a.split_len;
+  x.n_cache = min(a.split_len, a.M - x.j0);  // >= 1: n_split = ceil(M / split_len)
+  x.last = x.s == a.n_split - 1;
+  x.n_loc = x.n_cache + (x.last ? 1 : 0);    // local key n_cache is the new token
+  x.n_tiles = (x.n_loc + DecGeom<D>::kTileKeys - 1) / DecGeom<D>::kTileKeys;
+  return x;
+}
+
+// Keys per thread in the per-item passes over the split (256 threads).
+constexpr int kKeysPerThread = (kDecodeMaxSplitLen + 1 + kDecThreads - 1) / kDecThreads;
+
+// Reduces QG values per thread over the block: warp shuffles, then one row of
+// `red` per warp; every thread then reads the 8 rows.
+template <int QG, bool kMax>
+__device__ __forceinline__ void block_reduce_qg(float (&v)[QG], float (*red)[kDecodeMaxQg],
+                                                int warp, uint32_t lane) {
+#pragma unroll
+  for (int g = 0; g < QG; ++g)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float y = __shfl_xor_sync(0xffffffffu, v[g], o);
+      v[g] = kMax ? fmaxf(v[g], y) : v[g] + y;
+    }
+  if (lane == 0)
+#pragma unroll
+    for (int g = 0; g < QG; ++g) red[warp][g] = v[g];
+}
+
 template <int D, int QG>
 __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
     decode_split_kernel(const DecodeArgs a) {
@@ -122,22 +163,13 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
   DecHead& hd = *reinterpret_cast<DecHead*>(dsm + kDecStages * kDecTileBytes);
   static_assert(sizeof(DecHead) % 16 == 0, "logits must stay 16-byte aligned");
   float* lg = reinterpret_cast<float*>(dsm + kDecStages * kDecTileBytes + sizeof(DecHead));
+  float* red_o = lg + (a.split_len + 1) * QG;  // [warp][g][D]
+  // q rows of the item whose first K tile sits in ring slot x: qbuf + x * QG * D
+  uint16_t* qbuf = reinterpret_cast<uint16_t*>(red_o + kDecWarps * QG * D);
 
   const int tid = threadIdx.x, warp = tid >> 5;
   const uint32_t lane = static_cast<uint32_t>(tid & 31);
-  const int s = blockIdx.x;
-  const int grp = blockIdx.y;  // b * Hkv + h
-  const int b = grp / a.Hkv, h = grp % a.Hkv;
-  const int j0 = s * a.split_len;
-  const int n_cache = min(a.split_len, a.M - j0);  // >= 1: n_split = ceil(M / split_len)
-  const bool last = s == a.n_split - 1;
-  const int n_loc = n_cache + (last ? 1 : 0);       // local key n_cache is the new token
-  const int n_tiles = (n_loc + G::kTileKeys - 1) / G::kTileKeys;
-  const int n_all = 2 * n_tiles;                    // K tiles, then V tiles
-  const uint16_t* kc = a.k_cache + (static_cast<size_t>(grp) * a.M + j0) * D;
-  const uint16_t* vc = a.v_cache + (static_cast<size_t>(grp) * a.M + j0) * D;
-  const uint16_t* kn = a.k_new + static_cast<size_t>(grp) * D;
-  const uint16_t* vn = a.v_new + static_cast<size_t>(grp) * D;
+  const int n_items = a.n_split * a.B * a.Hkv;
 
   if (tid == 0) {
 #pragma unroll
@@ -147,139 +179,189 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
   }
   __syncthreads();
 
-  // tile t < n_tiles: K rows of local keys [t T, t T + T); then the same for V
-  auto issue = [&](int t) {
-    const bool is_v = t >= n_tiles;
-    const int k0 = (is_v ? t - n_tiles : t) * G::kTileKeys;
-    const int k1 = min(k0 + G::kTileKeys, n_loc);
-    const int rows_c = max(0, min(k1, n_cache) - k0);
-    const bool has_new = last && k1 > n_cache;
-    uint8_t* dst = ring + (t % kDecStages) * kDecTileBytes;
-    uint64_t* bar = &hd.full[t % kDecStages];
-    bar_expect_tx(bar, static_cast<uint32_t>((rows_c + (has_new ? 1 : 0)) * G::kRowBytes));
-    if (rows_c > 0)
-      bulk_load_once(dst, (is_v ? vc : kc) + static_cast<size_t>(k0) * D,
-                     static_cast<uint32_t>(rows_c * G::kRowBytes), bar);
-    if (has_new)
-      bulk_load_once(dst + rows_c * G::kRowBytes, is_v ? vn : kn, G::kRowBytes, bar);
-  };
-  int issued = 0;  // meaningful in thread 0 only
-  if (tid == 0) {
-    for (; issued < min(kDecStages, n_all); ++issued) issue(issued);
-  }
-
-  // this lane's slice of every head's query: chunks c0 (+ 8) of 8 elements
-  const int c0 = static_cast<int>(lane & 7u);
-  float qr[QG][8 * G::kCh];
-#pragma unroll
-  for (int g = 0; g < QG; ++g) {
-    if (g < a.qg) {
-      const uint16_t* qp = a.q + static_cast<size_t>(b * a.Hq + h * a.qg + g) * D;
-#pragma unroll
-      for (int ch = 0; ch < G::kCh; ++ch)
-        bf16x8_to_f32(__ldg(reinterpret_cast<const uint4*>(qp) + c0 + 8 * ch), &qr[g][8 * ch]);
-    } else {
-#pragma unroll
-      for (int e = 0; e < 8 * G::kCh; ++e) qr[g][e] = 0.f;
+  // Producer (thread 0): the CTA's items in order, each as its K tiles then
+  // its V tiles, one tile per ring slot freed; the stream of tiles runs on
+  // across items, so the ring never drains between them.
+  int issued = 0;
+  int p_it = blockIdx.x, p_t = 0;
+  DecItem p_x;
+  if (p_it < n_items) p_x = dec_item<D>(a, p_it);
+  auto issue_next = [&]() {
+    if (p_it >= n_items) return;
+    const bool is_v = p_t >= p_x.n_tiles;
+    const int k0 = (is_v ? p_t - p_x.n_tiles : p_t) * G::kTileKeys;
+    const int k1 = min(k0 + G::kTileKeys, p_x.n_loc);
+    const int rows_c = max(0, min(k1, p_x.n_cache) - k0);
+    const bool has_new = p_x.last && k1 > p_x.n_cache;
+    uint8_t* dst = ring + (issued % kDecStages) * kDecTileBytes;
+    uint64_t* bar = &hd.full[issued % kDecStages];
+    const uint32_t q_bytes = p_t == 0 ? static_cast<uint32_t>(a.qg * D * 2) : 0u;
+    bar_expect_tx(bar, static_cast<uint32_t>((rows_c + (has_new ? 1 : 0)) * G::kRowBytes) + q_bytes);
+    if (q_bytes) {
+      const int pb = p_x.grp / a.Hkv, ph = p_x.grp % a.Hkv;
+      bulk_load_once(qbuf + (issued % kDecStages) * QG * D,
+                     a.q + static_cast<size_t>(pb * a.Hq + ph * a.qg) * D, q_bytes, bar);
     }
-  }
+    if (rows_c > 0) {
+      const uint16_t* base = (is_v ? a.v_cache : a.k_cache) +
+                             (static_cast<size_t>(p_x.grp) * a.M + p_x.j0 + k0) * D;
+      bulk_load_once(dst, base, static_cast<uint32_t>(rows_c * G::kRowBytes), bar);
+    }
+    if (has_new)
+      bulk_load_once(dst + rows_c * G::kRowBytes,
+                     (is_v ? a.v_new : a.k_new) + static_cast<size_t>(p_x.grp) * D, G::kRowBytes,
+                     bar);
+    ++issued;
+    if (++p_t == 2 * p_x.n_tiles) {
+      p_t = 0;
+      p_it += gridDim.x;
+      if (p_it < n_items) p_x = dec_item<D>(a, p_it);
+    }
+  };
+  if (tid == 0)
+    for (int x = 0; x < kDecStages; ++x) issue_next();
 
-  const int hg = scatter_head<QG>(lane);
-  const bool writer = (QG == 8 || (lane & 1u) == 0) && hg < a.qg;
-  float* inc_row = a.score_inc + static_cast<size_t>(b * a.Hq + h * a.qg + (hg < a.qg ? hg : 0)) *
-                                     (static_cast<size_t>(a.M) + 1);
-  const int32_t* sp = a.slot_pos + static_cast<size_t>(grp) * a.M + j0;
   volatile int* abort_flag = &hd.abort;
+  const int c0 = static_cast<int>(lane & 7u);  // this lane's 16-byte chunks: c0 (+ 8)
+  const int hg = scatter_head<QG>(lane);
+  const bool dot_writer = (QG == 8 || (lane & 1u) == 0) && hg < a.qg;
+  int g_t = 0;  // tiles consumed so far (ring slot and phase)
 
-  // ---- Q K^T: logits of the split's keys (log2 units, masked = -inf)
-  float mx = -INFINITY;
-  int t = 0;
-  for (; t < n_tiles; ++t) {
-    const bool ok = wait_bar(&hd.full[t % kDecStages], (t / kDecStages) & 1, abort_flag,
-                             kWaitLimitNs);
-    if (ok) {
-      const uint8_t* tile = ring + (t % kDecStages) * kDecTileBytes;
-#pragma unroll 1
-      for (int r = 0; r < G::kTileKeys / 32; ++r) {
-        const int kk = r * 32 + warp * 4 + static_cast<int>(lane >> 3);  // key within the tile
-        const int kl = t * G::kTileKeys + kk;                             // key within the split
-        float dot[QG];
+  for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
+    const DecItem x = dec_item<D>(a, it);
+    const int b = x.grp / a.Hkv, h = x.grp % a.Hkv;
+    const size_t row0 = static_cast<size_t>(b * a.Hq + h * a.qg);  // first query head's row
+
+    // positions of the keys this thread masks below (in flight during Q K^T)
+    const int32_t* sp = a.slot_pos + static_cast<size_t>(x.grp) * a.M + x.j0;
+    int pos[kKeysPerThread];
 #pragma unroll
-        for (int g = 0; g < QG; ++g) dot[g] = 0.f;
-        if (kl < n_loc) {
-          const uint4* row = reinterpret_cast<const uint4*>(tile + kk * G::kRowBytes);
+    for (int u = 0; u < kKeysPerThread; ++u) {
+      const int k = tid + u * kDecThreads;
+      pos[u] = k < x.n_cache ? __ldg(sp + k) : 0;
+    }
+    // ---- Q K^T: raw dot products of the item's keys into lg
+    float qr[QG][8 * G::kCh];  // this lane's slice of every head's query
+    for (int t = 0; t < x.n_tiles; ++t, ++g_t) {
+      if (wait_bar(&hd.full[g_t % kDecStages], (g_t / kDecStages) & 1, abort_flag,
+                   kWaitLimitNs)) {
+        const uint8_t* tile = ring + (g_t % kDecStages) * kDecTileBytes;
+        if (t == 0) {  // the q rows arrived with this tile; read before its slot is reissued
+          const uint16_t* qs = qbuf + (g_t % kDecStages) * QG * D;
 #pragma unroll
-          for (int ch = 0; ch < G::kCh; ++ch) {
-            float kf[8];
-            bf16x8_to_f32(row[c0 + 8 * ch], kf);
+          for (int g = 0; g < QG; ++g) {
+            if (g < a.qg) {
 #pragma unroll
-            for (int e = 0; e < 8; ++e)
+              for (int ch = 0; ch < G::kCh; ++ch)
+                bf16x8_to_f32(reinterpret_cast<const uint4*>(qs + g * D)[c0 + 8 * ch],
+                              &qr[g][8 * ch]);
+            } else {
 #pragma unroll
-              for (int g = 0; g < QG; ++g) dot[g] = fmaf(qr[g][8 * ch + e], kf[e], dot[g]);
+              for (int e = 0; e < 8 * G::kCh; ++e) qr[g][e] = 0.f;
+            }
           }
         }
-        const float tot = reduce_scatter8<QG>(dot, lane);
-        if (writer && kl < n_loc) {
-          bool vis = true;
-          int j = a.M;  // the new token's column
-          if (kl < n_cache) {
-            const int pos = __ldg(sp + kl);
-            vis = pos >= 0 && pos <= a.pos0;
-            j = j0 + kl;
+#pragma unroll 1
+        for (int r = 0; r < G::kTileKeys / 32; ++r) {
+          const int kk = r * 32 + warp * 4 + static_cast<int>(lane >> 3);  // key within the tile
+          const int kl = t * G::kTileKeys + kk;                             // key within the item
+          float dot[QG];
+#pragma unroll
+          for (int g = 0; g < QG; ++g) dot[g] = 0.f;
+          if (kl < x.n_loc) {
+            const uint4* krow = reinterpret_cast<const uint4*>(tile + kk * G::kRowBytes);
+#pragma unroll
+            for (int ch = 0; ch < G::kCh; ++ch) {
+              float kf[8];
+              bf16x8_to_f32(krow[c0 + 8 * ch], kf);
+#pragma unroll
+              for (int e = 0; e < 8; ++e)
+#pragma unroll
+                for (int g = 0; g < QG; ++g) dot[g] = fmaf(qr[g][8 * ch + e], kf[e], dot[g]);
+            }
           }
-          const float v = vis ? tot * a.scale_log2 : -INFINITY;
-          lg[kl * QG + hg] = v;
-          inc_row[j] = v;
-          mx = fmaxf(mx, v);
+          const float tot = reduce_scatter8<QG>(dot, lane);
+          if (dot_writer && kl < x.n_loc) lg[kl * QG + hg] = tot;
+        }
+      }
+      __syncthreads();  // every warp is done with the slot; lg rows complete
+      if (*abort_flag) break;
+      if (tid == 0) issue_next();
+    }
+    if (*abort_flag) break;
+
+    // ---- mask, log2 scale, logits to score_inc (coalesced), split max
+    float mx[QG];
+#pragma unroll
+    for (int g = 0; g < QG; ++g) mx[g] = -INFINITY;
+#pragma unroll
+    for (int u = 0; u < kKeysPerThread; ++u) {
+      const int k = tid + u * kDecThreads;
+      if (k < x.n_loc) {
+        const bool vis = k < x.n_cache ? (pos[u] >= 0 && pos[u] <= a.pos0) : true;
+        const size_t j = k < x.n_cache ? static_cast<size_t>(x.j0 + k) : static_cast<size_t>(a.M);
+#pragma unroll
+        for (int g4 = 0; g4 < QG; g4 += 4) {
+          float4 v = *reinterpret_cast<const float4*>(lg + k * QG + g4);
+          float w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            w[e] = vis ? w[e] * a.scale_log2 : -INFINITY;
+            if (g4 + e < a.qg) {
+              a.score_inc[(row0 + g4 + e) * (static_cast<size_t>(a.M) + 1) + j] = w[e];
+              mx[g4 + e] = fmaxf(mx[g4 + e], w[e]);
+            }
+          }
+          *reinterpret_cast<float4*>(lg + k * QG + g4) = make_float4(w[0], w[1], w[2], w[3]);
         }
       }
     }
-    __syncthreads();  // every warp is done with the slot
-    if (*abort_flag) break;
-    if (tid == 0 && issued < n_all) issue(issued++);
-  }
-
-  // ---- split max per head, then p = exp2(a - m) in place and the split sum
-  const bool aborted_k = *abort_flag != 0;
-  if (!aborted_k) {
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-    if (QG == 4) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-    if (lane < 8u && (QG == 8 || (lane & 1u) == 0)) hd.red[warp][hg] = mx;
-  }
-  __syncthreads();
-  const int gp = tid % QG;  // the head of every lg entry this thread converts
-  float m_g = -INFINITY;
+    block_reduce_qg<QG, true>(mx, hd.red, warp, lane);
+    __syncthreads();
+    float m[QG];
 #pragma unroll
-  for (int w = 0; w < kDecWarps; ++w) m_g = fmaxf(m_g, hd.red[w][gp]);
-  float lsum = 0.f;
-  if (!aborted_k && gp < a.qg) {
-    for (int x = tid; x < n_loc * QG; x += kDecThreads) {
-      const float p = m_g > -INFINITY ? fast_exp2(lg[x] - m_g) : 0.f;
-      lg[x] = p;
-      lsum += p;
+    for (int g = 0; g < QG; ++g) {
+      m[g] = hd.red[0][g];
+#pragma unroll
+      for (int w = 1; w < kDecWarps; ++w) m[g] = fmaxf(m[g], hd.red[w][g]);
     }
-  }
-  // lanes holding the same head: lane bits >= log2(QG)
+    // ---- p = exp2(a - m) in place, split sums
+    float ls[QG];
 #pragma unroll
-  for (int o = QG; o < 32; o <<= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
-  __syncthreads();  // every thread has read hd.red (max) and written its p
-  if (lane < static_cast<uint32_t>(QG)) hd.red[warp][lane] = lsum;
+    for (int g = 0; g < QG; ++g) ls[g] = 0.f;
+#pragma unroll
+    for (int u = 0; u < kKeysPerThread; ++u) {
+      const int k = tid + u * kDecThreads;
+      if (k < x.n_loc) {
+#pragma unroll
+        for (int g4 = 0; g4 < QG; g4 += 4) {
+          float4 v = *reinterpret_cast<const float4*>(lg + k * QG + g4);
+          float w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float mg = m[g4 + e];
+            w[e] = mg > -INFINITY ? fast_exp2(w[e] - mg) : 0.f;
+            ls[g4 + e] += w[e];
+          }
+          *reinterpret_cast<float4*>(lg + k * QG + g4) = make_float4(w[0], w[1], w[2], w[3]);
+        }
+      }
+    }
+    block_reduce_qg<QG, false>(ls, hd.red2, warp, lane);
+    __syncthreads();  // p complete; hd.red2 holds the warps' sums
 
-  // ---- P V: one warp per key, lanes over d
-  float acc[QG][G::kVe];
+    // ---- P V: one warp per key, lanes over d
+    float acc[QG][G::kVe];
 #pragma unroll
-  for (int g = 0; g < QG; ++g)
+    for (int g = 0; g < QG; ++g)
 #pragma unroll
-    for (int e = 0; e < G::kVe; ++e) acc[g][e] = 0.f;
-  if (!aborted_k) {
-    for (; t < n_all; ++t) {
-      const bool ok = wait_bar(&hd.full[t % kDecStages], (t / kDecStages) & 1, abort_flag,
-                               kWaitLimitNs);
-      if (ok) {
-        const uint8_t* tile = ring + (t % kDecStages) * kDecTileBytes;
-        const int k0 = (t - n_tiles) * G::kTileKeys;
-        const int kend = min(G::kTileKeys, n_loc - k0);
+      for (int e = 0; e < G::kVe; ++e) acc[g][e] = 0.f;
+    for (int t = 0; t < x.n_tiles; ++t, ++g_t) {
+      if (wait_bar(&hd.full[g_t % kDecStages], (g_t / kDecStages) & 1, abort_flag,
+                   kWaitLimitNs)) {
+        const uint8_t* tile = ring + (g_t % kDecStages) * kDecTileBytes;
+        const int k0 = t * G::kTileKeys;
+        const int kend = min(G::kTileKeys, x.n_loc - k0);
 #pragma unroll 2
         for (int kk = warp; kk < kend; kk += kDecWarps) {
           float p[QG];
@@ -293,15 +375,16 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
           }
           float vf[G::kVe];
           if constexpr (D == 128) {
-            const uint2 u = *reinterpret_cast<const uint2*>(tile + kk * G::kRowBytes + lane * 8);
-            vf[0] = __uint_as_float(u.x << 16);
-            vf[1] = __uint_as_float(u.x & 0xFFFF0000u);
-            vf[2] = __uint_as_float(u.y << 16);
-            vf[3] = __uint_as_float(u.y & 0xFFFF0000u);
+            const uint2 uu = *reinterpret_cast<const uint2*>(tile + kk * G::kRowBytes + lane * 8);
+            vf[0] = __uint_as_float(uu.x << 16);
+            vf[1] = __uint_as_float(uu.x & 0xFFFF0000u);
+            vf[2] = __uint_as_float(uu.y << 16);
+            vf[3] = __uint_as_float(uu.y & 0xFFFF0000u);
           } else {
-            const uint32_t u = *reinterpret_cast<const uint32_t*>(tile + kk * G::kRowBytes + lane * 4);
-            vf[0] = __uint_as_float(u << 16);
-            vf[1] = __uint_as_float(u & 0xFFFF0000u);
+            const uint32_t uu =
+                *reinterpret_cast<const uint32_t*>(tile + kk * G::kRowBytes + lane * 4);
+            vf[0] = __uint_as_float(uu << 16);
+            vf[1] = __uint_as_float(uu & 0xFFFF0000u);
           }
 #pragma unroll
           for (int g = 0; g < QG; ++g)
@@ -311,8 +394,36 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
       }
       __syncthreads();
       if (*abort_flag) break;
-      if (tid == 0 && issued < n_all) issue(issued++);
+      if (tid == 0) issue_next();
     }
+    if (*abort_flag) break;
+
+    // ---- the item's partials: (max, sum, unnormalised output) per query head
+#pragma unroll
+    for (int g = 0; g < QG; ++g)
+#pragma unroll
+      for (int e = 0; e < G::kVe; ++e)
+        red_o[(warp * QG + g) * D + static_cast<int>(lane) * G::kVe + e] = acc[g][e];
+    __syncthreads();
+    for (int y = tid; y < a.qg * D; y += kDecThreads) {
+      const int g = y / D, dd = y % D;
+      float o = 0.f;
+#pragma unroll
+      for (int w = 0; w < kDecWarps; ++w) o += red_o[(w * QG + g) * D + dd];
+      a.part[((row0 + g) * a.n_split + x.s) * (2 + D) + 2 + dd] = o;
+    }
+    if (tid < a.qg) {
+      float l = 0.f, mt = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kDecWarps; ++w) {
+        l += hd.red2[w][tid];
+        mt = fmaxf(mt, hd.red[w][tid]);
+      }
+      float* pm = a.part + ((row0 + tid) * a.n_split + x.s) * (2 + D);
+      pm[0] = mt;
+      pm[1] = l;
+    }
+    __syncthreads();  // red_o, hd.red and hd.red2 are free for the next item
   }
 
   if (*abort_flag) {
@@ -320,37 +431,9 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
     if (tid == 0) {
       atomicOr(a.err, H2O_DEVERR_TIMEOUT);
       int never = 0;
-      for (int x = t; x < issued; ++x)
-        wait_bar(&hd.full[x % kDecStages], (x / kDecStages) & 1, &never, kWaitLimitNs / 16);
+      for (int y = g_t; y < issued; ++y)
+        wait_bar(&hd.full[y % kDecStages], (y / kDecStages) & 1, &never, kWaitLimitNs / 16);
     }
-    return;
-  }
-
-  // ---- combine the warps' partial outputs (the ring is free: every copy landed)
-  float* red_o = reinterpret_cast<float*>(ring);  // [warp][g][D]
-#pragma unroll
-  for (int g = 0; g < QG; ++g)
-#pragma unroll
-    for (int e = 0; e < G::kVe; ++e)
-      red_o[(warp * QG + g) * D + static_cast<int>(lane) * G::kVe + e] = acc[g][e];
-  __syncthreads();
-  const size_t row0 = static_cast<size_t>(b * a.Hq + h * a.qg);
-  for (int x = tid; x < a.qg * D; x += kDecThreads) {
-    const int g = x / D, dd = x % D;
-    float o = 0.f;
-#pragma unroll
-    for (int w = 0; w < kDecWarps; ++w) o += red_o[(w * QG + g) * D + dd];
-    a.part[((row0 + g) * a.n_split + s) * (2 + D) + 2 + dd] = o;
-  }
-  if (tid < a.qg) {
-    // thread tid < QG converted head gp = tid: m_g is that head's split max;
-    // hd.red now holds the warps' partial sums
-    float l = 0.f;
-#pragma unroll
-    for (int w = 0; w < kDecWarps; ++w) l += hd.red[w][tid];
-    float* pm = a.part + ((row0 + tid) * a.n_split + s) * (2 + D);
-    pm[0] = m_g;
-    pm[1] = l;
   }
 }
 
@@ -380,6 +463,7 @@ __device__ __forceinline__ float block_sum(float v, float* sh) {
 
 template <int D>
 __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const DecodeArgs a) {
+  extern __shared__ float fac[];  // [max(n_split, threads)]: exp2(m_s - m) per split
   __shared__ float sh[kCombineThreads / 32];
   const int tid = threadIdx.x;
   const size_t row = blockIdx.x;  // b * Hq + hq
@@ -390,24 +474,34 @@ __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const D
   float l = 0.f;
   for (int s = tid; s < a.n_split; s += kCombineThreads) {
     const float ms = part[s * (2 + D)];
-    if (ms > -INFINITY) l += part[s * (2 + D) + 1] * fast_exp2(ms - m);
+    const float f = ms > -INFINITY ? fast_exp2(ms - m) : 0.f;
+    fac[s] = f;
+    l += part[s * (2 + D) + 1] * f;
   }
-  l = block_sum(l, sh);
+  l = block_sum(l, sh);  // (its barriers also publish fac)
   // every row sees its own token, so m is finite and l >= 1
   const float lam = m + fast_log2(l);
   if (blockIdx.y == 0) {
     const float inv = 1.0f / l;
-    for (int dp = tid; dp < D / 2; dp += kCombineThreads) {
-      float o0 = 0.f, o1 = 0.f;
-      for (int s = 0; s < a.n_split; ++s) {
-        const float ms = part[s * (2 + D)];
-        if (ms > -INFINITY) {
-          const float f = fast_exp2(ms - m);
-          o0 = fmaf(f, part[s * (2 + D) + 2 + 2 * dp], o0);
-          o1 = fmaf(f, part[s * (2 + D) + 3 + 2 * dp], o1);
-        }
-      }
-      reinterpret_cast<uint32_t*>(a.out + row * D)[dp] = pack_bf16x2(o0 * inv, o1 * inv);
+    // thread (dd, q): output element dd, splits q, q + 2, ... (two halves)
+    constexpr int kHalves = kCombineThreads / D;
+    const int dd = tid % D, q = tid / D;
+    float o0 = 0.f, o1 = 0.f;
+    int s = q;
+    for (; s + kHalves < a.n_split; s += 2 * kHalves) {
+      o0 = fmaf(fac[s], part[s * (2 + D) + 2 + dd], o0);
+      o1 = fmaf(fac[s + kHalves], part[(s + kHalves) * (2 + D) + 2 + dd], o1);
+    }
+    if (s < a.n_split) o0 = fmaf(fac[s], part[s * (2 + D) + 2 + dd], o0);
+    const float o = o0 + o1;
+    __syncthreads();  // every thread is done with fac
+    fac[tid] = o;     // (fac holds at least kCombineThreads floats)
+    __syncthreads();
+    if (q == 0) {
+      float t = fac[dd];
+#pragma unroll
+      for (int x = 1; x < kHalves; ++x) t += fac[x * D + dd];
+      a.out[row * D + dd] = static_cast<uint16_t>(pack_bf16x2(t * inv, 0.f) & 0xFFFFu);
     }
   }
   float* inc = a.score_inc + row * (static_cast<size_t>(a.M) + 1);
@@ -417,29 +511,40 @@ __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const D
   for (int j = c0 + tid; j < c1; j += kCombineThreads) inc[j] = fast_exp2(inc[j] - lam);
 }
 
-template <int QG>
+template <int D, int QG>
 constexpr size_t split_smem(int split_len) {
   return kDecStages * kDecTileBytes + sizeof(DecHead) +
-         static_cast<size_t>(split_len + 1) * QG * sizeof(float);
+         static_cast<size_t>(split_len + 1) * QG * sizeof(float) +
+         static_cast<size_t>(kDecWarps) * QG * D * sizeof(float) +
+         static_cast<size_t>(kDecStages) * QG * D * sizeof(uint16_t);
 }
 
 template <int D, int QG>
 cudaError_t launch_split(const DecodeArgs& a, cudaStream_t stream) {
-  // the attribute is set once per device, for the largest split
-  static bool configured[64] = {};
+  // Persistent grid: as many CTAs as fit on the GPU at once (sized once per
+  // device for the largest split), each taking every gridDim-th work item.
+  static int resident[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev >= 64 || !configured[dev]) {
+  int n_res = dev < 64 ? resident[dev] : 0;
+  if (n_res == 0) {
+    const int smem_max = static_cast<int>(split_smem<D, QG>(kDecodeMaxSplitLen));
     e = cudaFuncSetAttribute(decode_split_kernel<D, QG>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(split_smem<QG>(kDecodeMaxSplitLen)));
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
     if (e != cudaSuccess) return e;
-    if (dev < 64) configured[dev] = true;
+    int per_sm = 0, sms = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_split_kernel<D, QG>,
+                                                      kDecThreads, smem_max);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    n_res = std::max(1, per_sm) * sms;
+    if (dev < 64) resident[dev] = n_res;
   }
-  const size_t smem = split_smem<QG>(a.split_len);
-  const dim3 grid(static_cast<unsigned>(a.n_split), static_cast<unsigned>(a.B * a.Hkv));
-  decode_split_kernel<D, QG><<<grid, kDecThreads, smem, stream>>>(a);
+  const int n_items = a.n_split * a.B * a.Hkv;
+  const size_t smem = split_smem<D, QG>(a.split_len);
+  decode_split_kernel<D, QG><<<std::min(n_items, n_res), kDecThreads, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
@@ -449,7 +554,8 @@ cudaError_t launch_d(const DecodeArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const dim3 grid(static_cast<unsigned>(a.B * a.Hq),
                   static_cast<unsigned>((a.M + 1 + kCombineCols - 1) / kCombineCols));
-  decode_combine_kernel<D><<<grid, kCombineThreads, 0, stream>>>(a);
+  const size_t smem = static_cast<size_t>(std::max(a.n_split, kCombineThreads)) * sizeof(float);
+  decode_combine_kernel<D><<<grid, kCombineThreads, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
@@ -458,12 +564,24 @@ cudaError_t launch_d(const DecodeArgs& a, cudaStream_t stream) {
 bool decode_plan(int B, int Hq, int Hkv, int d, int S, int M, int* split_len, int* n_split,
                  size_t* ws_bytes) {
   if (S != 1 || M < 1 || Hq / Hkv > kDecodeMaxQg) return false;
+  // Work items are (b, kv head, split); the persistent split kernel deals them
+  // round-robin to kDecodeResidentCtas CTAs, so a step costs about
+  // ceil(items / CTAs) items of (split_len + per-item overhead) keys.  Take
+  // the split length (a multiple of 16 in [128, 1536]) that minimises that.
   const int64_t groups = static_cast<int64_t>(B) * Hkv;
-  int64_t len = (static_cast<int64_t>(M) * groups + kDecodeTargetCtas - 1) / kDecodeTargetCtas;
-  len = (len + 63) / 64 * 64;
-  len = std::min<int64_t>(std::max<int64_t>(len, kDecodeMinSplitLen), kDecodeMaxSplitLen);
-  const int64_t n = (M + len - 1) / len;
-  *split_len = static_cast<int>(len);
+  int64_t best_len = kDecodeMaxSplitLen, best_cost = INT64_MAX;
+  for (int64_t len = kDecodeMinSplitLen; len <= kDecodeMaxSplitLen; len += 16) {
+    const int64_t n = (M + len - 1) / len;
+    const int64_t rounds = (groups * n + kDecodeResidentCtas - 1) / kDecodeResidentCtas;
+    const int64_t cost = rounds * (std::min<int64_t>(len, M) + kDecodeItemOverheadKeys);
+    if (cost < best_cost) {
+      best_cost = cost;
+      best_len = len;
+    }
+    if (len >= M) break;
+  }
+  const int64_t n = (M + best_len - 1) / best_len;
+  *split_len = static_cast<int>(best_len);
   *n_split = static_cast<int>(n);
   *ws_bytes = static_cast<size_t>(B) * Hq * n * (2 + d) * sizeof(float);
   return true;

@@ -54,9 +54,10 @@ struct UpdateArgs {
 
 // S = 1 (one query token per sequence): split-K decode kernels.
 constexpr int kDecodeMaxQg = 8;         // larger GQA groups take the chunk kernel
-constexpr int kDecodeMaxSplitLen = 2048;
-constexpr int kDecodeMinSplitLen = 256;
-constexpr int kDecodeTargetCtas = 608;  // 4 x 152 SMs
+constexpr int kDecodeMaxSplitLen = 1536;
+constexpr int kDecodeMinSplitLen = 128;
+constexpr int kDecodeResidentCtas = 304;     // split-kernel CTAs resident on a GB300 (2 x 152)
+constexpr int kDecodeItemOverheadKeys = 32;  // per-item cost, in keys, for choosing the split
 
 struct DecodeArgs {
   const uint16_t* q;        // (B, Hq, 1, d)
@@ -72,7 +73,7 @@ struct DecodeArgs {
   int B, Hq, Hkv, d, M, qg;
   int pos0;
   float scale_log2;
-  int split_len;            // cache slots per split (multiple of 64)
+  int split_len;            // cache slots per split (multiple of 16)
   int n_split;              // ceil(M / split_len); the last split also takes the new token
 };
 

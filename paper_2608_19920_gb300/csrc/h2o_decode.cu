@@ -241,7 +241,7 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
       pos[u] = k < x.n_cache ? __ldg(sp + k) : 0;
     }
     // ---- Q K^T: raw dot products of the item's keys into lg
-    float qr[QG][8 * G::kCh];  // this lane's slice of every head's query
+    float2 qr[QG][4 * G::kCh];  // this lane's slice of every head's query, element pairs
     for (int t = 0; t < x.n_tiles; ++t, ++g_t) {
       if (wait_bar(&hd.full[g_t % kDecStages], (g_t / kDecStages) & 1, abort_flag,
                    kWaitLimitNs)) {
@@ -250,14 +250,17 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
           const uint16_t* qs = qbuf + (g_t % kDecStages) * QG * D;
 #pragma unroll
           for (int g = 0; g < QG; ++g) {
-            if (g < a.qg) {
 #pragma unroll
-              for (int ch = 0; ch < G::kCh; ++ch)
-                bf16x8_to_f32(reinterpret_cast<const uint4*>(qs + g * D)[c0 + 8 * ch],
-                              &qr[g][8 * ch]);
-            } else {
+            for (int ch = 0; ch < G::kCh; ++ch) {
+              float f[8];
+              if (g < a.qg) {
+                bf16x8_to_f32(reinterpret_cast<const uint4*>(qs + g * D)[c0 + 8 * ch], f);
+              } else {
 #pragma unroll
-              for (int e = 0; e < 8 * G::kCh; ++e) qr[g][e] = 0.f;
+                for (int e = 0; e < 8; ++e) f[e] = 0.f;
+              }
+#pragma unroll
+              for (int e = 0; e < 4; ++e) qr[g][4 * ch + e] = make_float2(f[2 * e], f[2 * e + 1]);
             }
           }
         }
@@ -265,21 +268,29 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
         for (int r = 0; r < G::kTileKeys / 32; ++r) {
           const int kk = r * 32 + warp * 4 + static_cast<int>(lane >> 3);  // key within the tile
           const int kl = t * G::kTileKeys + kk;                             // key within the item
-          float dot[QG];
+          // packed fp32 FMAs over element pairs (even, odd), the two halves
+          // added at the end
+          float2 d2[QG];
 #pragma unroll
-          for (int g = 0; g < QG; ++g) dot[g] = 0.f;
+          for (int g = 0; g < QG; ++g) d2[g] = make_float2(0.f, 0.f);
           if (kl < x.n_loc) {
             const uint4* krow = reinterpret_cast<const uint4*>(tile + kk * G::kRowBytes);
 #pragma unroll
             for (int ch = 0; ch < G::kCh; ++ch) {
-              float kf[8];
-              bf16x8_to_f32(krow[c0 + 8 * ch], kf);
+              const uint4 u = krow[c0 + 8 * ch];
+              const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-              for (int e = 0; e < 8; ++e)
+              for (int e = 0; e < 4; ++e) {
+                const float2 kf = make_float2(__uint_as_float(w[e] << 16),
+                                              __uint_as_float(w[e] & 0xFFFF0000u));
 #pragma unroll
-                for (int g = 0; g < QG; ++g) dot[g] = fmaf(qr[g][8 * ch + e], kf[e], dot[g]);
+                for (int g = 0; g < QG; ++g) d2[g] = __ffma2_rn(qr[g][4 * ch + e], kf, d2[g]);
+              }
             }
           }
+          float dot[QG];
+#pragma unroll
+          for (int g = 0; g < QG; ++g) dot[g] = d2[g].x + d2[g].y;
           const float tot = reduce_scatter8<QG>(dot, lane);
           if (dot_writer && kl < x.n_loc) lg[kl * QG + hg] = tot;
         }
@@ -351,11 +362,11 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
     __syncthreads();  // p complete; hd.red2 holds the warps' sums
 
     // ---- P V: one warp per key, lanes over d
-    float acc[QG][G::kVe];
+    float2 acc[QG][G::kVe / 2];  // (d element 2e, 2e + 1) of this lane, per head
 #pragma unroll
     for (int g = 0; g < QG; ++g)
 #pragma unroll
-      for (int e = 0; e < G::kVe; ++e) acc[g][e] = 0.f;
+      for (int e = 0; e < G::kVe / 2; ++e) acc[g][e] = make_float2(0.f, 0.f);
     for (int t = 0; t < x.n_tiles; ++t, ++g_t) {
       if (wait_bar(&hd.full[g_t % kDecStages], (g_t / kDecStages) & 1, abort_flag,
                    kWaitLimitNs)) {
@@ -373,23 +384,21 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
             p[g4 + 2] = pv.z;
             p[g4 + 3] = pv.w;
           }
-          float vf[G::kVe];
+          float2 vf[G::kVe / 2];
           if constexpr (D == 128) {
             const uint2 uu = *reinterpret_cast<const uint2*>(tile + kk * G::kRowBytes + lane * 8);
-            vf[0] = __uint_as_float(uu.x << 16);
-            vf[1] = __uint_as_float(uu.x & 0xFFFF0000u);
-            vf[2] = __uint_as_float(uu.y << 16);
-            vf[3] = __uint_as_float(uu.y & 0xFFFF0000u);
+            vf[0] = make_float2(__uint_as_float(uu.x << 16), __uint_as_float(uu.x & 0xFFFF0000u));
+            vf[1] = make_float2(__uint_as_float(uu.y << 16), __uint_as_float(uu.y & 0xFFFF0000u));
           } else {
             const uint32_t uu =
                 *reinterpret_cast<const uint32_t*>(tile + kk * G::kRowBytes + lane * 4);
-            vf[0] = __uint_as_float(uu << 16);
-            vf[1] = __uint_as_float(uu & 0xFFFF0000u);
+            vf[0] = make_float2(__uint_as_float(uu << 16), __uint_as_float(uu & 0xFFFF0000u));
           }
 #pragma unroll
           for (int g = 0; g < QG; ++g)
 #pragma unroll
-            for (int e = 0; e < G::kVe; ++e) acc[g][e] = fmaf(p[g], vf[e], acc[g][e]);
+            for (int e = 0; e < G::kVe / 2; ++e)
+              acc[g][e] = __ffma2_rn(make_float2(p[g], p[g]), vf[e], acc[g][e]);
         }
       }
       __syncthreads();
@@ -402,8 +411,9 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
 #pragma unroll
     for (int g = 0; g < QG; ++g)
 #pragma unroll
-      for (int e = 0; e < G::kVe; ++e)
-        red_o[(warp * QG + g) * D + static_cast<int>(lane) * G::kVe + e] = acc[g][e];
+      for (int e = 0; e < G::kVe / 2; ++e)
+        *reinterpret_cast<float2*>(red_o + (warp * QG + g) * D + static_cast<int>(lane) * G::kVe +
+                                   2 * e) = acc[g][e];
     __syncthreads();
     for (int y = tid; y < a.qg * D; y += kDecThreads) {
       const int g = y / D, dd = y % D;

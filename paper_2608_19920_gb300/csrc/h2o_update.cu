@@ -511,13 +511,19 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
 // coalesced) and keeps the smallest (key << 32 | j).  Every CTA sends its
 // minimum to every CTA of the cluster; after a cluster barrier all know the
 // evicted slot.  Pass 2 (nothing is written before it, so a (b, h) without a
-// candidate stays unchanged): each CTA recomputes and writes acc_j of its
-// range, and the CTA holding the evicted slot writes the new token's score,
-// position, evict_idx and K/V rows there.
+// candidate stays unchanged): each CTA writes acc_j of its range (kept in
+// shared memory by pass 1 when the range fits, recomputed otherwise), and
+// the CTA holding the evicted slot writes the new token's score, position,
+// evict_idx and K/V rows there.
 constexpr int kDThreads = 512;
 constexpr int kDBatch = 6;  // slots per thread per batch of loads
 
-__global__ void __launch_bounds__(kDThreads, 2) update_decode_kernel(const UpdateArgs a, int C) {
+// acc_j of pass 1 kept for pass 2 when a CTA's range (x batch entries) fits
+constexpr size_t kDStashBytes = 96 * 1024;
+
+__global__ void __launch_bounds__(kDThreads, 2)
+    update_decode_kernel(const UpdateArgs a, int C, int stash_ok) {
+  extern __shared__ float stash[];  // [nb][per] when stash_ok
   __shared__ unsigned long long wmin[kDThreads / 32];
   __shared__ unsigned long long cmin[8];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -573,7 +579,11 @@ __global__ void __launch_bounds__(kDThreads, 2) update_decode_kernel(const Updat
       float acc[kDBatch];
       batch_acc(b0 + bi, base, acc);
 #pragma unroll
-      for (int u = 0; u < kDBatch; ++u) kacc[u] = bi == 0 ? acc[u] : __fadd_rn(kacc[u], acc[u]);
+      for (int u = 0; u < kDBatch; ++u) {
+        kacc[u] = bi == 0 ? acc[u] : __fadd_rn(kacc[u], acc[u]);
+        const int j = base + u * kDThreads;
+        if (stash_ok && j < jhi) stash[bi * per + (j - jlo)] = acc[u];
+      }
     }
 #pragma unroll
     for (int u = 0; u < kDBatch; ++u) {
@@ -619,7 +629,15 @@ __global__ void __launch_bounds__(kDThreads, 2) update_decode_kernel(const Updat
   for (int base = jlo + tid; base < jhi; base += kDThreads * kDBatch) {
     for (int bi = 0; bi < nb; ++bi) {
       float acc[kDBatch];
-      batch_acc(b0 + bi, base, acc);
+      if (stash_ok) {
+#pragma unroll
+        for (int u = 0; u < kDBatch; ++u) {
+          const int j = base + u * kDThreads;
+          acc[u] = j < jhi ? stash[bi * per + (j - jlo)] : 0.f;
+        }
+      } else {
+        batch_acc(b0 + bi, base, acc);
+      }
       float* sc = a.scores + (static_cast<size_t>(b0 + bi) * a.Hkv + h) * M;
 #pragma unroll
       for (int u = 0; u < kDBatch; ++u) {
@@ -651,10 +669,23 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
     int C = a.M / 8192;
     C = C < 1 ? 1 : (C > 8 ? 8 : C);
     const int groups = a.policy == H2O_POLICY_ORIG ? a.Hkv : a.B * a.Hkv;
+    const size_t per = (static_cast<size_t>(a.M) + C - 1) / C;
+    const size_t stash = per * (a.policy == H2O_POLICY_ORIG ? a.B : 1) * sizeof(float);
+    const int stash_ok = stash <= kDStashBytes ? 1 : 0;
+    static bool dconf[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev >= 64 || !dconf[dev]) {
+      e = cudaFuncSetAttribute(update_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(kDStashBytes));
+      if (e != cudaSuccess) return e;
+      if (dev < 64) dconf[dev] = true;
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(groups * C));
     cfg.blockDim = dim3(kDThreads);
-    cfg.dynamicSmemBytes = 0;
+    cfg.dynamicSmemBytes = stash_ok ? stash : 0;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -663,7 +694,7 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, update_decode_kernel, a, C);
+    return cudaLaunchKernelEx(&cfg, update_decode_kernel, a, C, stash_ok);
   }
   if (!smem_path) {
     const int groups = a.policy == H2O_POLICY_ORIG ? a.Hkv : a.B * a.Hkv;

@@ -5,7 +5,8 @@ workload: empty the cache, prefill M tokens, then every chunk of S tokens
 (h2o_sdpa_chunk + h2o_update).  Default workload: one Llama-3-8B-shaped layer
 (B=1, Hq=32, Hkv=8, d=128), T=32768 tokens, chunks of 512, cache of 4096 slots,
 recent window 512.  Inputs are seeded synthetic bf16 tensors resident in HBM
-(402 MB per step, more than the 129 MB L2, so each step streams them).
+(402 MB per step, more than the 129 MB L2, so each step streams them).  The
+timed steps replay one CUDA graph of the whole step (``--no-graph``: eager).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload NAME] [--no-e2e] [--no-cpu-baseline]
@@ -316,9 +317,24 @@ def run_ours(args, w):
     torch.cuda.synchronize()
     if h2o_device_errors() != 0:
         raise SystemExit("device-side error during warm-up")
+    # chunk-step durations (sdpa + update), eager launches, one step
+    one_step(record=True)
+    torch.cuda.synchronize()
+    chunk_step_ms = [a.elapsed_time(b) for a, b in ev]
+    # The whole step (cache reset, prefill, every chunk's two calls) is
+    # captured once as a CUDA graph and replayed: every kernel of the step
+    # runs on every replay, without the host's launch gaps between them.
+    graph = None
+    if args.graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            one_step()
+        graph.replay()
+        torch.cuda.synchronize()
+        if h2o_device_errors() != 0:
+            raise SystemExit("device-side error in the captured step")
 
     # ---- timed region: K steps, inputs resident in HBM
-    sdpa_ms = []
     barrier(world)
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
@@ -327,7 +343,10 @@ def run_ours(args, w):
         clk.mark_start()
         t0.record(stream)
         for s in range(args.steps):
-            one_step(record=(s == args.steps - 1))
+            if graph is not None:
+                graph.replay()
+            else:
+                one_step()
         t1.record(stream)
         torch.cuda.synchronize()
         clk.mark_end()
@@ -335,8 +354,6 @@ def run_ours(args, w):
     barrier(world)
     elapsed_ms = max_over_ranks(elapsed_ms, world)
     step_ms = elapsed_ms / args.steps
-    # chunk-step durations (sdpa + update) of the last timed step
-    chunk_step_ms = [a.elapsed_time(b) for a, b in ev]
     clocks = clk.summary()
     if h2o_device_errors() != 0:
         raise SystemExit("device-side error during the timed region")
@@ -345,6 +362,7 @@ def run_ours(args, w):
     kern = time_sdpa_kernel(w, layer, inputs, plan, stream, reps=max(3, args.steps))
 
     value = tokens_per_step * world / (step_ms / 1e3)
+    in_bytes = sum(x.numel() * x.element_size() for c in inputs for x in c)
     pk = peaks()
     alg_tflops = total_flops / (step_ms / 1e3) / 1e12
     line = {
@@ -354,7 +372,10 @@ def run_ours(args, w):
         "data": "synthetic (seeded Gaussian Q/K/V with planted heavy-hitter keys)",
         "config": {"workload": w.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d, "T": w.T,
                    "S": w.S, "M": w.M, "W": w.W, "tokens_per_step": tokens_per_step,
-                   "chunks_per_step": n_chunks, "l2": "inputs larger than L2 (402 MB per step)",
+                   "chunks_per_step": n_chunks,
+                   "l2": f"inputs larger than L2 ({in_bytes / 1e6:.0f} MB per step)"
+                         if in_bytes > 129e6 else f"{in_bytes / 1e6:.0f} MB of inputs per step",
+                   "launch": "CUDA graph of the whole step" if args.graph else "eager",
                    "parallelism": f"replicas x{world}"},
         "tflops": alg_tflops,
         "tflops_frac_of_peak": alg_tflops / pk["bf16_sus"],
@@ -406,6 +427,16 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
     inc, _, ws = layer._buf(e - p)
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
     clean = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
+
+    def call():
+        h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out=out,
+                       score_inc=inc, workspace=ws)
+
+    # the call is replayed from a CUDA graph, as in the timed steps
+    call()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        call()
     times = []
     for _ in range(reps + 2):
         # Evict the previous launch's data from L2 by writing a buffer twice
@@ -416,8 +447,7 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out=out,
-                       score_inc=inc, workspace=ws)
+        graph.replay()
         b.record(stream)
         torch.cuda.synchronize()
         times.append(a.elapsed_time(b))
@@ -500,6 +530,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama8b_32k", choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
+    ap.add_argument("--no-graph", dest="graph", action="store_false",
+                    help="launch the timed steps eagerly instead of replaying a CUDA graph")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--traffic", type=float, default=None,
                     help="DRAM bytes per launch of the dominant kernel from an ncu capture")

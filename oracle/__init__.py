@@ -1,6 +1,7 @@
 """Float64 CPU oracle (test infrastructure only; never on the product path)."""
-from .h2o_oracle import (POLICIES, SequenceState, chunk_bounds, lse_merge, run_sequence,
-                         sdpa_chunk, update)
+from .h2o_oracle import (POLICIES, SequenceState, chunk_bounds, evict_insert, lse_merge,
+                         run_sequence, scores_add, sdpa_cache, sdpa_chunk, step_paper_order,
+                         update)
 
 __all__ = ["sdpa_chunk", "update", "run_sequence", "SequenceState", "lse_merge", "chunk_bounds",
-           "POLICIES"]
+           "POLICIES", "sdpa_cache", "evict_insert", "scores_add", "step_paper_order"]

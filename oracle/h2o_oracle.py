@@ -42,6 +42,17 @@ Readings where the paper is silent (each is also listed in the design notes):
   ascending order (t = inc_0; t = t + inc_g) and then ``scores + t``; that is
   the order any implementation must follow to be compared bit for bit.
 
+The paper's own order of a chunk step (§3.1 last paragraph, §3.3.1: the new
+keys and values are written into the cache first, then SDPA runs over the
+N_C = M slots under the position mask) is the second path here:
+``evict_insert`` (the S slots with the smallest score phi^P, before this
+chunk's attention, take the chunk's tokens; their scores restart at 0),
+``sdpa_cache`` (N_k = M) and ``scores_add`` (Eq. 3 with this chunk's weights),
+chained by ``step_paper_order`` and ``run_sequence(order="paper")``.  Its
+readings: the same candidate rule (positions >= P + S - W protected, empty
+first, score, slot) and token-to-slot assignment as ``update``; h2o_norm
+divides by t - t(j) with t = P, the tokens processed when the choice is made.
+
 Parity: every function here is pinned by the not-gpu tests against dense
 causal attention, closed forms, the summed-weights identity of §A.6.2,
 invariants of §3.1-§3.3 and brute-force enumeration.
@@ -53,7 +64,8 @@ import math
 import numpy as np
 
 __all__ = ["sdpa_chunk", "update", "run_sequence", "SequenceState", "lse_merge",
-           "chunk_bounds", "POLICIES"]
+           "chunk_bounds", "POLICIES", "sdpa_cache", "evict_insert", "scores_add",
+           "step_paper_order"]
 
 
 def _token_positions(slot_pos_bh: np.ndarray, pos0: int, S: int) -> np.ndarray:
@@ -195,6 +207,136 @@ def update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0: in
                 evict_idx=evict)
 
 
+def sdpa_cache(q, k_cache, v_cache, slot_pos, pos0: int, scale: float | None = None, rows=None):
+    """SDPA over the M cache slots only, the chunk's own keys already written
+    there (the paper's order: §3.1 Eq. 2 with N_k = N_C, mask of §3.3.1).
+
+    Query row i (token pos0 + i) sees slot j iff 0 <= slot_pos[j] <= pos0 + i.
+    Returns (out (B,H_q,S,d), score_inc (B,H_q,M), lse (B,H_q,S)), float64;
+    ``rows`` as in ``sdpa_chunk``.
+    """
+    q = np.asarray(q, np.float64)
+    B, Hq, S, d = q.shape
+    ridx = np.arange(S) if rows is None else np.asarray(rows, np.int64)
+    Hkv, M = slot_pos.shape[1], slot_pos.shape[2]
+    assert Hq % Hkv == 0
+    qg = Hq // Hkv
+    if scale is None:
+        scale = 1.0 / math.sqrt(d)
+    out = np.zeros((B, Hq, len(ridx), d))
+    score_inc = np.zeros((B, Hq, M))
+    lse = np.zeros((B, Hq, len(ridx)))
+    for b in range(B):
+        for hq in range(Hq):
+            h = hq // qg
+            keys = np.asarray(k_cache[b, h], np.float64)
+            vals = np.asarray(v_cache[b, h], np.float64)
+            t = slot_pos[b, h].astype(np.int64)
+            qpos = pos0 + ridx[:, None]
+            visible = (t[None, :] >= 0) & (t[None, :] <= qpos)
+            a = scale * (q[b, hq][ridx] @ keys.T)
+            a = np.where(visible, a, -np.inf)
+            amax = a.max(axis=1, keepdims=True)
+            lam = amax + np.log(np.exp(a - amax).sum(axis=1, keepdims=True))
+            m = np.where(visible, np.exp(a - lam), 0.0)
+            out[b, hq] = m @ vals
+            score_inc[b, hq] = m.sum(axis=0)
+            lse[b, hq] = lam[:, 0]
+    return out, score_inc, lse
+
+
+def evict_insert(scores, slot_pos, k_new, v_new, k_cache, v_cache, pos0: int,
+                 recent_window: int, precision: str = "fp32", policy: str = "h2o"):
+    """First part of the paper-order chunk step (§3.1, §3.1.1, scatter of §3.2):
+    per (b, kv head) the S slots with the smallest score phi^P (this chunk has
+    not attended yet) receive the chunk's keys and values; the c-th smallest
+    evicted slot gets token pos0 + c and a score of 0.  Candidates, total
+    order and policies as in ``update``, with t = pos0 for h2o_norm.
+
+    Inputs are not modified.  Returns a dict like ``update``'s.
+    """
+    if policy not in POLICIES:
+        raise ValueError(f"unknown policy {policy!r}")
+    B, Hkv, M = slot_pos.shape
+    S = k_new.shape[2]
+    assert 1 <= S <= M
+    W = recent_window
+    if W < 0 or W > M:
+        raise ValueError("recent_window must lie in [0, M]")
+    ft = np.float32 if precision == "fp32" else np.float64
+    out_scores = np.array(scores, dtype=ft, copy=True)
+    out_pos = np.array(slot_pos, dtype=np.int32, copy=True)
+    out_k = np.array(k_cache, copy=True)
+    out_v = np.array(v_cache, copy=True)
+    evict = np.zeros((B, Hkv, S), np.int32)
+
+    def choose(rank_score, pos):
+        cand = np.nonzero(pos < pos0 + S - W)[0]
+        if cand.size < S:
+            raise ValueError("fewer eviction candidates than chunk tokens")
+        occupied = pos[cand] >= 0
+        rank0 = occupied.astype(np.int64)
+        rank1 = np.where(occupied, rank_score[cand], 0)
+        order = np.lexsort((cand, rank1, rank0))
+        return np.sort(cand[order[:S]])
+
+    for h in range(Hkv):
+        if policy == "h2o_orig":
+            tot = out_scores[0, h].copy()
+            for b in range(1, B):
+                tot = tot + out_scores[b, h]
+            shared = choose(tot, out_pos[0, h])
+        for b in range(B):
+            pos = out_pos[b, h]
+            if policy == "h2o":
+                chosen = choose(out_scores[b, h], pos)
+            elif policy == "h2o_norm":
+                age = np.maximum(pos0 - pos.astype(np.int64), 1).astype(ft)
+                chosen = choose(out_scores[b, h] / age, pos)
+            else:
+                chosen = shared
+            evict[b, h] = chosen
+            for c, e in enumerate(chosen):
+                out_k[b, h, e] = k_new[b, h, c]
+                out_v[b, h, e] = v_new[b, h, c]
+                out_pos[b, h, e] = pos0 + c
+                out_scores[b, h, e] = 0
+    return dict(scores=out_scores, slot_pos=out_pos, k_cache=out_k, v_cache=out_v,
+                evict_idx=evict)
+
+
+def scores_add(scores, score_inc, precision: str = "fp32"):
+    """Last part of the paper-order chunk step: Eq. 3 adds this chunk's summed
+    weights, summed over the GQA group (ascending g), to every slot's score.
+
+    scores (B, H_kv, M), score_inc (B, H_q, M).  Returns the new scores.
+    """
+    ft = np.float32 if precision == "fp32" else np.float64
+    B, Hkv, M = scores.shape
+    inc = np.asarray(score_inc, ft)
+    qg = inc.shape[1] // Hkv
+    out = np.array(scores, dtype=ft, copy=True)
+    for b in range(B):
+        for h in range(Hkv):
+            t = inc[b, h * qg].copy()
+            for g in range(1, qg):
+                t = t + inc[b, h * qg + g]
+            out[b, h] = out[b, h] + t
+    return out
+
+
+def step_paper_order(scores, slot_pos, k_cache, v_cache, q, k_new, v_new, pos0: int,
+                     recent_window: int, precision: str = "fp32", policy: str = "h2o",
+                     scale: float | None = None):
+    """One chunk in the paper's order: evict_insert, sdpa_cache, scores_add.
+    Returns (out, score_inc (B,H_q,M), state dict after the step)."""
+    st = evict_insert(scores, slot_pos, k_new, v_new, k_cache, v_cache, pos0, recent_window,
+                      precision, policy)
+    out, inc, _ = sdpa_cache(q, st["k_cache"], st["v_cache"], st["slot_pos"], pos0, scale)
+    st["scores"] = scores_add(st["scores"], inc, precision)
+    return out, inc, st
+
+
 class SequenceState:
     """Cache state of one attention layer: buffers of fixed length M (§3.1)."""
 
@@ -218,22 +360,31 @@ def chunk_bounds(T: int, M: int, S: int, prefill: int | None = None):
 
 def run_sequence(q, k, v, M: int, S: int, W: int, prefill: int | None = None,
                  scale: float | None = None, precision: str = "fp64", on_step=None,
-                 policy: str = "h2o"):
+                 policy: str = "h2o", order: str = "chunk"):
     """Sparse-attention pass over whole sequences: prefill, then chunks of S.
 
     q (B,H_q,T,d), k/v (B,H_kv,T,d).  Returns (out (B,H_q,T,d), final state).
+    ``order``: "chunk" (attend to the cache plus the chunk, then update) or
+    "paper" (evict and write first, then attend to the cache, then add scores).
     ``on_step(i, bounds, state_before, result)`` is called after every chunk.
     """
+    if order not in ("chunk", "paper"):
+        raise ValueError(f"unknown order {order!r}")
     B, Hq, T, d = q.shape
     Hkv = k.shape[1]
     st = SequenceState(B, Hkv, M, d, score_dtype=np.float64 if precision == "fp64" else np.float32)
     out = np.zeros((B, Hq, T, d))
     for i, (p, e) in enumerate(chunk_bounds(T, M, S, prefill)):
-        o, inc, _ = sdpa_chunk(q[:, :, p:e], st.k_cache, st.v_cache, k[:, :, p:e], v[:, :, p:e],
-                               st.slot_pos, p, scale)
+        if order == "paper":
+            o, inc, res = step_paper_order(st.scores, st.slot_pos, st.k_cache, st.v_cache,
+                                           q[:, :, p:e], k[:, :, p:e], v[:, :, p:e], p, W,
+                                           precision, policy, scale)
+        else:
+            o, inc, _ = sdpa_chunk(q[:, :, p:e], st.k_cache, st.v_cache, k[:, :, p:e],
+                                   v[:, :, p:e], st.slot_pos, p, scale)
+            res = update(st.scores, st.slot_pos, inc, k[:, :, p:e], v[:, :, p:e],
+                         st.k_cache, st.v_cache, p, W, precision, policy)
         out[:, :, p:e] = o
-        res = update(st.scores, st.slot_pos, inc, k[:, :, p:e], v[:, :, p:e],
-                     st.k_cache, st.v_cache, p, W, precision, policy)
         before = (st.scores, st.slot_pos, st.k_cache, st.v_cache)
         st.scores, st.slot_pos = res["scores"], res["slot_pos"]
         st.k_cache, st.v_cache = res["k_cache"], res["v_cache"]

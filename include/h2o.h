@@ -195,6 +195,42 @@ H2O_API int h2o_update_policy(const h2o_dims_t* dims, int64_t pos0, float* score
                               int32_t budget, int32_t recent_window, int32_t policy,
                               int32_t* evict_idx, void* stream);
 
+/*
+ * The paper's own order of a chunk step (§3.1 last paragraph, §3.3.1): the
+ * chunk's keys and values are written into the cache first, then SDPA runs
+ * over the M = N_C slots with the mask "row i sees slot j iff
+ * 0 <= slot_pos[j] <= pos0 + i", then the chunk's summed weights are added to
+ * the scores.  Three calls per chunk, in this order:
+ *
+ *   h2o_evict_insert  per (b, kv head), the S slots with the smallest score
+ *                     (before this chunk attends) under the rules of
+ *                     h2o_update_policy (candidates, total order, policies;
+ *                     h2o_norm's age is pos0 - slot_pos) take the chunk's
+ *                     K/V; the c-th smallest gets token pos0 + c, score 0.
+ *                     Every other slot is left as it is.  Arguments and
+ *                     errors as h2o_update_policy, without score_inc.
+ *   h2o_sdpa_cache    SDPA of the chunk's queries over the M slots only:
+ *                     out (B, Hq, S, d) bf16 and score_inc (B, Hq, M) f32;
+ *                     k_cache / v_cache / slot_pos as left by
+ *                     h2o_evict_insert (every query row then sees at least
+ *                     its own token).  M >= 1.  Workspace as for
+ *                     h2o_sdpa_chunk with the same dims
+ *                     (h2o_workspace_size).  Errors as h2o_sdpa_chunk.
+ *   h2o_scores_add    scores[b,h,j] += score_inc[b,h*qg+0,j] + ... +
+ *                     score_inc[b,h*qg+qg-1,j] (float32, ascending g, then
+ *                     added to the score) for every slot j < M.
+ */
+H2O_API int h2o_evict_insert(const h2o_dims_t* dims, int64_t pos0, float* scores,
+                   int32_t* slot_pos, const h2o_bf16* k_new, const h2o_bf16* v_new,
+                   h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget,
+                   int32_t recent_window, int32_t policy, int32_t* evict_idx, void* stream);
+H2O_API int h2o_sdpa_cache(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                   const int32_t* slot_pos, h2o_bf16* out, float* score_inc, void* workspace,
+                   size_t workspace_bytes, void* stream);
+H2O_API int h2o_scores_add(const h2o_dims_t* dims, float* scores, const float* score_inc,
+                   void* stream);
+
 /* Empties a cache before a new sequence: slot_pos (B, Hkv, M) int32 := -1 and
  * scores (B, Hkv, M) f32 := 0, enqueued on `stream` (the K/V buffers need no
  * clearing: empty slots are never attended and are overwritten first).  This

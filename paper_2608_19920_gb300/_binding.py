@@ -21,7 +21,7 @@ H2O_DEVERR_CANDIDATES = 2
 
 # Every symbol include/h2o.h declares.
 EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
-           "h2o_update_policy",
+           "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
            "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
            "h2o_version")
 
@@ -65,11 +65,15 @@ def load(path: str = LIB_PATH):
     lib.h2o_update.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, vp]
     lib.h2o_update_policy.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, i32, i32, i32,
                                       vp, vp]
+    lib.h2o_evict_insert.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, i32, i32, i32, vp, vp]
+    lib.h2o_sdpa_cache.argtypes = [dims_p, i64, f32, vp, vp, vp, vp, vp, vp, vp, ctypes.c_size_t,
+                                   vp]
+    lib.h2o_scores_add.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_status_string.argtypes = [ctypes.c_int]
     lib.h2o_status_string.restype = ctypes.c_char_p
     for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
-               "h2o_update_policy",
+               "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
                "h2o_cache_reset",
                "h2o_last_cuda_error",
                "h2o_device_errors", "h2o_version"):
@@ -240,6 +244,81 @@ def h2o_update_policy(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cach
     return h2o_update(scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache, pos0,
                       recent_window, evict_idx=evict_idx, budget=budget, stream=stream,
                       policy=policy)
+
+
+def h2o_evict_insert(scores, slot_pos, k_new, v_new, k_cache, v_cache, pos0: int,
+                     recent_window: int, policy: str = "h2o", evict_idx=None,
+                     budget: int | None = None, Hq: int | None = None, stream=None):
+    """Paper-order step, part 1 (see include/h2o.h): the S lowest-scored
+    candidate slots take the chunk's K/V, position pos0 + c and score 0, in
+    place.  ``Hq`` only fills the size struct (default: Hkv).  Returns evict_idx."""
+    lib = load()
+    dev = scores.device
+    B, Hkv, M = scores.shape
+    S, d = k_new.shape[2], k_new.shape[3]
+    if policy not in POLICY:
+        raise ValueError(f"unknown policy {policy!r}")
+    _expect(scores, "scores", (B, Hkv, M), torch.float32, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    _expect(k_new, "k_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect(v_new, "v_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect(k_cache, "k_cache", (B, Hkv, M, d), torch.bfloat16, dev)
+    _expect(v_cache, "v_cache", (B, Hkv, M, d), torch.bfloat16, dev)
+    if evict_idx is not None:
+        _expect(evict_idx, "evict_idx", (B, Hkv, S), torch.int32, dev)
+    dims = H2ODims(B, Hkv if Hq is None else Hq, Hkv, d, S, M)
+    st = lib.h2o_evict_insert(ctypes.byref(dims), int(pos0), _ptr(scores), _ptr(slot_pos),
+                              _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache),
+                              int(M if budget is None else budget), int(recent_window),
+                              POLICY[policy], _ptr(evict_idx), _stream(stream))
+    _check("h2o_evict_insert", st)
+    return evict_idx
+
+
+def h2o_sdpa_cache(q, k_cache, v_cache, slot_pos, pos0: int, scale: float = 0.0, out=None,
+                   score_inc=None, workspace=None, stream=None):
+    """Paper-order step, part 2: SDPA of the chunk over the M cache slots only
+    (the chunk's K/V already written there).  Returns (out (B,Hq,S,d) bf16,
+    score_inc (B,Hq,M) f32)."""
+    lib = load()
+    dev = q.device
+    B, Hq, S, d = q.shape
+    Hkv, M = k_cache.shape[1], k_cache.shape[2]
+    bf = torch.bfloat16
+    _expect(q, "q", (B, Hq, S, d), bf, dev)
+    _expect(k_cache, "k_cache", (B, Hkv, M, d), bf, dev)
+    _expect(v_cache, "v_cache", (B, Hkv, M, d), bf, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    if out is None:
+        out = torch.empty((B, Hq, S, d), dtype=bf, device=dev)
+    if score_inc is None:
+        score_inc = torch.empty((B, Hq, M), dtype=torch.float32, device=dev)
+    _expect(out, "out", (B, Hq, S, d), bf, dev)
+    _expect(score_inc, "score_inc", (B, Hq, M), torch.float32, dev)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    if workspace is None:
+        n = h2o_workspace_size(dims)
+        if n:
+            workspace = torch.empty(n, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.h2o_sdpa_cache(ctypes.byref(dims), int(pos0), float(scale), _ptr(q), _ptr(k_cache),
+                            _ptr(v_cache), _ptr(slot_pos), _ptr(out), _ptr(score_inc),
+                            _ptr(workspace), ws_bytes, _stream(stream))
+    _check("h2o_sdpa_cache", st)
+    return out, score_inc
+
+
+def h2o_scores_add(scores, score_inc, stream=None):
+    """Paper-order step, part 3: scores += the GQA-group sum of score_inc (B,Hq,M)."""
+    lib = load()
+    dev = scores.device
+    B, Hkv, M = scores.shape
+    Hq = score_inc.shape[1]
+    _expect(scores, "scores", (B, Hkv, M), torch.float32, dev)
+    _expect(score_inc, "score_inc", (B, Hq, M), torch.float32, dev)
+    dims = H2ODims(B, Hq, Hkv, 64, 1, M)
+    _check("h2o_scores_add", lib.h2o_scores_add(ctypes.byref(dims), _ptr(scores),
+                                                _ptr(score_inc), _stream(stream)))
 
 
 def h2o_cache_reset(slot_pos, scores, stream=None):

@@ -115,6 +115,150 @@ int check_dims(const h2o_dims_t* d) {
   return H2O_OK;
 }
 
+// h2o_sdpa_chunk (cache_only = false: keys are the M slots, then the chunk's
+// S tokens) and h2o_sdpa_cache (cache_only = true: the M slots only, the
+// chunk's keys already written there; k_new / v_new unused).
+int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
+              const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
+              const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out, float* score_inc,
+              void* workspace, size_t workspace_bytes, void* stream, bool cache_only) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (!q || !out || !score_inc || (!cache_only && (!k_new || !v_new))) return H2O_ERR_NULL;
+  if (D.M > 0 && (!k_cache || !v_cache || !slot_pos)) return H2O_ERR_NULL;
+  if (misaligned(q) || misaligned(k_new) || misaligned(v_new) || misaligned(out) ||
+      misaligned(score_inc) || (D.M > 0 && (misaligned(k_cache) || misaligned(v_cache) ||
+                                            misaligned(slot_pos))))
+    return H2O_ERR_ALIGN;
+  const int nk = cache_only ? D.M : D.M + D.S;  // key columns of a score_inc row
+  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
+  const int qg = D.Hq / D.Hkv;
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
+  int split_len = 0, n_split = 0;
+  size_t ws_need = 0;
+  const bool decode = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
+  if (decode && (!workspace || workspace_bytes < ws_need)) return H2O_ERR_WORKSPACE;
+  if (decode && misaligned(workspace)) return H2O_ERR_ALIGN;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  if (decode) {
+    // one query token per sequence: split-K kernels (h2o_decode.cu)
+    DecodeArgs a;
+    a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
+    a.slot_pos = slot_pos; a.out = out; a.score_inc = score_inc;
+    a.part = static_cast<float*>(workspace);
+    a.err = di->err_word;
+    a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.M = D.M; a.qg = qg;
+    a.pos0 = static_cast<int>(pos0);
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.split_len = split_len;
+    a.n_split = n_split;
+    a.with_new = cache_only ? 0 : 1;
+    a.nk = nk;
+    const cudaError_t e = launch_decode(a, s);
+    return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+  }
+  if ((st = get_encoder()) != H2O_OK) return st;
+
+  SdpaArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = qg;
+  a.pos0 = static_cast<int>(pos0);
+  a.scale_log2 = scale * 1.4426950408889634f;
+  if (D.S > kTileM) {
+    a.rows_box = kTileM;
+    a.heads_box = 1;
+    a.tiles_per_head = (D.S + kTileM - 1) / kTileM;
+    a.n_row_tiles = qg * a.tiles_per_head;
+  } else {
+    a.rows_box = (D.S + 31) / 32 * 32;
+    a.heads_box = kTileM / a.rows_box;
+    a.tiles_per_head = 0;
+    a.n_row_tiles = (qg + a.heads_box - 1) / a.heads_box;
+  }
+  a.n_cache_tiles = (D.M + kTileN - 1) / kTileN;
+  a.n_chunk_tiles = cache_only ? 0 : (D.S + kTileN - 1) / kTileN;
+  a.nk = nk;
+  a.slot_pos = slot_pos;
+  a.out = out;
+  a.score_inc = score_inc;
+  a.err = di->err_word;
+
+  const uint64_t G = static_cast<uint64_t>(D.B) * D.Hkv;
+  {
+    const uint64_t dq[4] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S),
+                            static_cast<uint64_t>(qg), G};
+    const uint32_t bq[4] = {64, static_cast<uint32_t>(a.rows_box), static_cast<uint32_t>(a.heads_box), 1};
+    if ((st = encode(&a.tm_q, q, 4, dq, bq)) != H2O_OK) return st;
+    // d = 128 runs on CTA pairs: each CTA loads 64 keys of a K tile and 64
+    // columns of a V tile; d = 64 loads whole 128-key tiles.
+    const uint64_t dn[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S), G};
+    const uint32_t bk[3] = {64, D.d == 128 ? kTileN / 2u : kTileN, 1};
+    const uint32_t bv[3] = {64, kTileN, 1};
+    const uint64_t dc[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.M), G};
+    if (cache_only) {  // no chunk tiles: the chunk maps are never read
+      if ((st = encode(&a.tm_kn, k_cache, 3, dc, bk)) != H2O_OK) return st;
+      if ((st = encode(&a.tm_vn, v_cache, 3, dc, bv)) != H2O_OK) return st;
+    } else {
+      if ((st = encode(&a.tm_kn, k_new, 3, dn, bk)) != H2O_OK) return st;
+      if ((st = encode(&a.tm_vn, v_new, 3, dn, bv)) != H2O_OK) return st;
+    }
+    if (D.M > 0) {
+      if ((st = encode(&a.tm_kc, k_cache, 3, dc, bk)) != H2O_OK) return st;
+      if ((st = encode(&a.tm_vc, v_cache, 3, dc, bv)) != H2O_OK) return st;
+    }
+  }
+  const size_t inc_bytes = static_cast<size_t>(G) * qg * static_cast<size_t>(nk) * sizeof(float);
+  cudaError_t e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = launch_sdpa(a, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return H2O_OK;
+}
+
+// h2o_update_policy (insert = false) and h2o_evict_insert (insert = true:
+// score_inc is not read and may be NULL).
+int update_impl(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+                const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
+                h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget, int32_t recent_window,
+                int32_t policy, int32_t* evict_idx, void* stream, bool insert) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (!scores || !slot_pos || (!insert && !score_inc) || !k_new || !v_new || !k_cache ||
+      !v_cache)
+    return H2O_ERR_NULL;
+  if (misaligned(scores) || misaligned(slot_pos) || misaligned(score_inc) || misaligned(k_new) ||
+      misaligned(v_new) || misaligned(k_cache) || misaligned(v_cache) ||
+      (evict_idx && misaligned(evict_idx)))
+    return H2O_ERR_ALIGN;
+  if (budget != D.M) return H2O_ERR_ARG;
+  if (policy != H2O_POLICY_H2O && policy != H2O_POLICY_NORM && policy != H2O_POLICY_ORIG)
+    return H2O_ERR_ARG;
+  if (D.M < 1 || D.S > D.M) return H2O_ERR_SHAPE;
+  if (recent_window < 0 || recent_window > D.M) return H2O_ERR_ARG;
+  if (D.M - std::max(0, recent_window - D.S) < D.S) return H2O_ERR_ARG;
+  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  UpdateArgs a;
+  a.scores = scores; a.slot_pos = slot_pos; a.score_inc = insert ? nullptr : score_inc;
+  a.k_new = k_new; a.v_new = v_new; a.k_cache = k_cache; a.v_cache = v_cache;
+  a.evict_idx = evict_idx; a.err = di->err_word;
+  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = D.Hq / D.Hkv;
+  a.pos0 = static_cast<int>(pos0);
+  a.W = recent_window;
+  a.policy = policy;
+  a.insert = insert ? 1 : 0;
+  const cudaError_t e = launch_update(a, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e);
+  return H2O_OK;
+}
+
 }  // namespace
 }  // namespace h2o
 
@@ -158,93 +302,17 @@ int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, co
                    const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
                    const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out,
                    float* score_inc, void* workspace, size_t workspace_bytes, void* stream) {
-  int st = check_dims(dims);
-  if (st != H2O_OK) return st;
-  const h2o_dims_t& D = *dims;
-  if (!q || !k_new || !v_new || !out || !score_inc) return H2O_ERR_NULL;
-  if (D.M > 0 && (!k_cache || !v_cache || !slot_pos)) return H2O_ERR_NULL;
-  if (misaligned(q) || misaligned(k_new) || misaligned(v_new) || misaligned(out) ||
-      misaligned(score_inc) || (D.M > 0 && (misaligned(k_cache) || misaligned(v_cache) ||
-                                            misaligned(slot_pos))))
-    return H2O_ERR_ALIGN;
-  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
-  if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
-  const int qg = D.Hq / D.Hkv;
-  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
-  int split_len = 0, n_split = 0;
-  size_t ws_need = 0;
-  const bool decode = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
-  if (decode && (!workspace || workspace_bytes < ws_need)) return H2O_ERR_WORKSPACE;
-  if (decode && misaligned(workspace)) return H2O_ERR_ALIGN;
-  DeviceInfo* di = nullptr;
-  if ((st = current_device(&di)) != H2O_OK) return st;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return sdpa_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, k_new, v_new, slot_pos, out,
+                   score_inc, workspace, workspace_bytes, stream, false);
+}
 
-  if (decode) {
-    // one query token per sequence: split-K kernels (h2o_decode.cu)
-    DecodeArgs a;
-    a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
-    a.slot_pos = slot_pos; a.out = out; a.score_inc = score_inc;
-    a.part = static_cast<float*>(workspace);
-    a.err = di->err_word;
-    a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.M = D.M; a.qg = qg;
-    a.pos0 = static_cast<int>(pos0);
-    a.scale_log2 = scale * 1.4426950408889634f;
-    a.split_len = split_len;
-    a.n_split = n_split;
-    const cudaError_t e = launch_decode(a, s);
-    return e == cudaSuccess ? H2O_OK : cuda_fail(e);
-  }
-  if ((st = get_encoder()) != H2O_OK) return st;
-
-  SdpaArgs a;
-  std::memset(&a, 0, sizeof(a));
-  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = qg;
-  a.pos0 = static_cast<int>(pos0);
-  a.scale_log2 = scale * 1.4426950408889634f;
-  if (D.S > kTileM) {
-    a.rows_box = kTileM;
-    a.heads_box = 1;
-    a.tiles_per_head = (D.S + kTileM - 1) / kTileM;
-    a.n_row_tiles = qg * a.tiles_per_head;
-  } else {
-    a.rows_box = (D.S + 31) / 32 * 32;
-    a.heads_box = kTileM / a.rows_box;
-    a.tiles_per_head = 0;
-    a.n_row_tiles = (qg + a.heads_box - 1) / a.heads_box;
-  }
-  a.n_cache_tiles = (D.M + kTileN - 1) / kTileN;
-  a.n_chunk_tiles = (D.S + kTileN - 1) / kTileN;
-  a.slot_pos = slot_pos;
-  a.out = out;
-  a.score_inc = score_inc;
-  a.err = di->err_word;
-
-  const uint64_t G = static_cast<uint64_t>(D.B) * D.Hkv;
-  {
-    const uint64_t dq[4] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S),
-                            static_cast<uint64_t>(qg), G};
-    const uint32_t bq[4] = {64, static_cast<uint32_t>(a.rows_box), static_cast<uint32_t>(a.heads_box), 1};
-    if ((st = encode(&a.tm_q, q, 4, dq, bq)) != H2O_OK) return st;
-    // d = 128 runs on CTA pairs: each CTA loads 64 keys of a K tile and 64
-    // columns of a V tile; d = 64 loads whole 128-key tiles.
-    const uint64_t dn[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S), G};
-    const uint32_t bk[3] = {64, D.d == 128 ? kTileN / 2u : kTileN, 1};
-    const uint32_t bv[3] = {64, kTileN, 1};
-    if ((st = encode(&a.tm_kn, k_new, 3, dn, bk)) != H2O_OK) return st;
-    if ((st = encode(&a.tm_vn, v_new, 3, dn, bv)) != H2O_OK) return st;
-    if (D.M > 0) {
-      const uint64_t dc[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.M), G};
-      if ((st = encode(&a.tm_kc, k_cache, 3, dc, bk)) != H2O_OK) return st;
-      if ((st = encode(&a.tm_vc, v_cache, 3, dc, bv)) != H2O_OK) return st;
-    }
-  }
-  const size_t inc_bytes = static_cast<size_t>(G) * qg * (static_cast<size_t>(D.M) + D.S) * sizeof(float);
-  cudaError_t e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
-  if (e != cudaSuccess) return cuda_fail(e);
-  e = launch_sdpa(a, s);
-  if (e != cudaSuccess) return cuda_fail(e);
-  return H2O_OK;
+int h2o_sdpa_cache(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
+                   const h2o_bf16* k_cache, const h2o_bf16* v_cache, const int32_t* slot_pos,
+                   h2o_bf16* out, float* score_inc, void* workspace, size_t workspace_bytes,
+                   void* stream) {
+  if (dims && dims->M < 1) return H2O_ERR_SHAPE;
+  return sdpa_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, nullptr, nullptr, slot_pos,
+                   out, score_inc, workspace, workspace_bytes, stream, true);
 }
 
 int h2o_sdpa_decode_static(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
@@ -286,6 +354,8 @@ int h2o_sdpa_decode_static(const h2o_dims_t* dims, int64_t pos0, float softmax_s
   a.scale_log2 = scale * 1.4426950408889634f;
   a.split_len = split_len;
   a.n_split = n_split;
+  a.with_new = 1;
+  a.nk = D.M + 1;
   e = launch_decode(a, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? H2O_OK : cuda_fail(e);
 }
@@ -302,35 +372,33 @@ int h2o_update_policy(const h2o_dims_t* dims, int64_t pos0, float* scores, int32
                       const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
                       h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget,
                       int32_t recent_window, int32_t policy, int32_t* evict_idx, void* stream) {
+  return update_impl(dims, pos0, scores, slot_pos, score_inc, k_new, v_new, k_cache, v_cache,
+                     budget, recent_window, policy, evict_idx, stream, false);
+}
+
+int h2o_evict_insert(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+                     const h2o_bf16* k_new, const h2o_bf16* v_new, h2o_bf16* k_cache,
+                     h2o_bf16* v_cache, int32_t budget, int32_t recent_window, int32_t policy,
+                     int32_t* evict_idx, void* stream) {
+  return update_impl(dims, pos0, scores, slot_pos, nullptr, k_new, v_new, k_cache, v_cache,
+                     budget, recent_window, policy, evict_idx, stream, true);
+}
+
+int h2o_scores_add(const h2o_dims_t* dims, float* scores, const float* score_inc, void* stream) {
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
-  if (!scores || !slot_pos || !score_inc || !k_new || !v_new || !k_cache || !v_cache)
-    return H2O_ERR_NULL;
-  if (misaligned(scores) || misaligned(slot_pos) || misaligned(score_inc) || misaligned(k_new) ||
-      misaligned(v_new) || misaligned(k_cache) || misaligned(v_cache) ||
-      (evict_idx && misaligned(evict_idx)))
-    return H2O_ERR_ALIGN;
-  if (budget != D.M) return H2O_ERR_ARG;
-  if (policy != H2O_POLICY_H2O && policy != H2O_POLICY_NORM && policy != H2O_POLICY_ORIG)
-    return H2O_ERR_ARG;
-  if (D.M < 1 || D.S > D.M) return H2O_ERR_SHAPE;
-  if (recent_window < 0 || recent_window > D.M) return H2O_ERR_ARG;
-  if (D.M - std::max(0, recent_window - D.S) < D.S) return H2O_ERR_ARG;
-  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  if (D.M < 1) return H2O_ERR_SHAPE;
+  if (!scores || !score_inc) return H2O_ERR_NULL;
+  if (misaligned(scores) || misaligned(score_inc)) return H2O_ERR_ALIGN;
   DeviceInfo* di = nullptr;
   if ((st = current_device(&di)) != H2O_OK) return st;
-  UpdateArgs a;
-  a.scores = scores; a.slot_pos = slot_pos; a.score_inc = score_inc;
-  a.k_new = k_new; a.v_new = v_new; a.k_cache = k_cache; a.v_cache = v_cache;
-  a.evict_idx = evict_idx; a.err = di->err_word;
-  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = D.Hq / D.Hkv;
-  a.pos0 = static_cast<int>(pos0);
-  a.W = recent_window;
-  a.policy = policy;
-  const cudaError_t e = launch_update(a, static_cast<cudaStream_t>(stream));
-  if (e != cudaSuccess) return cuda_fail(e);
-  return H2O_OK;
+  ScoresAddArgs a;
+  a.scores = scores;
+  a.score_inc = score_inc;
+  a.B = D.B; a.Hkv = D.Hkv; a.M = D.M; a.qg = D.Hq / D.Hkv;
+  const cudaError_t e = launch_scores_add(a, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
 }
 
 int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores, void* stream) {

@@ -128,8 +128,8 @@ __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int it) {
   x.s = it % a.n_split;
   x.j0 = x.s * a.split_len;
   x.n_cache = min(a.split_len, a.M - x.j0);  // >= 1: n_split = ceil(M / split_len)
-  x.last = x.s == a.n_split - 1;
-  x.n_loc = x.n_cache + (x.last ? 1 : 0);    // local key n_cache is the new token
+  x.last = x.s == a.n_split - 1 && a.with_new;  // this item also takes the new token
+  x.n_loc = x.n_cache + (x.last ? 1 : 0);        // local key n_cache is the new token
   x.n_tiles = (x.n_loc + DecGeom<D>::kTileKeys - 1) / DecGeom<D>::kTileKeys;
   return x;
 }
@@ -319,7 +319,7 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
           for (int e = 0; e < 4; ++e) {
             w[e] = vis ? w[e] * a.scale_log2 : -INFINITY;
             if (g4 + e < a.qg) {
-              a.score_inc[(row0 + g4 + e) * (static_cast<size_t>(a.M) + 1) + j] = w[e];
+              a.score_inc[(row0 + g4 + e) * static_cast<size_t>(a.nk) + j] = w[e];
               mx[g4 + e] = fmaxf(mx[g4 + e], w[e]);
             }
           }
@@ -514,9 +514,9 @@ __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const D
       a.out[row * D + dd] = static_cast<uint16_t>(pack_bf16x2(t * inv, 0.f) & 0xFFFFu);
     }
   }
-  float* inc = a.score_inc + row * (static_cast<size_t>(a.M) + 1);
+  float* inc = a.score_inc + row * static_cast<size_t>(a.nk);
   const int c0 = static_cast<int>(blockIdx.y) * kCombineCols;
-  const int c1 = min(c0 + kCombineCols, a.M + 1);
+  const int c1 = min(c0 + kCombineCols, a.nk);
 #pragma unroll 4
   for (int j = c0 + tid; j < c1; j += kCombineThreads) inc[j] = fast_exp2(inc[j] - lam);
 }
@@ -563,7 +563,7 @@ cudaError_t launch_d(const DecodeArgs& a, cudaStream_t stream) {
   cudaError_t e = a.qg <= 4 ? launch_split<D, 4>(a, stream) : launch_split<D, 8>(a, stream);
   if (e != cudaSuccess) return e;
   const dim3 grid(static_cast<unsigned>(a.B * a.Hq),
-                  static_cast<unsigned>((a.M + 1 + kCombineCols - 1) / kCombineCols));
+                  static_cast<unsigned>((a.nk + kCombineCols - 1) / kCombineCols));
   const size_t smem = static_cast<size_t>(std::max(a.n_split, kCombineThreads)) * sizeof(float);
   decode_combine_kernel<D><<<grid, kCombineThreads, smem, stream>>>(a);
   return cudaGetLastError();

@@ -33,7 +33,8 @@ struct SdpaArgs {
   int tiles_per_head;      // ceil(S / 128) when S > 128, else 0
   int n_row_tiles;         // CTAs per (b, kv head)
   int n_cache_tiles;       // ceil(M / 128)
-  int n_chunk_tiles;       // ceil(S / 128)
+  int n_chunk_tiles;       // ceil(S / 128); 0 for h2o_sdpa_cache (keys in the cache only)
+  int nk;                  // key columns of a score_inc row: M + S, or M for h2o_sdpa_cache
 };
 
 struct UpdateArgs {
@@ -50,6 +51,14 @@ struct UpdateArgs {
   int pos0;
   int W;
   int policy;              // H2O_POLICY_*
+  int insert;              // 1: h2o_evict_insert (rank on scores as they are, no score_inc;
+                           //    the new slots score 0; h2o_norm's t is pos0)
+};
+
+struct ScoresAddArgs {
+  float* scores;           // (B, Hkv, M) in/out
+  const float* score_inc;  // (B, Hq, M)
+  int B, Hkv, M, qg;
 };
 
 // S = 1 (one query token per sequence): split-K decode kernels.
@@ -75,6 +84,8 @@ struct DecodeArgs {
   float scale_log2;
   int split_len;            // cache slots per split (multiple of 16)
   int n_split;              // ceil(M / split_len); the last split also takes the new token
+  int with_new;             // 1: the new token is key column M; 0: h2o_sdpa_cache (none)
+  int nk;                   // score_inc row length: M + with_new
 };
 
 // Split of the M cache slots for the decode kernels (a function of the sizes
@@ -92,5 +103,6 @@ cudaError_t decode_static_scratch(void** ptr);
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);
+cudaError_t launch_scores_add(const ScoresAddArgs& a, cudaStream_t stream);
 
 }  // namespace h2o

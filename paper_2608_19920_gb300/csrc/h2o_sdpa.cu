@@ -205,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
   const bool leader = rank == 0;
   const int b = grp / a.Hkv;
   const int hkv = grp % a.Hkv;
-  const int NK = a.M + a.S;    // key columns per query head
+  const int NK = a.nk;         // key columns per query head (score_inc row length)
 
   int g_first = a.qg, i_lo = 0, i_hi = -1;
   const bool has_rows = row_range(a, rt, g_first, i_lo, i_hi);

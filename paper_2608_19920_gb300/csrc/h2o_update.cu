@@ -32,6 +32,8 @@
 // bound (a few MB per chunk), so the design minimises dependent round trips.
 // Otherwise one CTA per (b, kv head) recomputes keys from global memory on
 // every pass.  S = 1 has a kernel of its own (update_decode_kernel).
+#include <algorithm>
+
 #include "h2o_internal.h"
 #include "sm100.cuh"
 
@@ -55,6 +57,18 @@ __device__ __forceinline__ float group_sum(const float* inc, int stride, int qg,
   return t;
 }
 
+// The group sum of score_inc, or 0 for h2o_evict_insert (a.insert: the
+// paper's order ranks and keeps the scores as they were before the chunk).
+__device__ __forceinline__ float inc_group(const UpdateArgs& a, const float* inc, int stride,
+                                           int j) {
+  return a.insert ? 0.f : group_sum(inc, stride, a.qg, j);
+}
+
+// Tokens processed when the choice is made: t of h2o_norm's age t - t(j).
+__device__ __forceinline__ int t_choice(const UpdateArgs& a) {
+  return a.insert ? a.pos0 : a.pos0 + a.S;
+}
+
 // Selection key of a slot (step 2 above).  The rank value is the score for
 // h2o and h2o_orig (the caller passes the batch sum) and, for h2o_norm, the
 // score over the slot's age t - t(j), t = pos0 + S (fp32, rounded to nearest).
@@ -69,7 +83,7 @@ __device__ __forceinline__ uint32_t make_key(float acc, int pos, int thr, int po
 __device__ __forceinline__ float slot_acc(const UpdateArgs& a, int b, int h, int j) {
   const size_t grp = static_cast<size_t>(b) * a.Hkv + h;
   const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * a.qg) * (a.M + a.S);
-  return __fadd_rn(a.scores[grp * a.M + j], group_sum(inc, a.M + a.S, a.qg, j));
+  return __fadd_rn(a.scores[grp * a.M + j], inc_group(a, inc, a.M + a.S, j));
 }
 
 // Key of slot j for the selection of (b, h) (h2o_orig: of KV head h, b = 0);
@@ -81,7 +95,7 @@ __device__ __forceinline__ uint32_t slot_key(const UpdateArgs& a, int b, int h, 
   *acc_out = acc;
   if (a.policy == H2O_POLICY_ORIG)
     for (int bb = 1; bb < a.B; ++bb) acc = __fadd_rn(acc, slot_acc(a, bb, h, j));
-  return make_key(acc, pos, thr, a.policy, a.pos0 + a.S);
+  return make_key(acc, pos, thr, a.policy, t_choice(a));
 }
 
 // Exclusive block scan of one bit per thread; returns the prefix, total in *tot.
@@ -200,7 +214,7 @@ __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs
         const float* inc = a.score_inc + static_cast<size_t>(bb * a.Hq + h * a.qg) * (M + S);
         if (sel) {
           // the new token's own column
-          a.scores[g * M + j] = group_sum(inc + M, M + S, a.qg, static_cast<int>(c));
+          a.scores[g * M + j] = inc_group(a, inc + M, M + S, static_cast<int>(c));
           a.slot_pos[g * M + j] = a.pos0 + static_cast<int>(c);
           if (a.evict_idx) a.evict_idx[g * S + c] = j;
         } else {
@@ -298,7 +312,12 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
     const float* sc = scores_of(b);
     const float* inc = inc_of(b);
     float sv[kBatch], tv[kBatch];
-    if (vec && n == kBatch) {
+    if (a.insert) {  // scores as they are
+      for (int k = 0; k < n; ++k) {
+        sv[k] = sc[jb + k];
+        tv[k] = 0.f;
+      }
+    } else if (vec && n == kBatch) {
       float4 s4[2];
 #pragma unroll
       for (int q = 0; q < 2; ++q) s4[q] = *reinterpret_cast<const float4*>(sc + jb + 4 * q);
@@ -329,7 +348,7 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
     } else {
       for (int k = 0; k < n; ++k) {
         sv[k] = sc[jb + k];
-        tv[k] = group_sum(inc, NK, qg, jb + k);
+        tv[k] = inc_group(a, inc, NK, jb + k);
       }
     }
 #pragma unroll
@@ -357,13 +376,13 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
     // h2o_orig sums the batch entries in ascending b
     for (int bi = 0; bi < nb; ++bi) add_acc(b0 + bi, jb, n, tot, bi == 0);
     for (int k = 0; k < n; ++k) {
-      keys[jb + k] = make_key(tot[k], pv[k], thr, a.policy, a.pos0 + S);
+      keys[jb + k] = make_key(tot[k], pv[k], thr, a.policy, t_choice(a));
       if (!orig) accs[jb + k] = tot[k];
     }
   }
   // scores of the new tokens: their own columns M + c, summed over the group
   if (!orig)
-    for (int c = tid; c < S; c += kCThreads) nscore[c] = group_sum(inc_of(b0) + M, NK, qg, c);
+    for (int c = tid; c < S; c += kCThreads) nscore[c] = inc_group(a, inc_of(b0) + M, NK, c);
   // Every CTA of the cluster has read the old state before CTA 0 rewrites it.
   cluster_sync_all();
 
@@ -447,7 +466,7 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
             if (a.evict_idx) a.evict_idx[g * S + c] = j;
           }
           if (orig) {
-            scores_of(b)[j] = sel ? group_sum(inc_of(b) + M, NK, qg, static_cast<int>(c))
+            scores_of(b)[j] = sel ? inc_group(a, inc_of(b) + M, NK, static_cast<int>(c))
                                   : slot_acc(a, b, h, j);
           } else if (sel) {
             accs[j] = nscore[c];
@@ -534,7 +553,8 @@ __global__ void __launch_bounds__(kDThreads, 2)
   const int nb = orig ? a.B : 1;
   const int M = a.M, NK = M + 1, qg = a.qg;
   const int thr = a.pos0 + 1 - a.W;
-  const int t_now = a.pos0 + 1;
+  const int t_now = t_choice(a);
+  const int qg_inc = a.insert ? 0 : qg;  // score_inc rows read per slot
   const int per = (M + C - 1) / C;
   const int jlo = min(M, rank * per), jhi = min(M, jlo + per);
   const int32_t* pos_b0 = a.slot_pos + (static_cast<size_t>(b0) * a.Hkv + h) * M;
@@ -549,9 +569,9 @@ __global__ void __launch_bounds__(kDThreads, 2)
     for (int u = 0; u < kDBatch; ++u) {
       const int j = base + u * kDThreads;
       old[u] = j < jhi ? sc[j] : 0.f;
-      t[u] = j < jhi ? __ldg(inc + j) : 0.f;
+      t[u] = j < jhi && qg_inc > 0 ? __ldg(inc + j) : 0.f;
     }
-    for (int g = 1; g < qg; ++g) {
+    for (int g = 1; g < qg_inc; ++g) {
       float x[kDBatch];
 #pragma unroll
       for (int u = 0; u < kDBatch; ++u) {
@@ -652,7 +672,7 @@ __global__ void __launch_bounds__(kDThreads, 2)
     const int grp = b * a.Hkv + h;
     if (lane == 0) {
       const float* inc = a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK;
-      a.scores[static_cast<size_t>(grp) * M + e] = group_sum(inc, NK, qg, M);
+      a.scores[static_cast<size_t>(grp) * M + e] = inc_group(a, inc, NK, M);
       a.slot_pos[static_cast<size_t>(grp) * M + e] = a.pos0;
       if (a.evict_idx) a.evict_idx[grp] = e;
     }
@@ -660,7 +680,29 @@ __global__ void __launch_bounds__(kDThreads, 2)
   }
 }
 
+// Last part of the paper-order chunk step (Eq. 3): scores += the group sum of
+// score_inc, in the same float32 order as the update kernels (one thread per
+// slot; the kernel moves 4 (1 + q_g) bytes per slot and is bandwidth bound).
+__global__ void __launch_bounds__(256) scores_add_kernel(const ScoresAddArgs a) {
+  const size_t n = static_cast<size_t>(a.B) * a.Hkv * a.M;
+  const size_t stride = static_cast<size_t>(gridDim.x) * blockDim.x;
+  for (size_t x = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; x < n; x += stride) {
+    const size_t grp = x / a.M;
+    const int j = static_cast<int>(x % a.M);
+    const size_t b = grp / a.Hkv, h = grp % a.Hkv;
+    const float* inc = a.score_inc + (b * (a.Hkv * a.qg) + h * a.qg) * a.M;
+    a.scores[x] = __fadd_rn(a.scores[x], group_sum(inc, a.M, a.qg, j));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_scores_add(const ScoresAddArgs& a, cudaStream_t stream) {
+  const size_t n = static_cast<size_t>(a.B) * a.Hkv * a.M;
+  const size_t blocks = std::min<size_t>((n + 255) / 256, 152 * 8);
+  scores_add_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(a);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
   const size_t smem = (2 * static_cast<size_t>(a.M) + 2 * static_cast<size_t>(a.S)) * sizeof(uint32_t);

@@ -1,9 +1,11 @@
 """Chunk-loop driver for one attention layer with an H2O cache (§3.1, §A.4.1).
 
 The layer state (cache buffers, slot positions, scores) lives in torch tensors
-on the GPU; every step runs the library's two calls on the current stream:
-``h2o_sdpa_chunk`` then ``h2o_update``.  A sequence is a prefill of M tokens
-(attending to an empty cache) followed by chunks of S tokens.
+on the GPU; every step runs the library's calls on the current stream:
+``h2o_sdpa_chunk`` then ``h2o_update`` (the default order), or, in the
+paper's order, ``h2o_evict_insert``, ``h2o_sdpa_cache`` and ``h2o_scores_add``.
+A sequence is a prefill of M tokens (attending to an empty cache) followed by
+chunks of S tokens.
 """
 from __future__ import annotations
 
@@ -28,8 +30,14 @@ class H2OLayer:
 
     def __init__(self, B: int, Hq: int, Hkv: int, d: int, M: int, S: int, W: int,
                  device="cuda", scale: float = 0.0, keep_evictions: bool = True,
-                 policy: str = "h2o"):
-        """``policy``: eviction rule of §3.1.1, "h2o", "h2o_norm" or "h2o_orig"."""
+                 policy: str = "h2o", order: str = "chunk"):
+        """``policy``: eviction rule of §3.1.1, "h2o", "h2o_norm" or "h2o_orig".
+        ``order``: "chunk" (attend to the cache and the chunk, then update) or
+        "paper" (§3.1 / §3.3.1: evict and write first, attend to the cache,
+        then add the scores)."""
+        if order not in ("chunk", "paper"):
+            raise ValueError(f"unknown order {order!r}")
+        self.order = order
         self.B, self.Hq, self.Hkv, self.d, self.M, self.S, self.W = B, Hq, Hkv, d, M, S, W
         self.policy = policy
         self.scale = scale
@@ -50,7 +58,8 @@ class H2OLayer:
 
     def _buf(self, s: int):
         if s not in self._inc:
-            self._inc[s] = torch.empty((self.B, self.Hq, self.M + s), dtype=torch.float32,
+            nk = self.M if self.order == "paper" else self.M + s
+            self._inc[s] = torch.empty((self.B, self.Hq, nk), dtype=torch.float32,
                                        device=self.device)
             self._evict[s] = torch.empty((self.B, self.Hkv, s), dtype=torch.int32,
                                          device=self.device)
@@ -65,6 +74,16 @@ class H2OLayer:
         """
         s = q.shape[2]
         inc, ev, ws = self._buf(s)
+        if self.order == "paper":
+            lib.h2o_evict_insert(self.scores, self.slot_pos, k_new, v_new, self.k_cache,
+                                 self.v_cache, pos0, self.W, policy=self.policy,
+                                 evict_idx=ev if self.keep_evictions else None, Hq=self.Hq,
+                                 stream=stream)
+            out, inc = lib.h2o_sdpa_cache(q, self.k_cache, self.v_cache, self.slot_pos, pos0,
+                                          self.scale, out=out, score_inc=inc, workspace=ws,
+                                          stream=stream)
+            lib.h2o_scores_add(self.scores, inc, stream=stream)
+            return out, inc, ev
         out, inc = lib.h2o_sdpa_chunk(q, self.k_cache, self.v_cache, k_new, v_new, self.slot_pos,
                                       pos0, self.scale, out=out, score_inc=inc, workspace=ws,
                                       stream=stream)

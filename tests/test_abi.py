@@ -132,3 +132,28 @@ def test_binding_refuses_to_run_without_the_library(tmp_path):
             b.load(str(tmp_path / "missing.so"))
     finally:
         b._lib = saved
+
+
+def test_paper_order_argument_checks(lib):
+    """h2o_evict_insert / h2o_sdpa_cache / h2o_scores_add refuse bad arguments
+    on the host, before any device work."""
+    vp = ctypes.c_void_p
+    p = vp(0x1000)
+    d = _dims()
+    ev = lambda dims, budget=256, W=32, pos0=256, policy=0, ptrs=None: lib.h2o_evict_insert(
+        ctypes.byref(dims), pos0, *(ptrs or [p] * 6), budget, W, policy, None, None)
+    assert ev(d, budget=255) == ARG
+    assert ev(d, policy=3) == ARG
+    assert ev(d, W=257) == ARG
+    assert ev(_dims(S=300)) == SHAPE
+    assert ev(d, ptrs=[p] * 5 + [vp(0)]) == NULL
+    assert ev(d, ptrs=[vp(0x1004)] + [p] * 5) == ALIGN
+    sc = lambda dims, ptrs=None, ws=None, wsb=0: lib.h2o_sdpa_cache(
+        ctypes.byref(dims), 256, 0.0, *(ptrs or [p] * 6), ws, wsb, None)
+    assert sc(_dims(M=0)) == SHAPE
+    assert sc(d, ptrs=[p] * 5 + [vp(0)]) == NULL
+    assert sc(d, ptrs=[vp(0x1008)] + [p] * 5) == ALIGN
+    assert sc(_dims(S=1, M=100)) == WORKSPACE  # the decode kernels need their workspace
+    assert lib.h2o_scores_add(ctypes.byref(_dims(M=0)), p, p, None) == SHAPE
+    assert lib.h2o_scores_add(ctypes.byref(d), vp(0), p, None) == NULL
+    assert lib.h2o_scores_add(ctypes.byref(d), p, vp(0x1002), None) == ALIGN

@@ -53,10 +53,18 @@ def step_plan(w: wl.Workload):
     return chunk_bounds(w.T, w.M, w.S)
 
 
-def step_flops(w: wl.Workload):
+def visible_old(w: wl.Workload, S: int, order: str) -> int:
+    """Cache slots every row of a steady-state chunk sees besides the chunk's
+    own causal triangle: all M (attend, then evict), or M - S (the paper's
+    order: S slots already hold the chunk)."""
+    return w.M - S if order == "paper" else w.M
+
+
+def step_flops(w: wl.Workload, order: str = "chunk"):
     plan = step_plan(w)
     prefill = chunk_flops(w.B, w.Hq, w.d, plan[0][1], 0)
-    chunks = [chunk_flops(w.B, w.Hq, w.d, e - p, w.M) for p, e in plan[1:]]
+    chunks = [chunk_flops(w.B, w.Hq, w.d, e - p, visible_old(w, e - p, order))
+              for p, e in plan[1:]]
     return prefill, chunks
 
 
@@ -289,14 +297,15 @@ def run_ours(args, w):
     dev = torch.device("cuda", local)
     build_mod.build()
     plan = step_plan(w)
-    pre_flops, chunk_fl = step_flops(w)
+    pre_flops, chunk_fl = step_flops(w, args.order)
     total_flops = pre_flops + sum(chunk_fl)
     tokens_per_step = w.B * w.T
 
     inputs = make_inputs(w, dev)
     outs = [torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=dev)
             for p, e in plan]
-    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, keep_evictions=True)
+    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, keep_evictions=True,
+                     order=args.order)
     stream = torch.cuda.current_stream()
     n_chunks = len(plan) - 1
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -376,18 +385,20 @@ def run_ours(args, w):
                    "l2": f"inputs larger than L2 ({in_bytes / 1e6:.0f} MB per step)"
                          if in_bytes > 129e6 else f"{in_bytes / 1e6:.0f} MB of inputs per step",
                    "launch": "CUDA graph of the whole step" if args.graph else "eager",
+                   "order": args.order,
                    "parallelism": f"replicas x{world}"},
         "tflops": alg_tflops,
         "tflops_frac_of_peak": alg_tflops / pk["bf16_sus"],
         "chunk_step_ms_median": statistics.median(chunk_step_ms) if chunk_step_ms else None,
-        "gpu_launches": args.steps * sum(launches_per_chunk(e - p, w.M) for p, e in plan),
+        "gpu_launches": args.steps * sum(launches_per_chunk(e - p, w.M, args.order)
+                                         for p, e in plan),
         "clocks": clocks,
     }
     # the chunk SDPA is timed on its own (launch after launch, L2 flushed in
     # between): its denominator is the burst peak; the sustained one is given
     # alongside
     traffic = args.traffic if args.traffic is not None else (
-        SDPA_DRAM_BYTES if w.name == "llama8b_32k" else None)
+        SDPA_DRAM_BYTES if w.name == "llama8b_32k" and args.order == "chunk" else None)
     if w.S == 1:
         # decode: K and V read once per step, HBM bound
         line["roofline"] = {
@@ -399,7 +410,9 @@ def run_ours(args, w):
         }
     else:
         line["roofline"] = {
-            "bound": "tensor", "kernel": "sdpa_chunk_kernel<128,pair> (steady-state chunk)",
+            "bound": "tensor",
+            "kernel": "sdpa_chunk_kernel<128,pair> (steady-state chunk" +
+                      (", cache only)" if args.order == "paper" else ")"),
             "achieved": kern["alg_tflops"], "peak": pk["bf16"], "unit": "TFLOP/s",
             "frac": kern["alg_tflops"] / pk["bf16"], "traffic": traffic,
             "peak_source": f"{pk['source']} bf16 dense, burst",
@@ -416,11 +429,16 @@ def run_ours(args, w):
     return 0
 
 
-def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
+def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None, prepare=True):
     """Average duration of the steady-state chunk SDPA launch (CUDA events)."""
     import torch
-    from paper_2608_19920_gb300 import h2o_sdpa_chunk
+    from paper_2608_19920_gb300 import h2o_evict_insert, h2o_sdpa_cache, h2o_sdpa_chunk
     idx = len(plan) // 2 if idx is None else idx
+    if prepare and idx > 0:
+        # the cache as the sequence leaves it just before chunk idx
+        layer.reset()
+        for i in range(idx):
+            layer.step(*inputs[i], plan[i][0])
     p, e = plan[idx]
     q, k, v = inputs[idx]
     out = torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=q.device)
@@ -429,9 +447,16 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
     clean = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
 
     def call():
-        h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out=out,
-                       score_inc=inc, workspace=ws)
+        if layer.order == "paper":  # the cache already holds the chunk (filled by the caller)
+            h2o_sdpa_cache(q, layer.k_cache, layer.v_cache, layer.slot_pos, p, out=out,
+                           score_inc=inc, workspace=ws)
+        else:
+            h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out=out,
+                           score_inc=inc, workspace=ws)
 
+    if layer.order == "paper":
+        h2o_evict_insert(layer.scores, layer.slot_pos, k, v, layer.k_cache, layer.v_cache, p,
+                         layer.W, policy=layer.policy, Hq=layer.Hq)
     # the call is replayed from a CUDA graph, as in the timed steps
     call()
     graph = torch.cuda.CUDAGraph()
@@ -453,7 +478,7 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None):
         times.append(a.elapsed_time(b))
     times = times[2:]
     avg_ms = sum(times) / len(times)
-    flops = chunk_flops(w.B, w.Hq, w.d, e - p, w.M)
+    flops = chunk_flops(w.B, w.Hq, w.d, e - p, visible_old(w, e - p, layer.order))
     exec_flops = executed_mma_flops(w, e - p)
     kv_bytes = decode_kv_bytes(w)
     return dict(avg_us=avg_ms * 1e3, flops=flops, alg_tflops=flops / (avg_ms / 1e3) / 1e12,
@@ -465,10 +490,12 @@ def decode_kv_bytes(w):
     return 2.0 * w.B * w.Hkv * w.M * w.d * 2
 
 
-def launches_per_chunk(S, M):
+def launches_per_chunk(S, M, order="chunk"):
     """Kernels of this library one chunk launches: the SDPA (split + combine
-    when S = 1 and a cache exists) and the update."""
-    return 3 if S == 1 and M > 0 else 2
+    when S = 1 and a cache exists) and the update (the paper's order: the
+    eviction-insert, the SDPA and the score addition)."""
+    sdpa = 2 if S == 1 and M > 0 else 1
+    return sdpa + (2 if order == "paper" else 1)
 
 
 def executed_mma_flops(w, S):
@@ -530,6 +557,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama8b_32k", choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
+    ap.add_argument("--order", default="chunk", choices=["chunk", "paper"],
+                    help="chunk step order: attend then evict (default), or the paper's "
+                         "evict-and-write first")
     ap.add_argument("--no-graph", dest="graph", action="store_false",
                     help="launch the timed steps eagerly instead of replaying a CUDA graph")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
@@ -558,7 +588,7 @@ def run_kernel_only(args, w, n_fill: int = 8):
     build_mod.build()
     dev = torch.device("cuda", 0)
     plan = step_plan(w)[:n_fill + 2]
-    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev)
+    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, order=args.order)
     ins = []
     for p, e in plan:
         ins.append(tuple(torch.from_numpy(x).to(torch.bfloat16).to(dev)
@@ -567,7 +597,7 @@ def run_kernel_only(args, w, n_fill: int = 8):
     for (p, e), (q, k, v) in zip(plan[:-1], ins[:-1]):
         layer.step(q, k, v, p)
     kern = time_sdpa_kernel(w, layer, ins, plan, torch.cuda.current_stream(), reps=args.reps,
-                            idx=len(plan) - 1)
+                            idx=len(plan) - 1, prepare=False)
     torch.cuda.synchronize()
     assert h2o_device_errors() == 0
     print(json.dumps({"mode": "kernel", "workload": w.name, **kern}))

@@ -75,7 +75,8 @@ enum {
 /* Device error bits reported by h2o_device_errors(). */
 enum {
   H2O_DEVERR_TIMEOUT = 1,   /* a kernel's bounded wait on a barrier ran out */
-  H2O_DEVERR_CANDIDATES = 2 /* h2o_update found fewer than S evictable slots */
+  H2O_DEVERR_CANDIDATES = 2, /* h2o_update found fewer than S evictable slots */
+  H2O_DEVERR_INDEX = 4       /* h2o_kv_replace / h2o_kv_restore met an index outside [0, M) */
 };
 
 /* Bytes of scratch memory h2o_sdpa_chunk needs for `dims` (may be 0). */
@@ -230,6 +231,36 @@ H2O_API int h2o_sdpa_cache(const h2o_dims_t* dims, int64_t pos0, float softmax_s
                    size_t workspace_bytes, void* stream);
 H2O_API int h2o_scores_add(const h2o_dims_t* dims, float* scores, const float* score_inc,
                    void* stream);
+
+/*
+ * Replay-cache row operations (§3.2 recurrence, §A.1.1 scatter / gather):
+ *
+ *   h2o_kv_replace  for every (b, h, c): delta_k[b,h,c,:] = k_cache[b,h,e,:],
+ *                   then k_cache[b,h,e,:] = k_new[b,h,c,:], e = index[b,h,c];
+ *                   v likewise; slot_pos[b,h,e] := pos0 + c with its old value
+ *                   to delta_pos[b,h,c].  This is the cache write of a chunk
+ *                   whose eviction decisions are replayed from a log, keeping
+ *                   the rows it replaces (delta_key = gather(keys, index)).
+ *   h2o_kv_restore  the reverse recurrence: k_cache[b,h,e,:] = delta_k[b,h,c,:],
+ *                   v likewise, slot_pos[b,h,e] = delta_pos[b,h,c].
+ *
+ *   index      (B, Hkv, S) int32, distinct within each (b, h); an entry
+ *              outside [0, M) skips its row and records H2O_DEVERR_INDEX
+ *   k_new, v_new (B, Hkv, S, d) bf16 (replace)
+ *   k_cache, v_cache (B, Hkv, M, d) bf16, in place
+ *   slot_pos   (B, Hkv, M) int32 in place, or NULL (positions untouched)
+ *   delta_k, delta_v (B, Hkv, S, d) bf16: out of replace (both NULL: no
+ *              gather), in of restore; delta_pos (B, Hkv, S) int32 likewise
+ *              (NULL: positions are not saved / restored)
+ * dims->Hq only has to be a multiple of dims->Hkv.
+ */
+H2O_API int h2o_kv_replace(const h2o_dims_t* dims, int64_t pos0, const int32_t* index,
+                   const h2o_bf16* k_new, const h2o_bf16* v_new, h2o_bf16* k_cache,
+                   h2o_bf16* v_cache, int32_t* slot_pos, h2o_bf16* delta_k, h2o_bf16* delta_v,
+                   int32_t* delta_pos, void* stream);
+H2O_API int h2o_kv_restore(const h2o_dims_t* dims, const int32_t* index,
+                   const h2o_bf16* delta_k, const h2o_bf16* delta_v, const int32_t* delta_pos,
+                   h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t* slot_pos, void* stream);
 
 /* Empties a cache before a new sequence: slot_pos (B, Hkv, M) int32 := -1 and
  * scores (B, Hkv, M) f32 := 0, enqueued on `stream` (the K/V buffers need no

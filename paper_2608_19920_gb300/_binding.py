@@ -18,10 +18,12 @@ LIB_PATH = os.path.join(_PKG, "libh2o_gb300.so")
 H2O_OK = 0
 H2O_DEVERR_TIMEOUT = 1
 H2O_DEVERR_CANDIDATES = 2
+H2O_DEVERR_INDEX = 4
 
 # Every symbol include/h2o.h declares.
 EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
            "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
+           "h2o_kv_replace", "h2o_kv_restore",
            "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
            "h2o_version")
 
@@ -69,12 +71,14 @@ def load(path: str = LIB_PATH):
     lib.h2o_sdpa_cache.argtypes = [dims_p, i64, f32, vp, vp, vp, vp, vp, vp, vp, ctypes.c_size_t,
                                    vp]
     lib.h2o_scores_add.argtypes = [dims_p, vp, vp, vp]
+    lib.h2o_kv_replace.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.h2o_kv_restore.argtypes = [dims_p, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_status_string.argtypes = [ctypes.c_int]
     lib.h2o_status_string.restype = ctypes.c_char_p
     for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
                "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
-               "h2o_cache_reset",
+               "h2o_kv_replace", "h2o_kv_restore", "h2o_cache_reset",
                "h2o_last_cuda_error",
                "h2o_device_errors", "h2o_version"):
         getattr(lib, fn).restype = ctypes.c_int
@@ -319,6 +323,57 @@ def h2o_scores_add(scores, score_inc, stream=None):
     dims = H2ODims(B, Hq, Hkv, 64, 1, M)
     _check("h2o_scores_add", lib.h2o_scores_add(ctypes.byref(dims), _ptr(scores),
                                                 _ptr(score_inc), _stream(stream)))
+
+
+def h2o_kv_replace(index, k_new, v_new, k_cache, v_cache, pos0: int, slot_pos=None,
+                   delta_k=None, delta_v=None, delta_pos=None, stream=None):
+    """Replay-cache write (see include/h2o.h): the chunk's rows go to the slots
+    ``index`` (B,Hkv,S) int32, in place; the replaced rows / positions go to the
+    delta buffers when given.  Returns (delta_k, delta_v, delta_pos)."""
+    lib = load()
+    dev = k_cache.device
+    B, Hkv, M, d = k_cache.shape
+    S = index.shape[2]
+    bf = torch.bfloat16
+    _expect(index, "index", (B, Hkv, S), torch.int32, dev)
+    for t, n, shp in ((k_new, "k_new", (B, Hkv, S, d)), (v_new, "v_new", (B, Hkv, S, d)),
+                      (v_cache, "v_cache", (B, Hkv, M, d))):
+        _expect(t, n, shp, bf, dev)
+    if slot_pos is not None:
+        _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    if delta_k is not None or delta_v is not None:
+        _expect(delta_k, "delta_k", (B, Hkv, S, d), bf, dev)
+        _expect(delta_v, "delta_v", (B, Hkv, S, d), bf, dev)
+    if delta_pos is not None:
+        _expect(delta_pos, "delta_pos", (B, Hkv, S), torch.int32, dev)
+    dims = H2ODims(B, Hkv, Hkv, d, S, M)
+    _check("h2o_kv_replace", lib.h2o_kv_replace(
+        ctypes.byref(dims), int(pos0), _ptr(index), _ptr(k_new), _ptr(v_new), _ptr(k_cache),
+        _ptr(v_cache), _ptr(slot_pos), _ptr(delta_k), _ptr(delta_v), _ptr(delta_pos),
+        _stream(stream)))
+    return delta_k, delta_v, delta_pos
+
+
+def h2o_kv_restore(index, delta_k, delta_v, k_cache, v_cache, slot_pos=None, delta_pos=None,
+                   stream=None):
+    """The reverse recurrence: scatter the saved rows (and positions) back, in place."""
+    lib = load()
+    dev = k_cache.device
+    B, Hkv, M, d = k_cache.shape
+    S = index.shape[2]
+    bf = torch.bfloat16
+    _expect(index, "index", (B, Hkv, S), torch.int32, dev)
+    _expect(delta_k, "delta_k", (B, Hkv, S, d), bf, dev)
+    _expect(delta_v, "delta_v", (B, Hkv, S, d), bf, dev)
+    _expect(v_cache, "v_cache", (B, Hkv, M, d), bf, dev)
+    if slot_pos is not None:
+        _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    if delta_pos is not None:
+        _expect(delta_pos, "delta_pos", (B, Hkv, S), torch.int32, dev)
+    dims = H2ODims(B, Hkv, Hkv, d, S, M)
+    _check("h2o_kv_restore", lib.h2o_kv_restore(
+        ctypes.byref(dims), _ptr(index), _ptr(delta_k), _ptr(delta_v), _ptr(delta_pos),
+        _ptr(k_cache), _ptr(v_cache), _ptr(slot_pos), _stream(stream)))
 
 
 def h2o_cache_reset(slot_pos, scores, stream=None):

@@ -401,6 +401,61 @@ int h2o_scores_add(const h2o_dims_t* dims, float* scores, const float* score_inc
   return e == cudaSuccess ? H2O_OK : cuda_fail(e);
 }
 
+int h2o_kv_replace(const h2o_dims_t* dims, int64_t pos0, const int32_t* index,
+                   const h2o_bf16* k_new, const h2o_bf16* v_new, h2o_bf16* k_cache,
+                   h2o_bf16* v_cache, int32_t* slot_pos, h2o_bf16* delta_k, h2o_bf16* delta_v,
+                   int32_t* delta_pos, void* stream) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (D.M < 1 || D.S > D.M) return H2O_ERR_SHAPE;
+  if (!index || !k_new || !v_new || !k_cache || !v_cache) return H2O_ERR_NULL;
+  if ((delta_k == nullptr) != (delta_v == nullptr)) return H2O_ERR_NULL;
+  if (misaligned(index) || misaligned(k_new) || misaligned(v_new) || misaligned(k_cache) ||
+      misaligned(v_cache) || misaligned(slot_pos) || misaligned(delta_k) ||
+      misaligned(delta_v) || misaligned(delta_pos))
+    return H2O_ERR_ALIGN;
+  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  ReplayArgs a;
+  a.index = index; a.k_new = k_new; a.v_new = v_new; a.k_cache = k_cache; a.v_cache = v_cache;
+  a.slot_pos = slot_pos; a.delta_k = delta_k; a.delta_v = delta_v;
+  a.delta_pos = slot_pos ? delta_pos : nullptr;
+  a.err = di->err_word;
+  a.B = D.B; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M;
+  a.pos0 = static_cast<int>(pos0);
+  a.restore = 0;
+  const cudaError_t e = launch_kv_rows(a, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_kv_restore(const h2o_dims_t* dims, const int32_t* index, const h2o_bf16* delta_k,
+                   const h2o_bf16* delta_v, const int32_t* delta_pos, h2o_bf16* k_cache,
+                   h2o_bf16* v_cache, int32_t* slot_pos, void* stream) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (D.M < 1 || D.S > D.M) return H2O_ERR_SHAPE;
+  if (!index || !delta_k || !delta_v || !k_cache || !v_cache) return H2O_ERR_NULL;
+  if (misaligned(index) || misaligned(delta_k) || misaligned(delta_v) || misaligned(k_cache) ||
+      misaligned(v_cache) || misaligned(slot_pos) || misaligned(delta_pos))
+    return H2O_ERR_ALIGN;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  ReplayArgs a;
+  a.index = index; a.k_new = nullptr; a.v_new = nullptr; a.k_cache = k_cache;
+  a.v_cache = v_cache; a.slot_pos = slot_pos;
+  a.delta_k = const_cast<h2o_bf16*>(delta_k); a.delta_v = const_cast<h2o_bf16*>(delta_v);
+  a.delta_pos = const_cast<int32_t*>(delta_pos);
+  a.err = di->err_word;
+  a.B = D.B; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M;
+  a.pos0 = 0;
+  a.restore = 1;
+  const cudaError_t e = launch_kv_rows(a, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
 int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores, void* stream) {
   int st = check_dims(dims);
   if (st != H2O_OK) return st;

@@ -100,6 +100,24 @@ bool decode_plan(int B, int Hq, int Hkv, int d, int S, int M, int* split_len, in
 constexpr size_t kDecodeStaticScratchBytes = size_t(8) << 20;
 cudaError_t decode_static_scratch(void** ptr);
 
+// h2o_kv_replace / h2o_kv_restore (h2o_replay.cu)
+struct ReplayArgs {
+  const int32_t* index;      // (B, Hkv, S) slots, distinct per (b, h)
+  const uint16_t* k_new;     // (B, Hkv, S, d) replace only
+  const uint16_t* v_new;
+  uint16_t* k_cache;         // (B, Hkv, M, d) in/out
+  uint16_t* v_cache;
+  int32_t* slot_pos;         // (B, Hkv, M) in/out, may be null
+  uint16_t* delta_k;         // (B, Hkv, S, d): out (replace, may be null) or in (restore)
+  uint16_t* delta_v;
+  int32_t* delta_pos;        // (B, Hkv, S): likewise, may be null
+  int* err;
+  int B, Hkv, d, S, M;
+  int pos0;
+  int restore;               // 0: replace, 1: restore
+};
+
+cudaError_t launch_kv_rows(const ReplayArgs& a, cudaStream_t stream);
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);

@@ -157,3 +157,21 @@ def test_paper_order_argument_checks(lib):
     assert lib.h2o_scores_add(ctypes.byref(_dims(M=0)), p, p, None) == SHAPE
     assert lib.h2o_scores_add(ctypes.byref(d), vp(0), p, None) == NULL
     assert lib.h2o_scores_add(ctypes.byref(d), p, vp(0x1002), None) == ALIGN
+
+
+def test_replay_rows_argument_checks(lib):
+    """h2o_kv_replace / h2o_kv_restore refuse bad arguments on the host."""
+    vp = ctypes.c_void_p
+    p = vp(0x1000)
+    d = _dims()
+    rep = lambda dims, ptrs, pos0=256: lib.h2o_kv_replace(ctypes.byref(dims), pos0, *ptrs, None)
+    ok = [p] * 5 + [None, None, None, None]
+    assert rep(_dims(M=0, S=1), ok) == SHAPE
+    assert rep(_dims(S=300), ok) == SHAPE
+    assert rep(d, [vp(0)] + ok[1:]) == NULL
+    assert rep(d, [p] * 5 + [None, p, None, None]) == NULL   # delta_k without delta_v
+    assert rep(d, [p] * 4 + [vp(0x1008)] + [None] * 4) == ALIGN
+    assert rep(d, ok, pos0=-1) == ARG
+    res = lambda dims, ptrs: lib.h2o_kv_restore(ctypes.byref(dims), *ptrs, None)
+    assert res(d, [p, p, vp(0), None, p, p, None]) == NULL
+    assert res(d, [p, p, p, None, p, vp(0x100c), None]) == ALIGN

@@ -2,8 +2,9 @@
 from .h2o_oracle import (POLICIES, SequenceState, chunk_bounds, evict_insert, lse_merge,
                          run_sequence, scores_add, sdpa_cache, sdpa_chunk, step_paper_order,
                          update)
+from .backward import sdpa_chunk_backward
 from .replay import kv_replace, kv_restore
 
 __all__ = ["sdpa_chunk", "update", "run_sequence", "SequenceState", "lse_merge", "chunk_bounds",
            "POLICIES", "sdpa_cache", "evict_insert", "scores_add", "step_paper_order",
-           "kv_replace", "kv_restore"]
+           "kv_replace", "kv_restore", "sdpa_chunk_backward"]

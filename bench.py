@@ -566,8 +566,9 @@ def main():
     ap.add_argument("--traffic", type=float, default=None,
                     help="DRAM bytes per launch of the dominant kernel from an ncu capture")
     ap.add_argument("--ref-budget", type=float, default=20.0)
-    ap.add_argument("--mode", default="step", choices=["step", "kernel"],
-                    help="kernel: only repeat the steady-state chunk SDPA launch (for profiling)")
+    ap.add_argument("--mode", default="step", choices=["step", "kernel", "backward"],
+                    help="kernel: only repeat the steady-state chunk SDPA launch (for profiling); "
+                         "backward: time the gradient of that chunk (h2o_sdpa_chunk_backward)")
     ap.add_argument("--reps", type=int, default=5)
     args = ap.parse_args()
     if args.warmup < 3:
@@ -577,6 +578,8 @@ def main():
         return run_reference(args, w)
     if args.mode == "kernel":
         return run_kernel_only(args, w)
+    if args.mode == "backward":
+        return run_backward(args, w)
     return run_ours(args, w)
 
 
@@ -601,6 +604,69 @@ def run_kernel_only(args, w, n_fill: int = 8):
     torch.cuda.synchronize()
     assert h2o_device_errors() == 0
     print(json.dumps({"mode": "kernel", "workload": w.name, **kern}))
+    return 0
+
+
+def run_backward(args, w, n_fill: int = 8):
+    """Times h2o_sdpa_chunk_backward on the chunk after a prefill and ``n_fill``
+    chunks (the forward's inputs and output, an all-ones-scaled random dout),
+    L2 flushed before each launch, replayed from a CUDA graph."""
+    import torch
+    from paper_2608_19920_gb300 import (H2OLayer, build as build_mod, h2o_backward_workspace_size,
+                                       h2o_device_errors, h2o_sdpa_chunk, h2o_sdpa_chunk_backward)
+    from paper_2608_19920_gb300._binding import H2ODims
+    build_mod.build()
+    dev = torch.device("cuda", 0)
+    plan = step_plan(w)[:n_fill + 2]
+    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev)
+    ins = [tuple(torch.from_numpy(x).to(torch.bfloat16).to(dev) for x in wl.batch_tokens(w, p, e))
+           for p, e in plan]
+    layer.reset()
+    for (p, e), (q, k, v) in zip(plan[:-1], ins[:-1]):
+        layer.step(q, k, v, p)
+    p, e = plan[-1]
+    q, k, v = ins[-1]
+    S = e - p
+    out, _ = h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p)
+    dout = torch.randn(out.shape, device=dev, generator=torch.Generator(dev).manual_seed(0))
+    dout = dout.to(torch.bfloat16)
+    ws = torch.empty(h2o_backward_workspace_size(H2ODims(w.B, w.Hq, w.Hkv, w.d, S, w.M)),
+                     dtype=torch.uint8, device=dev)
+
+    def call():
+        h2o_sdpa_chunk_backward(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out,
+                                dout, workspace=ws)
+
+    call()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        call()
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    clean = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    times = []
+    for _ in range(args.reps + 2):
+        flush.zero_()
+        clean.sum()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        graph.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(b))
+    assert h2o_device_errors() == 0
+    avg_ms = sum(times[2:]) / len(times[2:])
+    # five contractions over the visible keys (Q K^T again, dout V^T, dS K,
+    # dS^T Q, P^T dout): 2.5 times the forward's algorithmic flops
+    flops = 2.5 * chunk_flops(w.B, w.Hq, w.d, S, w.M)
+    executed = 10.0 * w.B * w.Hq * S * w.d * (w.M + S)
+    pk = peaks()
+    tf = flops / (avg_ms / 1e3) / 1e12
+    print(json.dumps({"mode": "backward", "workload": w.name, "S": S, "avg_us": avg_ms * 1e3,
+                      "flops": flops, "alg_tflops": tf, "executed_tflops": executed / flops * tf,
+                      "frac_of_bf16_peak": tf / pk["bf16"], "workspace_bytes": ws.numel()}))
     return 0
 
 

@@ -69,7 +69,8 @@ enum {
   H2O_ERR_CUDA = -7,        /* a CUDA runtime call failed; see h2o_last_cuda_error */
   H2O_ERR_TIMEOUT = -8,     /* device: a bounded wait ran out (reported by h2o_device_errors) */
   H2O_ERR_DEVICE = -9,      /* device: fewer eviction candidates than S, etc. */
-  H2O_ERR_NODEVICE = -10    /* no usable sm_100-family GPU is current */
+  H2O_ERR_NODEVICE = -10,   /* no usable sm_100-family GPU is current */
+  H2O_ERR_BLAS = -11        /* a cuBLASLt call failed; its cublasStatus_t in h2o_last_cuda_error */
 };
 
 /* Device error bits reported by h2o_device_errors(). */
@@ -261,6 +262,40 @@ H2O_API int h2o_kv_replace(const h2o_dims_t* dims, int64_t pos0, const int32_t* 
 H2O_API int h2o_kv_restore(const h2o_dims_t* dims, const int32_t* index,
                    const h2o_bf16* delta_k, const h2o_bf16* delta_v, const int32_t* delta_pos,
                    h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t* slot_pos, void* stream);
+
+/*
+ * Gradient of one chunk of h2o_sdpa_chunk (§3.1 Eq. 2 with the mask of
+ * §3.3.1), for the loss sum(out * dout): the backward pass the paper's
+ * fine-tuning runs through every chunk (§3.2; the KV cache policy itself is not
+ * differentiated).  Per (b, kv head) the probabilities are recomputed from q
+ * and the keys; with D_i = dout_i . out_i and dS = P * (dout V^T - D):
+ *
+ *   dq = scale dS K,   d[k_cache; k_new] = scale dS^T Q,   d[v_cache; v_new] = P^T dout
+ *
+ * summed over the q_g query heads of the group for the keys and values.
+ *
+ *   q, k_cache, v_cache, k_new, v_new, slot_pos, pos0, softmax_scale: as for
+ *              h2o_sdpa_chunk (the same call's inputs)
+ *   out        (B, Hq, S, d) bf16, the output h2o_sdpa_chunk returned
+ *   dout       (B, Hq, S, d) bf16, gradient of the loss w.r.t. out
+ *   dq         (B, Hq, S, d) f32, written
+ *   dk_cache, dv_cache (B, Hkv, M, d) f32, written (may be NULL when M == 0)
+ *   dk_new, dv_new     (B, Hkv, S, d) f32, written
+ *   workspace  at least h2o_backward_workspace_size(dims) bytes: 32 MiB for
+ *              cuBLASLt plus the materialised (B Hkv) x (q_g S) x (M + S)
+ *              score matrices (fp32 scores, bf16 P and dS)
+ *
+ * The five contractions run on cuBLASLt (bf16 operands, fp32 accumulation);
+ * a failure there returns H2O_ERR_BLAS.  Cache slots no row sees get zero
+ * gradient.
+ */
+H2O_API int h2o_backward_workspace_size(const h2o_dims_t* dims, size_t* bytes);
+H2O_API int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                   const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
+                   const h2o_bf16* out, const h2o_bf16* dout, float* dq, float* dk_cache,
+                   float* dv_cache, float* dk_new, float* dv_new, void* workspace,
+                   size_t workspace_bytes, void* stream);
 
 /* Empties a cache before a new sequence: slot_pos (B, Hkv, M) int32 := -1 and
  * scores (B, Hkv, M) f32 := 0, enqueued on `stream` (the K/V buffers need no

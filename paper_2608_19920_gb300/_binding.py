@@ -23,7 +23,8 @@ H2O_DEVERR_INDEX = 4
 # Every symbol include/h2o.h declares.
 EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
            "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
-           "h2o_kv_replace", "h2o_kv_restore",
+           "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
+           "h2o_sdpa_chunk_backward",
            "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
            "h2o_version")
 
@@ -73,12 +74,15 @@ def load(path: str = LIB_PATH):
     lib.h2o_scores_add.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_kv_replace.argtypes = [dims_p, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.h2o_kv_restore.argtypes = [dims_p, vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.h2o_backward_workspace_size.argtypes = [dims_p, ctypes.POINTER(ctypes.c_size_t)]
+    lib.h2o_sdpa_chunk_backward.argtypes = [dims_p, i64, f32] + [vp] * 14 + [ctypes.c_size_t, vp]
     lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_status_string.argtypes = [ctypes.c_int]
     lib.h2o_status_string.restype = ctypes.c_char_p
     for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
                "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
-               "h2o_kv_replace", "h2o_kv_restore", "h2o_cache_reset",
+               "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
+               "h2o_sdpa_chunk_backward", "h2o_cache_reset",
                "h2o_last_cuda_error",
                "h2o_device_errors", "h2o_version"):
         getattr(lib, fn).restype = ctypes.c_int
@@ -374,6 +378,48 @@ def h2o_kv_restore(index, delta_k, delta_v, k_cache, v_cache, slot_pos=None, del
     _check("h2o_kv_restore", lib.h2o_kv_restore(
         ctypes.byref(dims), _ptr(index), _ptr(delta_k), _ptr(delta_v), _ptr(delta_pos),
         _ptr(k_cache), _ptr(v_cache), _ptr(slot_pos), _stream(stream)))
+
+
+def h2o_backward_workspace_size(dims: H2ODims) -> int:
+    lib = load()
+    n = ctypes.c_size_t(0)
+    _check("h2o_backward_workspace_size",
+           lib.h2o_backward_workspace_size(ctypes.byref(dims), ctypes.byref(n)))
+    return n.value
+
+
+def h2o_sdpa_chunk_backward(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, out, dout,
+                            scale: float = 0.0, workspace=None, stream=None):
+    """Gradient of sum(out * dout) for one h2o_sdpa_chunk call (see include/h2o.h).
+    Returns fp32 (dq, dk_cache, dv_cache, dk_new, dv_new)."""
+    lib = load()
+    dev = q.device
+    B, Hq, S, d = q.shape
+    Hkv, M = k_new.shape[1], k_cache.shape[2]
+    bf = torch.bfloat16
+    for t, n, shp, dt in ((q, "q", (B, Hq, S, d), bf), (k_cache, "k_cache", (B, Hkv, M, d), bf),
+                          (v_cache, "v_cache", (B, Hkv, M, d), bf),
+                          (k_new, "k_new", (B, Hkv, S, d), bf), (v_new, "v_new", (B, Hkv, S, d), bf),
+                          (slot_pos, "slot_pos", (B, Hkv, M), torch.int32),
+                          (out, "out", (B, Hq, S, d), bf), (dout, "dout", (B, Hq, S, d), bf)):
+        _expect(t, n, shp, dt, dev)
+    f32 = torch.float32
+    dq = torch.empty((B, Hq, S, d), dtype=f32, device=dev)
+    dkc = torch.empty((B, Hkv, M, d), dtype=f32, device=dev)
+    dvc = torch.empty_like(dkc)
+    dkn = torch.empty((B, Hkv, S, d), dtype=f32, device=dev)
+    dvn = torch.empty_like(dkn)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    if workspace is None:
+        workspace = torch.empty(h2o_backward_workspace_size(dims), dtype=torch.uint8, device=dev)
+    ws_bytes = workspace.numel() * workspace.element_size()
+    st = lib.h2o_sdpa_chunk_backward(
+        ctypes.byref(dims), int(pos0), float(scale), _ptr(q), _ptr(k_cache), _ptr(v_cache),
+        _ptr(k_new), _ptr(v_new), _ptr(slot_pos), _ptr(out), _ptr(dout), _ptr(dq),
+        _ptr(dkc if M else None), _ptr(dvc if M else None), _ptr(dkn), _ptr(dvn),
+        _ptr(workspace), ws_bytes, _stream(stream))
+    _check("h2o_sdpa_chunk_backward", st)
+    return dq, dkc, dvc, dkn, dvn
 
 
 def h2o_cache_reset(slot_pos, scores, stream=None):

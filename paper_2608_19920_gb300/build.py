@@ -18,7 +18,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libh2o_gb300.so")
-SOURCES = ["h2o_api.cu", "h2o_sdpa.cu", "h2o_decode.cu", "h2o_update.cu", "h2o_replay.cu"]
+SOURCES = ["h2o_api.cu", "h2o_sdpa.cu", "h2o_decode.cu", "h2o_update.cu", "h2o_replay.cu",
+           "h2o_backward.cu"]
 HEADERS = ["h2o_internal.h", "sm100.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden",
@@ -65,7 +66,9 @@ def build(force: bool = False, verbose: bool = False) -> str:
     with open(os.path.join(BUILD, "ptxas.log"), "w") as f:
         f.write("\n".join(log))
     tmp = LIB + ".tmp"
-    cmd = [cc, *ARCH, "-shared", "-o", tmp, *[o for _, o, _ in results]]
+    cuda_lib = os.path.join(os.path.dirname(os.path.dirname(cc)), "lib64")
+    cmd = [cc, *ARCH, "-shared", "-o", tmp, *[o for _, o, _ in results], "-lcublasLt",
+           "-Xlinker", f"-rpath={cuda_lib}"]
     p = subprocess.run(cmd, capture_output=True, text=True)
     if p.returncode != 0:
         raise RuntimeError(f"link failed:\n{p.stdout}{p.stderr}")

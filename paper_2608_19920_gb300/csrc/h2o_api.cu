@@ -281,6 +281,7 @@ const char* h2o_status_string(int s) {
     case H2O_ERR_TIMEOUT: return "a device-side bounded wait ran out";
     case H2O_ERR_DEVICE: return "device-side error (fewer eviction candidates than S)";
     case H2O_ERR_NODEVICE: return "no usable sm_100-family GPU is current";
+    case H2O_ERR_BLAS: return "a cuBLASLt call failed (status in h2o_last_cuda_error)";
     default: return "unknown status";
   }
 }
@@ -454,6 +455,56 @@ int h2o_kv_restore(const h2o_dims_t* dims, const int32_t* index, const h2o_bf16*
   a.restore = 1;
   const cudaError_t e = launch_kv_rows(a, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_backward_workspace_size(const h2o_dims_t* dims, size_t* bytes) {
+  const int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  if (!bytes) return H2O_ERR_NULL;
+  *bytes = backward_workspace_bytes(dims->B, dims->Hq, dims->Hkv, dims->S, dims->M);
+  return H2O_OK;
+}
+
+int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                            const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                            const h2o_bf16* k_new, const h2o_bf16* v_new,
+                            const int32_t* slot_pos, const h2o_bf16* out,
+                            const h2o_bf16* dout, float* dq, float* dk_cache, float* dv_cache,
+                            float* dk_new, float* dv_new, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (!q || !k_new || !v_new || !out || !dout || !dq || !dk_new || !dv_new) return H2O_ERR_NULL;
+  if (D.M > 0 && (!k_cache || !v_cache || !slot_pos || !dk_cache || !dv_cache))
+    return H2O_ERR_NULL;
+  if (misaligned(q) || misaligned(k_cache) || misaligned(v_cache) || misaligned(k_new) ||
+      misaligned(v_new) || misaligned(slot_pos) || misaligned(out) || misaligned(dout) ||
+      misaligned(dq) || misaligned(dk_cache) || misaligned(dv_cache) || misaligned(dk_new) ||
+      misaligned(dv_new) || misaligned(workspace))
+    return H2O_ERR_ALIGN;
+  if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
+  if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
+  if (!workspace || workspace_bytes < backward_workspace_bytes(D.B, D.Hq, D.Hkv, D.S, D.M))
+    return H2O_ERR_WORKSPACE;
+  DeviceInfo* di = nullptr;
+  if ((st = current_device(&di)) != H2O_OK) return st;
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
+  BackwardArgs a = {};
+  a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
+  a.slot_pos = slot_pos; a.out = out; a.dout = dout;
+  a.dq = dq; a.dk_cache = dk_cache; a.dv_cache = dv_cache; a.dk_new = dk_new; a.dv_new = dv_new;
+  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = D.Hq / D.Hkv;
+  a.pos0 = static_cast<int>(pos0);
+  a.scale = scale;
+  a.scale_log2 = scale * 1.4426950408889634f;
+  const BackwardStatus bs = launch_backward(a, workspace, static_cast<cudaStream_t>(stream));
+  if (bs.cuda != cudaSuccess) return cuda_fail(bs.cuda);
+  if (bs.blas != 0) {
+    t_last_cuda_error = bs.blas;
+    return H2O_ERR_BLAS;
+  }
+  return H2O_OK;
 }
 
 int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores, void* stream) {

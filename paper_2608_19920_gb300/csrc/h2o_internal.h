@@ -118,6 +118,37 @@ struct ReplayArgs {
 };
 
 cudaError_t launch_kv_rows(const ReplayArgs& a, cudaStream_t stream);
+
+// h2o_sdpa_chunk_backward (h2o_backward.cu)
+struct BackwardArgs {
+  const uint16_t* q;         // (B, Hq, S, d) bf16
+  const uint16_t* k_cache;   // (B, Hkv, M, d)
+  const uint16_t* v_cache;
+  const uint16_t* k_new;     // (B, Hkv, S, d)
+  const uint16_t* v_new;
+  const int32_t* slot_pos;   // (B, Hkv, M)
+  const uint16_t* out;       // (B, Hq, S, d) forward output
+  const uint16_t* dout;      // (B, Hq, S, d) gradient of the loss w.r.t. out
+  float* dq;                 // (B, Hq, S, d) fp32
+  float* dk_cache;           // (B, Hkv, M, d) fp32
+  float* dv_cache;
+  float* dk_new;             // (B, Hkv, S, d) fp32
+  float* dv_new;
+  float* sbuf;               // workspace: S, then dP (groups x R x (M + S)) fp32
+  uint16_t* pbuf;            // P, bf16
+  uint16_t* dsbuf;           // dS, bf16
+  float* drow;               // D per stacked row
+  int B, Hq, Hkv, d, S, M, qg;
+  int pos0;
+  float scale;               // softmax scale
+  float scale_log2;          // scale * log2(e)
+};
+struct BackwardStatus {
+  cudaError_t cuda = cudaSuccess;
+  int blas = 0;              // cublasStatus_t, 0 = success
+};
+size_t backward_workspace_bytes(int B, int Hq, int Hkv, int S, int M);
+BackwardStatus launch_backward(BackwardArgs a, void* workspace, cudaStream_t stream);
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);

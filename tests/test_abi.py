@@ -175,3 +175,26 @@ def test_replay_rows_argument_checks(lib):
     res = lambda dims, ptrs: lib.h2o_kv_restore(ctypes.byref(dims), *ptrs, None)
     assert res(d, [p, p, vp(0), None, p, p, None]) == NULL
     assert res(d, [p, p, p, None, p, vp(0x100c), None]) == ALIGN
+
+
+def test_backward_argument_checks(lib):
+    """h2o_sdpa_chunk_backward refuses bad arguments on the host (through the
+    binding's declared argument types)."""
+    vp = ctypes.c_void_p
+    p = vp(0x1000)
+    d = _dims()
+    n = ctypes.c_size_t(0)
+    assert lib.h2o_backward_workspace_size(ctypes.byref(d), ctypes.byref(n)) == OK
+    G, R, NK = 2, 2 * 32, 256 + 32
+    cells = G * R * NK
+    a256 = lambda x: (x + 255) // 256 * 256
+    assert n.value == (32 << 20) + a256(cells * 4) + 2 * a256(cells * 2) + a256(G * R * 4)
+    bwd = lambda dims, ptrs, ws=p, wsb=n.value, pos0=256: lib.h2o_sdpa_chunk_backward(
+        ctypes.byref(dims), pos0, 0.0, *ptrs, ws, wsb, None)
+    ok = [p] * 13
+    assert bwd(d, ok, ws=None) == WORKSPACE
+    assert bwd(d, ok, wsb=n.value - 1) == WORKSPACE
+    assert bwd(d, [vp(0)] + ok[1:]) == NULL
+    assert bwd(d, ok[:8] + [vp(0x1004)] + ok[9:]) == ALIGN
+    assert bwd(d, ok, pos0=-1) == ARG
+    assert bwd(_dims(d=96), ok) == UNSUP

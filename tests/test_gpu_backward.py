@@ -1,0 +1,73 @@
+"""GPU parity of the chunk-SDPA gradient (h2o_sdpa_chunk_backward) against the
+float64 oracle, through the C ABI.
+
+Tolerance (derived from the arithmetic): the kernel rounds P and dS to bf16
+(relative 2^-9 each) before the fp32-accumulated contractions, and uses the
+bf16 forward output in D = dout . out; each gradient tensor must lie within
+1e-2 of its own max-abs value elementwise.  Slots no row sees get exactly 0."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import sdpa_chunk_backward as ref_backward
+from paper_2608_19920_gb300 import (build, h2o_device_errors, h2o_sdpa_chunk,
+                                   h2o_sdpa_chunk_backward)
+from paper_2608_19920_gb300 import workloads as wl
+
+from test_gpu_parity import bf, f32
+
+pytestmark = pytest.mark.gpu
+
+GRAD_RTOL = 1e-2
+
+
+@pytest.fixture(scope="module")
+def dev():
+    build.build()
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    return torch.device("cuda:0")
+
+
+CASES = [
+    # B, Hq, Hkv, d, S, M, n_empty, n_future, pos0
+    (1, 4, 2, 64, 32, 256, 0, 0, 256),       # the tiny workload's chunk shape
+    (2, 8, 2, 128, 20, 300, 17, 5, 900),     # ragged S and M, empty and future slots
+    (3, 6, 3, 64, 1, 130, 5, 0, 140),        # one token
+    (1, 4, 4, 128, 200, 0, 0, 0, 0),         # no cache (a prefill)
+    (1, 32, 8, 128, 512, 4096, 0, 0, 8192),  # the Llama-3-8B-shaped chunk
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: "x".join(map(str, c)))
+def test_backward_matches_oracle(dev, case):
+    B, Hq, Hkv, d, S, M, n_empty, n_future, pos0 = case
+    rng = np.random.default_rng(hash(case) % 2**32)
+    st = wl.random_state(rng, B, Hkv, M, d, pos0=pos0, n_empty=n_empty)
+    for b in range(B):
+        for h in range(Hkv):
+            occ = np.nonzero(st["slot_pos"][b, h] >= 0)[0]
+            for k in range(min(n_future, len(occ))):
+                st["slot_pos"][b, h, occ[k]] = pos0 + (k % S)
+    q = wl.round_bf16(rng.standard_normal((B, Hq, S, d), dtype=np.float32))
+    kn = wl.round_bf16(rng.standard_normal((B, Hkv, S, d), dtype=np.float32))
+    vn = wl.round_bf16(rng.standard_normal((B, Hkv, S, d), dtype=np.float32))
+    dout = wl.round_bf16(rng.standard_normal((B, Hq, S, d), dtype=np.float32))
+    g = dict(q=bf(q, dev), kc=bf(st["k_cache"], dev), vc=bf(st["v_cache"], dev), kn=bf(kn, dev),
+             vn=bf(vn, dev), sp=torch.from_numpy(st["slot_pos"]).to(dev))
+    out, _ = h2o_sdpa_chunk(g["q"], g["kc"], g["vc"], g["kn"], g["vn"], g["sp"], pos0)
+    grads = h2o_sdpa_chunk_backward(g["q"], g["kc"], g["vc"], g["kn"], g["vn"], g["sp"], pos0, out,
+                                    bf(dout, dev))
+    torch.cuda.synchronize()
+    assert h2o_device_errors() == 0
+    refs = ref_backward(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"], pos0, dout)
+    for name, gpu, ref in zip(("dq", "dk_cache", "dv_cache", "dk_new", "dv_new"), grads, refs):
+        if ref.size == 0:
+            continue
+        x = gpu.cpu().numpy().astype(np.float64)
+        scale = np.abs(ref).max()
+        err = np.abs(x - ref).max()
+        assert err <= GRAD_RTOL * scale + 1e-6, f"{name}: max err {err:.3e} vs max {scale:.3e}"
+    if M:
+        hidden = (st["slot_pos"] < 0) | (st["slot_pos"] > pos0 + S - 1)
+        assert (grads[1].cpu().numpy()[hidden] == 0).all()
+        assert (grads[2].cpu().numpy()[hidden] == 0).all()

@@ -16,9 +16,23 @@
  *                   recent window and writes the chunk's keys and values into
  *                   them (the scatter of §3.2 / §A.1.1).
  *
+ * With one query token per sequence (S = 1) h2o_sdpa_chunk runs split-K decode
+ * kernels that need a workspace (h2o_workspace_size).  Further calls:
+ *   h2o_update_policy                the h2o_norm / h2o_orig variants (§3.1.1)
+ *   h2o_evict_insert, h2o_sdpa_cache, h2o_scores_add
+ *                                    the paper's own order of a chunk step
+ *                                    (write first, then attend; §3.1, §3.3.1)
+ *   h2o_kv_replace, h2o_kv_restore   replay-cache row writes and the reverse
+ *                                    recurrence (§3.2, §A.1.1)
+ *   h2o_sdpa_chunk_backward          the gradient of one chunk's SDPA
+ *   h2o_sdpa_decode_static           S = 1 SDPA on a fixed internal scratch
+ *
  * Conventions for every call:
  *  - All array arguments are DEVICE pointers, allocated and owned by the
- *    caller; the library allocates no memory and keeps no per-call state.
+ *    caller; the library allocates no device memory of its own (the scratch
+ *    of h2o_sdpa_decode_static and the error word are static device arrays;
+ *    h2o_sdpa_chunk_backward uses cuBLASLt in the caller's workspace) and
+ *    keeps no per-call state.
  *    Every array is dense, row-major (C order) with the shape given, and must
  *    be 16-byte aligned.
  *  - bf16 arrays hold IEEE bfloat16 bit patterns (h2o_bf16 = uint16_t).

@@ -329,6 +329,13 @@ H2O_API int h2o_last_cuda_error(void);
  * failure. */
 H2O_API int h2o_device_errors(void);
 
+/* Self-test of device-side failure detection (no paper counterpart): one
+ * small kernel waits on a barrier that nothing completes, with the same
+ * bounded wait every kernel of the library uses, gives up after limit_ns
+ * (1 us .. 100 ms, else H2O_ERR_ARG) and records H2O_DEVERR_TIMEOUT, which
+ * h2o_device_errors() then reports.  The context stays usable. */
+H2O_API int h2o_selftest_bounded_wait(int64_t limit_ns, void* stream);
+
 /* Library version as major*10000 + minor*100 + patch. */
 H2O_API int h2o_version(void);
 

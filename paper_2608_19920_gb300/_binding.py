@@ -24,7 +24,7 @@ H2O_DEVERR_INDEX = 4
 EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
            "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
            "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
-           "h2o_sdpa_chunk_backward",
+           "h2o_sdpa_chunk_backward", "h2o_selftest_bounded_wait",
            "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
            "h2o_version")
 
@@ -76,13 +76,14 @@ def load(path: str = LIB_PATH):
     lib.h2o_kv_restore.argtypes = [dims_p, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.h2o_backward_workspace_size.argtypes = [dims_p, ctypes.POINTER(ctypes.c_size_t)]
     lib.h2o_sdpa_chunk_backward.argtypes = [dims_p, i64, f32] + [vp] * 14 + [ctypes.c_size_t, vp]
+    lib.h2o_selftest_bounded_wait.argtypes = [i64, vp]
     lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_status_string.argtypes = [ctypes.c_int]
     lib.h2o_status_string.restype = ctypes.c_char_p
     for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
                "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
                "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
-               "h2o_sdpa_chunk_backward", "h2o_cache_reset",
+               "h2o_sdpa_chunk_backward", "h2o_selftest_bounded_wait", "h2o_cache_reset",
                "h2o_last_cuda_error",
                "h2o_device_errors", "h2o_version"):
         getattr(lib, fn).restype = ctypes.c_int
@@ -431,6 +432,12 @@ def h2o_cache_reset(slot_pos, scores, stream=None):
     dims = H2ODims(B, Hkv, Hkv, 64, 1, M)
     _check("h2o_cache_reset", lib.h2o_cache_reset(ctypes.byref(dims), _ptr(slot_pos),
                                                   _ptr(scores), _stream(stream)))
+
+
+def h2o_selftest_bounded_wait(limit_ns: int = 5_000_000, stream=None):
+    """Runs the device-side bounded-wait self-test (see include/h2o.h)."""
+    _check("h2o_selftest_bounded_wait",
+           load().h2o_selftest_bounded_wait(int(limit_ns), _stream(stream)))
 
 
 def h2o_device_errors() -> int:

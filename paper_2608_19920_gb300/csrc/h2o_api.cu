@@ -11,6 +11,7 @@
 
 #include "../../include/h2o.h"
 #include "h2o_internal.h"
+#include "sm100.cuh"
 
 namespace h2o {
 
@@ -257,6 +258,22 @@ int update_impl(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* sl
   const cudaError_t e = launch_update(a, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e);
   return H2O_OK;
+}
+
+// Waits on an mbarrier nothing completes, with the bounded wait every kernel
+// uses; when the limit runs out it records H2O_DEVERR_TIMEOUT and returns.
+__global__ void selftest_wait_kernel(int* err, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    bar_init(&bar, 1);  // one arrival expected; none ever comes
+    abort_flag = 0;
+    fence_bar_init();
+  }
+  __syncthreads();
+  const bool ok = wait_bar(&bar, 0, &abort_flag, limit_ns);
+  __syncthreads();
+  if (threadIdx.x == 0 && !ok) atomicOr(err, H2O_DEVERR_TIMEOUT);
 }
 
 }  // namespace
@@ -519,6 +536,17 @@ int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores, vo
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(slot_pos, 0xFF, n * sizeof(int32_t), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(scores, 0, n * sizeof(float), s);
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_selftest_bounded_wait(int64_t limit_ns, void* stream) {
+  if (limit_ns < 1000 || limit_ns > 100000000) return H2O_ERR_ARG;  // 1 us .. 100 ms
+  DeviceInfo* di = nullptr;
+  const int st = current_device(&di);
+  if (st != H2O_OK) return st;
+  selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(
+      di->err_word, static_cast<uint64_t>(limit_ns));
+  const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? H2O_OK : cuda_fail(e);
 }
 

@@ -198,3 +198,8 @@ def test_backward_argument_checks(lib):
     assert bwd(d, ok[:8] + [vp(0x1004)] + ok[9:]) == ALIGN
     assert bwd(d, ok, pos0=-1) == ARG
     assert bwd(_dims(d=96), ok) == UNSUP
+
+
+def test_selftest_limit_is_checked_on_the_host(lib):
+    assert lib.h2o_selftest_bounded_wait(10, None) == ARG          # below 1 us
+    assert lib.h2o_selftest_bounded_wait(10 ** 9, None) == ARG     # above 100 ms

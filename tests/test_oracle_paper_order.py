@@ -4,7 +4,7 @@ freed slots, run SDPA over the M cache slots under the position mask, then add
 the chunk's summed weights to the scores (Eq. 3).
 
 Each check ties the oracle to something other than itself: dense causal
-attention, the independently pinned the benchmark spec-order oracle where no eviction
+attention, the independently pinned default-order oracle (attend, then evict) where no eviction
 happens, closed forms, invariants and brute-force enumeration.
 """
 import itertools
@@ -101,7 +101,7 @@ def test_rows_sum_to_one_and_hidden_slots_get_nothing():
 
 def test_evicted_tokens_do_not_influence_the_chunk():
     """The chunk attends after the eviction: the evicted slots' old K/V cannot
-    change its output (unlike the benchmark spec order, where they are visible)."""
+    change its output (unlike the default order, where they are visible)."""
     rng = np.random.default_rng(6)
     B, Hq, Hkv, M, d, S, pos0 = 1, 4, 2, 24, 8, 5, 80
     st = wl.random_state(rng, B, Hkv, M, d, pos0=pos0)
@@ -116,7 +116,7 @@ def test_evicted_tokens_do_not_influence_the_chunk():
                 v2[b, h, e] = -5.0
     o2, _, _ = step_paper_order(st["scores"], st["slot_pos"], k2, v2, q, kn, vn, pos0, 0)
     np.testing.assert_array_equal(o1, o2)
-    # the benchmark spec order does see them
+    # the default order (attend, then evict) does see them
     a1, _, _ = sdpa_chunk(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"], pos0)
     a2, _, _ = sdpa_chunk(q, k2, v2, kn, vn, st["slot_pos"], pos0)
     assert not np.allclose(a1, a2)

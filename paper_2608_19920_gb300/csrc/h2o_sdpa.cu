@@ -613,72 +613,75 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       const bool partial = (e & kTilePartial) != 0;
       const uint32_t s_base = tS + lane_addr + buf * 128 + u * 64;
       if (!pass2) {
-        // pass 1 (one row per thread, 64 columns): running max and sum of exp2
-        const int col0 = (e & kTileIdxMask) * kTileN + u * 64;
-        float v[64];
-        {
-          uint32_t r[32];
-          tmem_ld32_async(s_base, r);
-          tmem_wait_ld(r);
+        // pass 1 (one row per thread, 64 columns in two halves of 32): running
+        // max and sum of exp2, updated after each half, so that only 32 values
+        // are live; the S buffer is released once both halves are loaded
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          const int col0 = (e & kTileIdxMask) * kTileN + u * 64 + 32 * h;
+          float v[32];
+          {
+            uint32_t r[32];
+            tmem_ld32_async(s_base + 32 * h, r);
+            tmem_wait_ld(r);
 #pragma unroll
-          for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
-          tmem_ld32_async(s_base + 32, r);
-          tmem_wait_ld(r);
-#pragma unroll
-          for (int k = 0; k < 32; ++k) v[32 + k] = __uint_as_float(r[k]);
-        }
-        tc_fence_before_sync();
-        __syncwarp();
-        if (lane == 0) arrive_issuer<kPair>(&sm.bar_sread[buf]);  // S buffer may be overwritten
-        if (!partial) {
-          float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
-#pragma unroll
-          for (int k = 4; k < 64; k += 4) {
-            mx0 = fmaxf(mx0, v[k]);
-            mx1 = fmaxf(mx1, v[k + 1]);
-            mx2 = fmaxf(mx2, v[k + 2]);
-            mx3 = fmaxf(mx3, v[k + 3]);
+            for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
           }
-          const float m_new = fmaxf(m_run, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2);
-          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-          for (int k = 0; k < 64; k += 4) {
-            s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
-            s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
-            s2 += fast_exp2(fmaf(v[k + 2], sl2, -m_new));
-            s3 += fast_exp2(fmaf(v[k + 3], sl2, -m_new));
+          if (h == 1) {
+            tc_fence_before_sync();
+            __syncwarp();
+            if (lane == 0) arrive_issuer<kPair>(&sm.bar_sread[buf]);  // S buffer may be overwritten
           }
-          l_run = l_run * fast_exp2(m_run - m_new) + ((s0 + s1) + (s2 + s3));
-          m_run = m_new;
-        } else {
-          uint64_t vis = 0ull;  // bit k: column col0 + k visible to this row
-          if (valid) {
-            if (chunk) {
+          if (!partial) {
+            float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
 #pragma unroll
-              for (int k = 0; k < 64; ++k)
-                if (col0 + k <= i && col0 + k < a.S) vis |= 1ull << k;
-            } else {
-              for (int k = 0; k < 64; ++k) {
-                const int j = col0 + k;
-                const int pos = j < a.M ? __ldg(sp_base + j) : -1;
-                if (pos >= 0 && pos <= qpos) vis |= 1ull << k;
+            for (int k = 4; k < 32; k += 4) {
+              mx0 = fmaxf(mx0, v[k]);
+              mx1 = fmaxf(mx1, v[k + 1]);
+              mx2 = fmaxf(mx2, v[k + 2]);
+              mx3 = fmaxf(mx3, v[k + 3]);
+            }
+            const float m_new = fmaxf(m_run, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2);
+            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+            for (int k = 0; k < 32; k += 4) {
+              s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
+              s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
+              s2 += fast_exp2(fmaf(v[k + 2], sl2, -m_new));
+              s3 += fast_exp2(fmaf(v[k + 3], sl2, -m_new));
+            }
+            l_run = l_run * fast_exp2(m_run - m_new) + ((s0 + s1) + (s2 + s3));
+            m_run = m_new;
+          } else {
+            uint32_t vis = 0u;  // bit k: column col0 + k visible to this row
+            if (valid) {
+              if (chunk) {
+#pragma unroll
+                for (int k = 0; k < 32; ++k)
+                  if (col0 + k <= i && col0 + k < a.S) vis |= 1u << k;
+              } else {
+                for (int k = 0; k < 32; ++k) {
+                  const int j = col0 + k;
+                  const int pos = j < a.M ? __ldg(sp_base + j) : -1;
+                  if (pos >= 0 && pos <= qpos) vis |= 1u << k;
+                }
               }
             }
-          }
-          float mx = -INFINITY;
+            float mx = -INFINITY;
 #pragma unroll
-          for (int k = 0; k < 64; ++k)
-            if ((vis >> k) & 1ull) mx = fmaxf(mx, v[k] * sl2);
-          const float m_new = fmaxf(m_run, mx);
-          if (m_new > -INFINITY) {
-            float s0 = 0.f, s1 = 0.f;
+            for (int k = 0; k < 32; ++k)
+              if ((vis >> k) & 1u) mx = fmaxf(mx, v[k] * sl2);
+            const float m_new = fmaxf(m_run, mx);
+            if (m_new > -INFINITY) {
+              float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-            for (int k = 0; k < 64; k += 2) {
-              if ((vis >> k) & 1ull) s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
-              if ((vis >> (k + 1)) & 1ull) s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
+              for (int k = 0; k < 32; k += 2) {
+                if ((vis >> k) & 1u) s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
+                if ((vis >> (k + 1)) & 1u) s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
+              }
+              l_run = l_run * fast_exp2(m_run - m_new) + (s0 + s1);
+              m_run = m_new;
             }
-            l_run = l_run * fast_exp2(m_run - m_new) + (s0 + s1);
-            m_run = m_new;
           }
         }
       } else {

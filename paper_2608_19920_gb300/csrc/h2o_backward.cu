@@ -114,6 +114,158 @@ __global__ void __launch_bounds__(kRowThreads) bwd_ds_kernel(const BackwardArgs 
   }
 }
 
+// ---- vectorised forms: N_k and M multiples of 4, 16-byte aligned buffers ----
+// A row of N_k fp32 scores is then a run of float4s, and no group of four
+// columns straddles the cache / chunk boundary.  Each thread keeps four 16-byte
+// loads in flight: one 4-byte load per thread (the scalar kernels above) holds
+// too few bytes in flight per SM to cover the HBM latency.
+constexpr int kVecUnroll = 4;
+
+// Visibility of columns 4v .. 4v+3 of row (query i, position qpos) as a 4-bit
+// mask: cache slots by their positions p (§3.3.1), chunk columns causally.
+__device__ __forceinline__ unsigned vis_mask4(int v, int mv, int4 p, int qpos, int i, int M) {
+  if (v < mv)
+    return static_cast<unsigned>(p.x >= 0 && p.x <= qpos) |
+           static_cast<unsigned>(p.y >= 0 && p.y <= qpos) << 1 |
+           static_cast<unsigned>(p.z >= 0 && p.z <= qpos) << 2 |
+           static_cast<unsigned>(p.w >= 0 && p.w <= qpos) << 3;
+  const int n = i - (4 * v - M) + 1;  // chunk columns t .. t+3 visible while t <= i
+  return n <= 0 ? 0u : n >= 4 ? 15u : (1u << n) - 1u;
+}
+
+// (m, l) <- the pair whose sum of 2^(y - m) covers both sets: the online
+// softmax merge; an empty set is (-inf, 0).
+__device__ __forceinline__ void merge_ml(float& m, float& l, float m2, float l2) {
+  const float mn = fmaxf(m, m2);
+  if (mn == -INFINITY) return;
+  l = l * fast_exp2(m - mn) + l2 * fast_exp2(m2 - mn);
+  m = mn;
+}
+
+// The softmax pass with one DRAM read of the S row: a per-thread online
+// (max, sum) over base-2 logits, merged across the CTA; the write pass reads
+// the row again while it is still in L2 (streaming, its last use).
+__global__ void __launch_bounds__(kRowThreads, 4) bwd_softmax_vec_kernel(const BackwardArgs a) {
+  __shared__ float sh_m[kRowThreads / 32], sh_l[kRowThreads / 32], sh[kRowThreads / 32];
+  const size_t row = blockIdx.x;
+  const int R = a.qg * a.S;
+  const size_t g = row / R;
+  const int r = static_cast<int>(row % R);
+  const int gg = r / a.S, i = r % a.S;
+  const int nv = (a.M + a.S) >> 2, mv = a.M >> 2;
+  const float4* s4 = reinterpret_cast<const float4*>(a.sbuf) + row * nv;
+  uint2* p4 = reinterpret_cast<uint2*>(a.pbuf) + row * nv;
+  const int4* sp4 = reinterpret_cast<const int4*>(a.slot_pos + g * a.M);
+  const int qpos = a.pos0 + i;
+  const float c = a.scale_log2;
+
+  float m = -INFINITY, l = 0.f;
+  for (int v0 = threadIdx.x; v0 < nv; v0 += kVecUnroll * kRowThreads) {
+    float4 x[kVecUnroll];
+    int4 p[kVecUnroll];
+#pragma unroll
+    for (int u = 0; u < kVecUnroll; ++u) {
+      const int v = v0 + u * kRowThreads;
+      x[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      p[u] = make_int4(-1, -1, -1, -1);
+      if (v < nv) x[u] = s4[v];
+      if (v < mv) p[u] = __ldg(sp4 + v);
+    }
+#pragma unroll
+    for (int u = 0; u < kVecUnroll; ++u) {
+      const int v = v0 + u * kRowThreads;
+      const unsigned vm = v < nv ? vis_mask4(v, mv, p[u], qpos, i, a.M) : 0u;
+      if (vm == 0) continue;
+      const float y0 = (vm & 1u) ? x[u].x * c : -INFINITY;
+      const float y1 = (vm & 2u) ? x[u].y * c : -INFINITY;
+      const float y2 = (vm & 4u) ? x[u].z * c : -INFINITY;
+      const float y3 = (vm & 8u) ? x[u].w * c : -INFINITY;
+      const float mx = fmaxf(fmaxf(y0, y1), fmaxf(y2, y3));
+      if (mx > m) {
+        l *= fast_exp2(m - mx);
+        m = mx;
+      }
+      l += (fast_exp2(y0 - m) + fast_exp2(y1 - m)) + (fast_exp2(y2 - m) + fast_exp2(y3 - m));
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+    merge_ml(m, l, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, l, o));
+  if ((threadIdx.x & 31) == 0) {
+    sh_m[threadIdx.x >> 5] = m;
+    sh_l[threadIdx.x >> 5] = l;
+  }
+  __syncthreads();
+  m = sh_m[0];
+  l = sh_l[0];
+  for (int x = 1; x < kRowThreads / 32; ++x) merge_ml(m, l, sh_m[x], sh_l[x]);
+  const float lam = m + fast_log2(l);  // every row sees its own token
+
+  for (int v0 = threadIdx.x; v0 < nv; v0 += kVecUnroll * kRowThreads) {
+    float4 x[kVecUnroll];
+    int4 p[kVecUnroll];
+#pragma unroll
+    for (int u = 0; u < kVecUnroll; ++u) {
+      const int v = v0 + u * kRowThreads;
+      x[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      p[u] = make_int4(-1, -1, -1, -1);
+      if (v < nv) x[u] = __ldcs(s4 + v);
+      if (v < mv) p[u] = __ldg(sp4 + v);
+    }
+#pragma unroll
+    for (int u = 0; u < kVecUnroll; ++u) {
+      const int v = v0 + u * kRowThreads;
+      if (v >= nv) continue;
+      const unsigned vm = vis_mask4(v, mv, p[u], qpos, i, a.M);
+      const float e0 = (vm & 1u) ? fast_exp2(x[u].x * c - lam) : 0.f;
+      const float e1 = (vm & 2u) ? fast_exp2(x[u].y * c - lam) : 0.f;
+      const float e2 = (vm & 4u) ? fast_exp2(x[u].z * c - lam) : 0.f;
+      const float e3 = (vm & 8u) ? fast_exp2(x[u].w * c - lam) : 0.f;
+      p4[v] = make_uint2(pack_bf16x2(e0, e1), pack_bf16x2(e2, e3));
+    }
+  }
+  const int b = static_cast<int>(g / a.Hkv), h = static_cast<int>(g % a.Hkv);
+  const size_t orow = (static_cast<size_t>(b * a.Hq + h * a.qg + gg) * a.S + i) * a.d;
+  float dsum = 0.f;
+  for (int e = threadIdx.x; e < a.d; e += kRowThreads)
+    dsum += from_bf16(a.dout[orow + e]) * from_bf16(a.out[orow + e]);
+  dsum = block_reduce(dsum, sh, false);
+  if (threadIdx.x == 0) a.drow[row] = dsum;
+}
+
+// dS = P * (dP - D), one CTA per stacked row, four float4 / 8-byte loads in
+// flight per thread; dP is read for the last time (streaming).
+__global__ void __launch_bounds__(kRowThreads, 4) bwd_ds_vec_kernel(const BackwardArgs a) {
+  const size_t row = blockIdx.x;
+  const int nv = (a.M + a.S) >> 2;
+  const float dr = a.drow[row];
+  const float4* s4 = reinterpret_cast<const float4*>(a.sbuf) + row * nv;
+  const uint2* p4 = reinterpret_cast<const uint2*>(a.pbuf) + row * nv;
+  uint2* ds4 = reinterpret_cast<uint2*>(a.dsbuf) + row * nv;
+  for (int v0 = threadIdx.x; v0 < nv; v0 += kVecUnroll * kRowThreads) {
+    float4 x[kVecUnroll];
+    uint2 p[kVecUnroll];
+#pragma unroll
+    for (int u = 0; u < kVecUnroll; ++u) {
+      const int v = v0 + u * kRowThreads;
+      if (v < nv) {
+        x[u] = __ldcs(s4 + v);
+        p[u] = p4[v];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kVecUnroll; ++u) {
+      const int v = v0 + u * kRowThreads;
+      if (v >= nv) continue;
+      const float d0 = __uint_as_float(p[u].x << 16) * (x[u].x - dr);
+      const float d1 = __uint_as_float(p[u].x & 0xFFFF0000u) * (x[u].y - dr);
+      const float d2 = __uint_as_float(p[u].y << 16) * (x[u].z - dr);
+      const float d3 = __uint_as_float(p[u].y & 0xFFFF0000u) * (x[u].w - dr);
+      ds4[v] = make_uint2(pack_bf16x2(d0, d1), pack_bf16x2(d2, d3));
+    }
+  }
+}
+
 // ------------------------------------------------------------ cuBLASLt --
 struct LtState {
   std::once_flag once;
@@ -242,17 +394,28 @@ BackwardStatus launch_backward(BackwardArgs a, void* workspace, cudaStream_t str
   gemm(true, false, M, R, d, 1.f, a.k_cache, d, sKc, a.q, d, sQ, 0.f, a.sbuf, NK, sS);
   gemm(true, false, S, R, d, 1.f, a.k_new, d, sKn, a.q, d, sQ, 0.f, a.sbuf + M, NK, sS);
   if (st != CUBLAS_STATUS_SUCCESS) { out.blas = st; return out; }
-  bwd_softmax_kernel<<<static_cast<unsigned>(static_cast<size_t>(G) * R), kRowThreads, 0, stream>>>(a);
+  // the vectorised passes need float4 rows (N_k, M multiples of 4) and 16-byte
+  // aligned workspace and slot positions; every other shape takes the scalar ones
+  const bool vec = NK % 4 == 0 && M % 4 == 0 &&
+                   (reinterpret_cast<uintptr_t>(workspace) & 15u) == 0 &&
+                   (reinterpret_cast<uintptr_t>(a.slot_pos) & 15u) == 0;
+  const unsigned rows = static_cast<unsigned>(static_cast<size_t>(G) * R);
+  if (vec)
+    bwd_softmax_vec_kernel<<<rows, kRowThreads, 0, stream>>>(a);
+  else
+    bwd_softmax_kernel<<<rows, kRowThreads, 0, stream>>>(a);
   if ((ce = cudaGetLastError()) != cudaSuccess) { out.cuda = ce; return out; }
   // dP = dout V^T into the same buffer
   gemm(true, false, M, R, d, 1.f, a.v_cache, d, sKc, a.dout, d, sQ, 0.f, a.sbuf, NK, sS);
   gemm(true, false, S, R, d, 1.f, a.v_new, d, sKn, a.dout, d, sQ, 0.f, a.sbuf + M, NK, sS);
   if (st != CUBLAS_STATUS_SUCCESS) { out.blas = st; return out; }
-  {
+  if (vec) {
+    bwd_ds_vec_kernel<<<rows, kRowThreads, 0, stream>>>(a);
+  } else {
     const size_t blocks = std::min<size_t>(static_cast<size_t>(G) * R, 152 * 8);
     bwd_ds_kernel<<<static_cast<unsigned>(blocks), kRowThreads, 0, stream>>>(a);
-    if ((ce = cudaGetLastError()) != cudaSuccess) { out.cuda = ce; return out; }
   }
+  if ((ce = cudaGetLastError()) != cudaSuccess) { out.cuda = ce; return out; }
   // dQ^T (d x R) = K^T dS^T: cache block, then += chunk block
   gemm(false, false, d, R, M, a.scale, a.k_cache, d, sKc, a.dsbuf, NK, sS, 0.f, a.dq, d, sQ);
   gemm(false, false, d, R, S, a.scale, a.k_new, d, sKn, a.dsbuf + M, NK, sS, M > 0 ? 1.f : 0.f,

@@ -142,11 +142,41 @@ __device__ __forceinline__ void merge_ml(float& m, float& l, float m2, float l2)
   m = mn;
 }
 
-// The softmax pass with one DRAM read of the S row: a per-thread online
-// (max, sum) over base-2 logits, merged across the CTA; the write pass reads
-// the row again while it is still in L2 (streaming, its last use).
-__global__ void __launch_bounds__(kRowThreads, 4) bwd_softmax_vec_kernel(const BackwardArgs a) {
-  __shared__ float sh_m[kRowThreads / 32], sh_l[kRowThreads / 32], sh[kRowThreads / 32];
+// The softmax pass with one DRAM read of the S row, one CTA of kVecThreads per
+// stacked row: a per-thread online (max, sum) over base-2 logits and D's dot
+// product, merged across the CTA at one barrier.  kKeep (the row fits one trip
+// of kVecUnroll float4s per thread, N_k <= 4096): the write pass takes the
+// values still held in registers; otherwise it reads the row again while it is
+// in L2 (streaming, its last use).  Four CTAs per SM: 512-thread CTAs (one trip
+// up to N_k = 8192, two per SM) measured slower, having fewer rows in flight.
+constexpr int kVecThreads = 256;
+
+__device__ __forceinline__ void online4(float4 x, unsigned vm, float c, float& m, float& l) {
+  if (vm == 0) return;
+  const float y0 = (vm & 1u) ? x.x * c : -INFINITY;
+  const float y1 = (vm & 2u) ? x.y * c : -INFINITY;
+  const float y2 = (vm & 4u) ? x.z * c : -INFINITY;
+  const float y3 = (vm & 8u) ? x.w * c : -INFINITY;
+  const float mx = fmaxf(fmaxf(y0, y1), fmaxf(y2, y3));
+  if (mx > m) {
+    l *= fast_exp2(m - mx);
+    m = mx;
+  }
+  l += (fast_exp2(y0 - m) + fast_exp2(y1 - m)) + (fast_exp2(y2 - m) + fast_exp2(y3 - m));
+}
+
+__device__ __forceinline__ uint2 probs4(float4 x, unsigned vm, float c, float lam) {
+  const float e0 = (vm & 1u) ? fast_exp2(x.x * c - lam) : 0.f;
+  const float e1 = (vm & 2u) ? fast_exp2(x.y * c - lam) : 0.f;
+  const float e2 = (vm & 4u) ? fast_exp2(x.z * c - lam) : 0.f;
+  const float e3 = (vm & 8u) ? fast_exp2(x.w * c - lam) : 0.f;
+  return make_uint2(pack_bf16x2(e0, e1), pack_bf16x2(e2, e3));
+}
+
+template <bool kKeep>
+__global__ void __launch_bounds__(kVecThreads, 4) bwd_softmax_vec_kernel(const BackwardArgs a) {
+  constexpr int T = kVecThreads, U = kVecUnroll, W = kVecThreads / 32;
+  __shared__ float sh_m[W], sh_l[W], sh_d[W];
   const size_t row = blockIdx.x;
   const int R = a.qg * a.S;
   const size_t g = row / R;
@@ -159,78 +189,84 @@ __global__ void __launch_bounds__(kRowThreads, 4) bwd_softmax_vec_kernel(const B
   const int qpos = a.pos0 + i;
   const float c = a.scale_log2;
 
+  // D = dout . out of this row (query head h q_g + gg, token i), d <= T: the
+  // two loads go out ahead of the row's and are used after them
+  const int b = static_cast<int>(g / a.Hkv), h = static_cast<int>(g % a.Hkv);
+  const size_t orow = (static_cast<size_t>(b * a.Hq + h * a.qg + gg) * a.S + i) * a.d;
+  uint16_t dv = 0, ov = 0;
+  if (static_cast<int>(threadIdx.x) < a.d) {
+    dv = a.dout[orow + threadIdx.x];
+    ov = a.out[orow + threadIdx.x];
+  }
+
   float m = -INFINITY, l = 0.f;
-  for (int v0 = threadIdx.x; v0 < nv; v0 += kVecUnroll * kRowThreads) {
-    float4 x[kVecUnroll];
-    int4 p[kVecUnroll];
+  float4 x[U];
+  unsigned vm[U];
 #pragma unroll
-    for (int u = 0; u < kVecUnroll; ++u) {
-      const int v = v0 + u * kRowThreads;
+  for (int u = 0; u < U; ++u) vm[u] = 0u;
+  for (int v0 = threadIdx.x; v0 < nv; v0 += U * T) {
+    int4 p[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int v = v0 + u * T;
       x[u] = make_float4(0.f, 0.f, 0.f, 0.f);
       p[u] = make_int4(-1, -1, -1, -1);
       if (v < nv) x[u] = s4[v];
       if (v < mv) p[u] = __ldg(sp4 + v);
     }
 #pragma unroll
-    for (int u = 0; u < kVecUnroll; ++u) {
-      const int v = v0 + u * kRowThreads;
-      const unsigned vm = v < nv ? vis_mask4(v, mv, p[u], qpos, i, a.M) : 0u;
-      if (vm == 0) continue;
-      const float y0 = (vm & 1u) ? x[u].x * c : -INFINITY;
-      const float y1 = (vm & 2u) ? x[u].y * c : -INFINITY;
-      const float y2 = (vm & 4u) ? x[u].z * c : -INFINITY;
-      const float y3 = (vm & 8u) ? x[u].w * c : -INFINITY;
-      const float mx = fmaxf(fmaxf(y0, y1), fmaxf(y2, y3));
-      if (mx > m) {
-        l *= fast_exp2(m - mx);
-        m = mx;
-      }
-      l += (fast_exp2(y0 - m) + fast_exp2(y1 - m)) + (fast_exp2(y2 - m) + fast_exp2(y3 - m));
+    for (int u = 0; u < U; ++u) {
+      const int v = v0 + u * T;
+      vm[u] = v < nv ? vis_mask4(v, mv, p[u], qpos, i, a.M) : 0u;
+      online4(x[u], vm[u], c, m, l);
     }
   }
+  float dsum = from_bf16(dv) * from_bf16(ov);
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1)
+  for (int o = 16; o > 0; o >>= 1) {
     merge_ml(m, l, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, l, o));
+    dsum += __shfl_xor_sync(0xffffffffu, dsum, o);
+  }
   if ((threadIdx.x & 31) == 0) {
     sh_m[threadIdx.x >> 5] = m;
     sh_l[threadIdx.x >> 5] = l;
+    sh_d[threadIdx.x >> 5] = dsum;
   }
   __syncthreads();
   m = sh_m[0];
   l = sh_l[0];
-  for (int x = 1; x < kRowThreads / 32; ++x) merge_ml(m, l, sh_m[x], sh_l[x]);
+  for (int w = 1; w < W; ++w) merge_ml(m, l, sh_m[w], sh_l[w]);
   const float lam = m + fast_log2(l);  // every row sees its own token
+  if (threadIdx.x == 0) {
+    float dr = 0.f;
+    for (int w = 0; w < W; ++w) dr += sh_d[w];
+    a.drow[row] = dr;
+  }
 
-  for (int v0 = threadIdx.x; v0 < nv; v0 += kVecUnroll * kRowThreads) {
-    float4 x[kVecUnroll];
-    int4 p[kVecUnroll];
+  if constexpr (kKeep) {  // nv <= U T: x and vm hold this thread's whole share
 #pragma unroll
-    for (int u = 0; u < kVecUnroll; ++u) {
-      const int v = v0 + u * kRowThreads;
-      x[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-      p[u] = make_int4(-1, -1, -1, -1);
-      if (v < nv) x[u] = __ldcs(s4 + v);
-      if (v < mv) p[u] = __ldg(sp4 + v);
+    for (int u = 0; u < U; ++u) {
+      const int v = threadIdx.x + u * T;
+      if (v < nv) p4[v] = probs4(x[u], vm[u], c, lam);
     }
+  } else {
+    for (int v0 = threadIdx.x; v0 < nv; v0 += U * T) {
+      int4 p[U];
 #pragma unroll
-    for (int u = 0; u < kVecUnroll; ++u) {
-      const int v = v0 + u * kRowThreads;
-      if (v >= nv) continue;
-      const unsigned vm = vis_mask4(v, mv, p[u], qpos, i, a.M);
-      const float e0 = (vm & 1u) ? fast_exp2(x[u].x * c - lam) : 0.f;
-      const float e1 = (vm & 2u) ? fast_exp2(x[u].y * c - lam) : 0.f;
-      const float e2 = (vm & 4u) ? fast_exp2(x[u].z * c - lam) : 0.f;
-      const float e3 = (vm & 8u) ? fast_exp2(x[u].w * c - lam) : 0.f;
-      p4[v] = make_uint2(pack_bf16x2(e0, e1), pack_bf16x2(e2, e3));
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + u * T;
+        x[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        p[u] = make_int4(-1, -1, -1, -1);
+        if (v < nv) x[u] = __ldcs(s4 + v);
+        if (v < mv) p[u] = __ldg(sp4 + v);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + u * T;
+        if (v < nv) p4[v] = probs4(x[u], vis_mask4(v, mv, p[u], qpos, i, a.M), c, lam);
+      }
     }
   }
-  const int b = static_cast<int>(g / a.Hkv), h = static_cast<int>(g % a.Hkv);
-  const size_t orow = (static_cast<size_t>(b * a.Hq + h * a.qg + gg) * a.S + i) * a.d;
-  float dsum = 0.f;
-  for (int e = threadIdx.x; e < a.d; e += kRowThreads)
-    dsum += from_bf16(a.dout[orow + e]) * from_bf16(a.out[orow + e]);
-  dsum = block_reduce(dsum, sh, false);
-  if (threadIdx.x == 0) a.drow[row] = dsum;
 }
 
 // dS = P * (dP - D), one CTA per stacked row, four float4 / 8-byte loads in
@@ -396,12 +432,14 @@ BackwardStatus launch_backward(BackwardArgs a, void* workspace, cudaStream_t str
   if (st != CUBLAS_STATUS_SUCCESS) { out.blas = st; return out; }
   // the vectorised passes need float4 rows (N_k, M multiples of 4) and 16-byte
   // aligned workspace and slot positions; every other shape takes the scalar ones
-  const bool vec = NK % 4 == 0 && M % 4 == 0 &&
+  const bool vec = NK % 4 == 0 && M % 4 == 0 && d <= kVecThreads &&
                    (reinterpret_cast<uintptr_t>(workspace) & 15u) == 0 &&
                    (reinterpret_cast<uintptr_t>(a.slot_pos) & 15u) == 0;
   const unsigned rows = static_cast<unsigned>(static_cast<size_t>(G) * R);
-  if (vec)
-    bwd_softmax_vec_kernel<<<rows, kRowThreads, 0, stream>>>(a);
+  if (vec && NK / 4 <= kVecUnroll * kVecThreads)
+    bwd_softmax_vec_kernel<true><<<rows, kVecThreads, 0, stream>>>(a);
+  else if (vec)
+    bwd_softmax_vec_kernel<false><<<rows, kVecThreads, 0, stream>>>(a);
   else
     bwd_softmax_kernel<<<rows, kRowThreads, 0, stream>>>(a);
   if ((ce = cudaGetLastError()) != cudaSuccess) { out.cuda = ce; return out; }

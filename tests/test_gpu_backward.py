@@ -34,6 +34,7 @@ CASES = [
     (2, 8, 2, 128, 20, 300, 17, 5, 900),     # ragged S and M, empty and future slots
     (3, 6, 3, 64, 1, 130, 5, 0, 140),        # one token
     (1, 4, 2, 64, 6, 130, 3, 2, 150),        # N_k a multiple of 4, M not: the scalar passes
+    (1, 2, 1, 64, 8, 4100, 20, 3, 4200),     # N_k > 4096: the softmax pass reads each row twice
     (1, 4, 4, 128, 200, 0, 0, 0, 0),         # no cache (a prefill)
     (1, 32, 8, 128, 512, 4096, 0, 0, 8192),  # the Llama-3-8B-shaped chunk
 ]

@@ -32,6 +32,7 @@ def _load(fname, mutation=None):
             pos = src.index(old, pos + 1)
         src = src[:pos] + new + src[pos + len(old):]
     mod = types.ModuleType("oracle_variant_" + fname.replace(".", "_"))
+    mod.__package__ = "oracle"  # relative imports resolve to the untouched oracle
     exec(compile(src, fname, "exec"), mod.__dict__)
     return mod
 
@@ -172,8 +173,41 @@ def pin_backward_fd(bmod, fmod):
     return True
 
 
+def pin_quant(q):
+    """Hand rows with known codes (max 127 -> s = 1; max 254 -> s = 2), their
+    read-back values, bf16 rounding against torch and by hand."""
+    x = np.array([[127.0, -63.5, 1.0, 0.5, -0.5, 1.5, 2.5, 0.0]], np.float32)
+    codes, s = q.quantize_rows(x)
+    if s[0] != 1.0 or codes[0].tolist() != [127, -64, 1, 0, 0, 2, 2, 0]:
+        return False
+    codes, s = q.quantize_rows(np.array([[-254.0, 3.0, 5.0, -7.0]], np.float32))
+    if s[0] != 2.0 or codes[0].tolist() != [-127, 2, 2, -4]:
+        return False
+    if q.dequantize_rows(codes, s)[0].tolist() != [-254.0, 4.0, 4.0, -8.0]:
+        return False
+    y = np.float32([1 + 2 ** -8, 1 + 3 * 2 ** -8, 3.14159, -2.71828e-3])
+    return np.array_equal(q.round_to_bf16(y), torch.from_numpy(y).to(torch.bfloat16).float().numpy())
+
+
+def pin_q8_write(q):
+    """The slots evict_insert_q8 overwrites hold the chunk's own K (and V) rows,
+    within half a step."""
+    rng = np.random.default_rng(97)
+    st = wl.random_state(rng, 1, 1, 8, 8, pos0=30)
+    kc, ks = q.quantize_rows(st["k_cache"])
+    vc, vs = q.quantize_rows(st["v_cache"])
+    _, kn, vn = _rand_seq(rng, 1, 1, 1, 2, 8)
+    res = q.evict_insert_q8(st["scores"], st["slot_pos"], kn, vn, kc, ks, vc, vs, 30, 0)
+    for c, e in enumerate(res["evict_idx"][0, 0]):
+        for codes, sc, new in ((res["k_codes"], res["k_scales"], kn), (res["v_codes"], res["v_scales"], vn)):
+            if np.abs(codes[0, 0, e] * np.float64(sc[0, 0, e]) - new[0, 0, c]).max() > 0.51 * sc[0, 0, e]:
+                return False
+    return True
+
+
 def _all_pins(mods):
     h, r, b = mods["h2o_oracle.py"], mods["replay.py"], mods["backward.py"]
+    qm = mods["quant.py"]
     return {
         "dense": pin_dense(h),
         "dense_paper": pin_dense(h, "paper"),
@@ -182,6 +216,8 @@ def _all_pins(mods):
         "evict_insert": pin_evict_insert(h),
         "replay": pin_replay(r),
         "backward_fd": pin_backward_fd(b, h),
+        "quant": pin_quant(qm),
+        "q8_write": pin_q8_write(qm),
     }
 
 
@@ -213,9 +249,16 @@ MUTATIONS = {
     "backward_without_mask": ("backward.py", 'a = a.masked_fill(~visible, float("-inf"))',
                               "a = a", 0),
     "backward_wrong_scale": ("backward.py", "scale = 1.0 / math.sqrt(d)", "scale = 1.0 / d", 0),
+    "quant_scale_over_128": ("quant.py", "QMAX = 127", "QMAX = 128", 0),
+    "quant_rounds_toward_zero": ("quant.py", "np.clip(np.rint(ratio)", "np.clip(np.trunc(ratio)", 0),
+    "dequant_drops_scale": ("quant.py", " * np.asarray(scales, np.float32)[..., None]", "", 0),
+    "bf16_truncates": ("quant.py", "r = ((u + 0x7FFF + lsb) >> 16) << 16", "r = (u >> 16) << 16", 0),
+    "bf16_ties_away": ("quant.py", "u + 0x7FFF + lsb", "u + 0x8000", 0),
+    "q8_write_swaps_k_and_v": ("quant.py", "kc[b, h, e], ks[b, h, e] = qk[b, h, c], sk[b, h, c]",
+                               "kc[b, h, e], ks[b, h, e] = qv[b, h, c], sv[b, h, c]", 0),
 }
 
-FILES = ("h2o_oracle.py", "replay.py", "backward.py")
+FILES = ("h2o_oracle.py", "replay.py", "backward.py", "quant.py")
 
 
 def test_untouched_oracle_passes_every_pin():

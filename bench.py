@@ -211,16 +211,21 @@ def barrier(world: int):
 
 
 # ---------------------------------------------------------- CPU baseline --
-def oracle_sample(w: wl.Workload, budget_s: float = 12.0, max_chunks: int = 8):
+def oracle_sample(w: wl.Workload, budget_s: float = 12.0, max_chunks: int = 8,
+                  kv_bits: int = 16):
     """Times the float64 oracle on chunk steps of the workload (cache full).
 
     Sample: starting from a full cache (random state of the right shape), the
-    oracle runs chunk steps (sparse SDPA + update) until ``budget_s`` seconds
-    or ``max_chunks`` chunks; returns tokens/s and a description."""
-    from oracle import sdpa_chunk, update
+    oracle runs chunk steps (sparse SDPA + update; with ``kv_bits`` 8 their
+    8-bit buffer forms) until ``budget_s`` seconds or ``max_chunks`` chunks;
+    returns tokens/s and a description."""
+    from oracle import quantize_rows, sdpa_chunk, sdpa_chunk_q8, update, update_q8
     rng = np.random.default_rng(0)
     p0 = w.M + w.S  # a position in the steady state
     st = wl.random_state(rng, w.B, w.Hkv, w.M, w.d, pos0=p0)
+    if kv_bits == 8:
+        st["k_codes"], st["k_scales"] = quantize_rows(st["k_cache"])
+        st["v_codes"], st["v_scales"] = quantize_rows(st["v_cache"])
     n, t_total = 0, 0.0
     while n < max_chunks and t_total < budget_s:
         p = p0 + n * w.S
@@ -228,18 +233,23 @@ def oracle_sample(w: wl.Workload, budget_s: float = 12.0, max_chunks: int = 8):
             break
         q, k, v = wl.batch_tokens(w, p, p + w.S)
         t0 = time.perf_counter()
-        _, inc, _ = sdpa_chunk(q, st["k_cache"], st["v_cache"], k, v, st["slot_pos"], p)
-        r = update(st["scores"], st["slot_pos"], inc, k, v, st["k_cache"], st["v_cache"], p, w.W,
-                   "fp64")
+        if kv_bits == 8:
+            buf = [st[x] for x in ("k_codes", "k_scales", "v_codes", "v_scales")]
+            _, inc, _ = sdpa_chunk_q8(q, *buf, k, v, st["slot_pos"], p)
+            r = update_q8(st["scores"], st["slot_pos"], inc, k, v, *buf, p, w.W, "fp64")
+        else:
+            _, inc, _ = sdpa_chunk(q, st["k_cache"], st["v_cache"], k, v, st["slot_pos"], p)
+            r = update(st["scores"], st["slot_pos"], inc, k, v, st["k_cache"], st["v_cache"], p,
+                       w.W, "fp64")
         t_total += time.perf_counter() - t0
-        st = dict(scores=r["scores"], slot_pos=r["slot_pos"], k_cache=r["k_cache"],
-                  v_cache=r["v_cache"])
+        st = {x: r[x] for x in r if x != "evict_idx"}
         n += 1
     tokens = n * w.S * w.B
     return dict(value=tokens / t_total, unit="tokens/s", cores=os.cpu_count(), kind="oracle",
                 seconds=t_total,
                 sample=(f"{n} steady-state chunk steps ({w.S} tokens x B={w.B}, cache of {w.M} "
-                        f"slots full) of the {w.name} workload, float64 NumPy oracle"))
+                        f"slots full{', 8-bit K/V buffers' if kv_bits == 8 else ''}) of the "
+                        f"{w.name} workload, float64 NumPy oracle"))
 
 
 def run_reference(args, w):
@@ -249,7 +259,7 @@ def run_reference(args, w):
     times = []
     tokens = 0
     for i in range(args.warmup + args.steps):
-        r = oracle_sample(w, budget_s=args.ref_budget, max_chunks=1)
+        r = oracle_sample(w, budget_s=args.ref_budget, max_chunks=1, kv_bits=args.kv_bits)
         if i >= args.warmup:
             times.append(r["seconds"])
             tokens += w.S * w.B
@@ -305,7 +315,7 @@ def run_ours(args, w):
     outs = [torch.empty((w.B, w.Hq, e - p, w.d), dtype=torch.bfloat16, device=dev)
             for p, e in plan]
     layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, keep_evictions=True,
-                     order=args.order)
+                     order=args.order, kv_bits=args.kv_bits)
     stream = torch.cuda.current_stream()
     n_chunks = len(plan) - 1
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -386,23 +396,27 @@ def run_ours(args, w):
                          if in_bytes > 129e6 else f"{in_bytes / 1e6:.0f} MB of inputs per step",
                    "launch": "CUDA graph of the whole step" if args.graph else "eager",
                    "order": args.order,
+                   "kv_buffers": "int8 codes + fp32 row scales" if args.kv_bits == 8 else "bf16",
                    "parallelism": f"replicas x{world}"},
         "tflops": alg_tflops,
         "tflops_frac_of_peak": alg_tflops / pk["bf16_sus"],
         "chunk_step_ms_median": statistics.median(chunk_step_ms) if chunk_step_ms else None,
-        "gpu_launches": args.steps * sum(launches_per_chunk(e - p, w.M, args.order)
-                                         for p, e in plan),
+        "gpu_launches": args.steps * sum(launches_per_chunk(e - p, w.M, args.order,
+                                                            args.kv_bits) for p, e in plan),
         "clocks": clocks,
     }
     # the chunk SDPA is timed on its own (launch after launch, L2 flushed in
     # between): its denominator is the burst peak; the sustained one is given
     # alongside
     traffic = args.traffic if args.traffic is not None else (
-        SDPA_DRAM_BYTES if w.name == "llama8b_32k" and args.order == "chunk" else None)
+        SDPA_DRAM_BYTES if w.name == "llama8b_32k" and args.order == "chunk" and
+        args.kv_bits == 16 else None)
     if w.S == 1:
         # decode: K and V read once per step, HBM bound
         line["roofline"] = {
-            "bound": "hbm", "kernel": "decode_split_kernel + decode_combine_kernel (one step)",
+            "bound": "hbm",
+            "kernel": ("kv_dequantize_kernel + " if args.kv_bits == 8 else "") +
+                      "decode_split_kernel + decode_combine_kernel (one step)",
             "achieved": kern["gbs"], "peak": pk["hbm"], "unit": "GB/s",
             "frac": kern["gbs"] / pk["hbm"], "traffic": traffic,
             "peak_source": f"{pk['source']} HBM copy bandwidth",
@@ -411,7 +425,8 @@ def run_ours(args, w):
     else:
         line["roofline"] = {
             "bound": "tensor",
-            "kernel": "sdpa_chunk_kernel<128,pair> (steady-state chunk" +
+            "kernel": ("kv_dequantize_kernel + " if args.kv_bits == 8 else "") +
+                      "sdpa_chunk_kernel<128,pair> (steady-state chunk" +
                       (", cache only)" if args.order == "paper" else ")"),
             "achieved": kern["alg_tflops"], "peak": pk["bf16"], "unit": "TFLOP/s",
             "frac": kern["alg_tflops"] / pk["bf16"], "traffic": traffic,
@@ -423,7 +438,7 @@ def run_ours(args, w):
     if args.e2e:
         line["e2e"] = run_e2e(w, layer, plan, outs, dev, args, world)
     if args.cpu_baseline and rank == 0 and world == 1:
-        line["cpu_baseline"] = oracle_sample(w)
+        line["cpu_baseline"] = oracle_sample(w, kv_bits=args.kv_bits)
     if rank == 0:
         print(json.dumps(line))
     return 0
@@ -432,7 +447,8 @@ def run_ours(args, w):
 def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None, prepare=True):
     """Average duration of the steady-state chunk SDPA launch (CUDA events)."""
     import torch
-    from paper_2608_19920_gb300 import h2o_evict_insert, h2o_sdpa_cache, h2o_sdpa_chunk
+    from paper_2608_19920_gb300 import (h2o_evict_insert, h2o_evict_insert_q8, h2o_sdpa_cache,
+                                       h2o_sdpa_cache_q8, h2o_sdpa_chunk, h2o_sdpa_chunk_q8)
     idx = len(plan) // 2 if idx is None else idx
     if prepare and idx > 0:
         # the cache as the sequence leaves it just before chunk idx
@@ -446,15 +462,28 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None, prepare=Tru
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
     clean = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=q.device)
 
+    q8 = layer.kv_bits == 8
+    buf = (layer.k_codes, layer.k_scales, layer.v_codes, layer.v_scales) if q8 else None
+
     def call():
         if layer.order == "paper":  # the cache already holds the chunk (filled by the caller)
-            h2o_sdpa_cache(q, layer.k_cache, layer.v_cache, layer.slot_pos, p, out=out,
-                           score_inc=inc, workspace=ws)
+            if q8:
+                h2o_sdpa_cache_q8(q, *buf, layer.slot_pos, p, out=out, score_inc=inc,
+                                  workspace=ws)
+            else:
+                h2o_sdpa_cache(q, layer.k_cache, layer.v_cache, layer.slot_pos, p, out=out,
+                               score_inc=inc, workspace=ws)
+        elif q8:
+            h2o_sdpa_chunk_q8(q, *buf, k, v, layer.slot_pos, p, out=out, score_inc=inc,
+                              workspace=ws)
         else:
             h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out=out,
                            score_inc=inc, workspace=ws)
 
-    if layer.order == "paper":
+    if layer.order == "paper" and q8:
+        h2o_evict_insert_q8(layer.scores, layer.slot_pos, k, v, *buf, p, layer.W,
+                            policy=layer.policy, Hq=layer.Hq)
+    elif layer.order == "paper":
         h2o_evict_insert(layer.scores, layer.slot_pos, k, v, layer.k_cache, layer.v_cache, p,
                          layer.W, policy=layer.policy, Hq=layer.Hq)
     # the call is replayed from a CUDA graph, as in the timed steps
@@ -480,22 +509,25 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None, prepare=Tru
     avg_ms = sum(times) / len(times)
     flops = chunk_flops(w.B, w.Hq, w.d, e - p, visible_old(w, e - p, layer.order))
     exec_flops = executed_mma_flops(w, e - p)
-    kv_bytes = decode_kv_bytes(w)
+    kv_bytes = decode_kv_bytes(w, layer.kv_bits)
     return dict(avg_us=avg_ms * 1e3, flops=flops, alg_tflops=flops / (avg_ms / 1e3) / 1e12,
                 exec_ratio=exec_flops / flops, bytes=kv_bytes, gbs=kv_bytes / (avg_ms / 1e3) / 1e9)
 
 
-def decode_kv_bytes(w):
-    """Algorithmic bytes of one decode step: every cache K and V row read once."""
-    return 2.0 * w.B * w.Hkv * w.M * w.d * 2
+def decode_kv_bytes(w, kv_bits: int = 16):
+    """Algorithmic bytes of one decode step: every cache K and V row read once
+    (8-bit buffers: d codes and a 4-byte scale per row)."""
+    row = w.d * 2 if kv_bits == 16 else w.d + 4
+    return 2.0 * w.B * w.Hkv * w.M * row
 
 
-def launches_per_chunk(S, M, order="chunk"):
+def launches_per_chunk(S, M, order="chunk", kv_bits=16):
     """Kernels of this library one chunk launches: the SDPA (split + combine
     when S = 1 and a cache exists) and the update (the paper's order: the
-    eviction-insert, the SDPA and the score addition)."""
+    eviction-insert, the SDPA and the score addition); 8-bit buffers add the
+    read-back before the SDPA and the quantising scatter after the update."""
     sdpa = 2 if S == 1 and M > 0 else 1
-    return sdpa + (2 if order == "paper" else 1)
+    return sdpa + (2 if order == "paper" else 1) + (2 if kv_bits == 8 else 0)
 
 
 def executed_mma_flops(w, S):
@@ -588,6 +620,9 @@ def main():
     ap.add_argument("--order", default="chunk", choices=["chunk", "paper"],
                     help="chunk step order: attend then evict (default), or the paper's "
                          "evict-and-write first")
+    ap.add_argument("--kv-bits", type=int, default=16, choices=[16, 8],
+                    help="cache buffers: bf16 rows (default) or int8 codes with a float32 "
+                         "scale per row")
     ap.add_argument("--no-graph", dest="graph", action="store_false",
                     help="launch the timed steps eagerly instead of replaying a CUDA graph")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
@@ -619,7 +654,8 @@ def run_kernel_only(args, w, n_fill: int = 8):
     build_mod.build()
     dev = torch.device("cuda", 0)
     plan = step_plan(w)[:n_fill + 2]
-    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, order=args.order)
+    layer = H2OLayer(w.B, w.Hq, w.Hkv, w.d, w.M, w.S, w.W, device=dev, order=args.order,
+                     kv_bits=args.kv_bits)
     ins = []
     for p, e in plan:
         ins.append(tuple(torch.from_numpy(x).to(torch.bfloat16).to(dev)

@@ -26,6 +26,9 @@
  *                                    recurrence (§3.2, §A.1.1)
  *   h2o_sdpa_chunk_backward          the gradient of one chunk's SDPA
  *   h2o_sdpa_decode_static           S = 1 SDPA on a fixed internal scratch
+ *   h2o_kv_quantize, h2o_kv_dequantize, h2o_update_q8, h2o_evict_insert_q8,
+ *   h2o_sdpa_chunk_q8, h2o_sdpa_cache_q8, h2o_q8_workspace_size
+ *                                    8-bit K/V cache buffers (§4 setup)
  *
  * Conventions for every call:
  *  - All array arguments are DEVICE pointers, allocated and owned by the
@@ -276,6 +279,69 @@ H2O_API int h2o_kv_replace(const h2o_dims_t* dims, int64_t pos0, const int32_t* 
 H2O_API int h2o_kv_restore(const h2o_dims_t* dims, const int32_t* index,
                    const h2o_bf16* delta_k, const h2o_bf16* delta_v, const int32_t* delta_pos,
                    h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t* slot_pos, void* stream);
+
+/*
+ * 8-bit K/V cache buffers (§4 setup: the KV cache buffers are stored in 8
+ * bits; the format below is this library's, the paper names none).
+ *
+ * Every cache row of d elements (one token's key, or its value, in one KV
+ * head) is d signed codes and one scale, symmetric per row:
+ *   s = max_e |x_e| / 127                      (float32, IEEE division)
+ *   c_e = round_half_even(x_e / s), clipped to [-127, 127]  (float32 ratio)
+ * An all-zero row has s = 0 and codes 0.  A row reads back as
+ * bf16(float32(c) * s) (the product in float32, rounded to nearest even):
+ * the attention computes on those bf16 values as it does on a bf16 cache.
+ *
+ * Buffers: k_codes / v_codes (B, Hkv, M, d) int8; k_scales / v_scales
+ * (B, Hkv, M) float32; slot_pos and scores as for the bf16 calls.
+ *
+ *   h2o_kv_quantize    x (n_rows, d) bf16 -> codes (n_rows, d), scales (n_rows);
+ *                      d is 64 or 128; n_rows == 0 enqueues nothing.
+ *   h2o_kv_dequantize  codes, scales -> x (n_rows, d) bf16, the read-back above.
+ *   h2o_update_q8, h2o_evict_insert_q8
+ *                      h2o_update_policy / h2o_evict_insert on 8-bit buffers:
+ *                      the same slots, scores and positions; the chosen slots
+ *                      take the chunk's rows (k_new, v_new bf16) quantised.
+ *                      evict_idx (B, Hkv, S) is required: the call sets it to
+ *                      -1, the update writes the chosen slots, then a second
+ *                      kernel quantises the rows into them.  A (b, h) left
+ *                      unchanged (H2O_DEVERR_CANDIDATES) keeps -1 and its
+ *                      buffers.  Errors as h2o_update_policy.
+ *   h2o_sdpa_chunk_q8, h2o_sdpa_cache_q8
+ *                      h2o_sdpa_chunk / h2o_sdpa_cache with the cache read
+ *                      through the 8-bit buffers (the chunk's own k_new /
+ *                      v_new stay bf16 in h2o_sdpa_chunk_q8).  The workspace
+ *                      (h2o_q8_workspace_size bytes, 16-byte aligned) holds
+ *                      the K and V rows read back to bf16 (2 B d per slot
+ *                      each; 8 MiB each for B = 1, Hkv = 8, M = 4096, d = 128,
+ *                      which stays in L2) ahead of the attention's own
+ *                      workspace.  Errors as h2o_sdpa_chunk / h2o_sdpa_cache.
+ */
+H2O_API int h2o_kv_quantize(int64_t n_rows, int32_t d, const h2o_bf16* x, int8_t* codes,
+                   float* scales, void* stream);
+H2O_API int h2o_kv_dequantize(int64_t n_rows, int32_t d, const int8_t* codes,
+                   const float* scales, h2o_bf16* x, void* stream);
+H2O_API int h2o_q8_workspace_size(const h2o_dims_t* dims, size_t* bytes);
+H2O_API int h2o_update_q8(const h2o_dims_t* dims, int64_t pos0, float* scores,
+                   int32_t* slot_pos, const float* score_inc, const h2o_bf16* k_new,
+                   const h2o_bf16* v_new, int8_t* k_codes, float* k_scales, int8_t* v_codes,
+                   float* v_scales, int32_t budget, int32_t recent_window, int32_t policy,
+                   int32_t* evict_idx, void* stream);
+H2O_API int h2o_evict_insert_q8(const h2o_dims_t* dims, int64_t pos0, float* scores,
+                   int32_t* slot_pos, const h2o_bf16* k_new, const h2o_bf16* v_new,
+                   int8_t* k_codes, float* k_scales, int8_t* v_codes, float* v_scales,
+                   int32_t budget, int32_t recent_window, int32_t policy, int32_t* evict_idx,
+                   void* stream);
+H2O_API int h2o_sdpa_chunk_q8(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const int8_t* k_codes, const float* k_scales,
+                   const int8_t* v_codes, const float* v_scales, const h2o_bf16* k_new,
+                   const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out,
+                   float* score_inc, void* workspace, size_t workspace_bytes, void* stream);
+H2O_API int h2o_sdpa_cache_q8(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const int8_t* k_codes, const float* k_scales,
+                   const int8_t* v_codes, const float* v_scales, const int32_t* slot_pos,
+                   h2o_bf16* out, float* score_inc, void* workspace, size_t workspace_bytes,
+                   void* stream);
 
 /*
  * Gradient of one chunk of h2o_sdpa_chunk (§3.1 Eq. 2 with the mask of

@@ -25,6 +25,8 @@ EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2
            "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
            "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
            "h2o_sdpa_chunk_backward", "h2o_selftest_bounded_wait",
+           "h2o_kv_quantize", "h2o_kv_dequantize", "h2o_q8_workspace_size", "h2o_update_q8",
+           "h2o_evict_insert_q8", "h2o_sdpa_chunk_q8", "h2o_sdpa_cache_q8",
            "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
            "h2o_version")
 
@@ -77,6 +79,13 @@ def load(path: str = LIB_PATH):
     lib.h2o_backward_workspace_size.argtypes = [dims_p, ctypes.POINTER(ctypes.c_size_t)]
     lib.h2o_sdpa_chunk_backward.argtypes = [dims_p, i64, f32] + [vp] * 14 + [ctypes.c_size_t, vp]
     lib.h2o_selftest_bounded_wait.argtypes = [i64, vp]
+    lib.h2o_kv_quantize.argtypes = [i64, i32, vp, vp, vp, vp]
+    lib.h2o_kv_dequantize.argtypes = [i64, i32, vp, vp, vp, vp]
+    lib.h2o_q8_workspace_size.argtypes = [dims_p, ctypes.POINTER(ctypes.c_size_t)]
+    lib.h2o_update_q8.argtypes = [dims_p, i64] + [vp] * 9 + [i32, i32, i32, vp, vp]
+    lib.h2o_evict_insert_q8.argtypes = [dims_p, i64] + [vp] * 8 + [i32, i32, i32, vp, vp]
+    lib.h2o_sdpa_chunk_q8.argtypes = [dims_p, i64, f32] + [vp] * 11 + [ctypes.c_size_t, vp]
+    lib.h2o_sdpa_cache_q8.argtypes = [dims_p, i64, f32] + [vp] * 9 + [ctypes.c_size_t, vp]
     lib.h2o_cache_reset.argtypes = [dims_p, vp, vp, vp]
     lib.h2o_status_string.argtypes = [ctypes.c_int]
     lib.h2o_status_string.restype = ctypes.c_char_p
@@ -84,6 +93,8 @@ def load(path: str = LIB_PATH):
                "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
                "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
                "h2o_sdpa_chunk_backward", "h2o_selftest_bounded_wait", "h2o_cache_reset",
+               "h2o_kv_quantize", "h2o_kv_dequantize", "h2o_q8_workspace_size",
+               "h2o_update_q8", "h2o_evict_insert_q8", "h2o_sdpa_chunk_q8", "h2o_sdpa_cache_q8",
                "h2o_last_cuda_error",
                "h2o_device_errors", "h2o_version"):
         getattr(lib, fn).restype = ctypes.c_int
@@ -454,3 +465,165 @@ def h2o_status_string(status: int) -> str:
 
 def h2o_version() -> int:
     return load().h2o_version()
+
+
+# ---------------------------------------------------- 8-bit K/V buffers --
+
+def h2o_kv_quantize(x, codes=None, scales=None, stream=None):
+    """Rows (..., d) bf16 -> (codes (..., d) int8, scales (...) f32), per-row
+    symmetric (see include/h2o.h)."""
+    lib = load()
+    dev = x.device
+    d = x.shape[-1]
+    _expect(x, "x", x.shape, torch.bfloat16, dev)
+    if codes is None:
+        codes = torch.empty(x.shape, dtype=torch.int8, device=dev)
+    if scales is None:
+        scales = torch.empty(x.shape[:-1], dtype=torch.float32, device=dev)
+    _expect(codes, "codes", x.shape, torch.int8, dev)
+    _expect(scales, "scales", x.shape[:-1], torch.float32, dev)
+    n = x.numel() // d if d else 0
+    _check("h2o_kv_quantize", lib.h2o_kv_quantize(int(n), int(d), _ptr(x), _ptr(codes),
+                                                  _ptr(scales), _stream(stream)))
+    return codes, scales
+
+
+def h2o_kv_dequantize(codes, scales, out=None, stream=None):
+    """codes (..., d) int8 + scales (...) f32 -> the bf16 rows they read back as."""
+    lib = load()
+    dev = codes.device
+    d = codes.shape[-1]
+    _expect(codes, "codes", codes.shape, torch.int8, dev)
+    _expect(scales, "scales", codes.shape[:-1], torch.float32, dev)
+    if out is None:
+        out = torch.empty(codes.shape, dtype=torch.bfloat16, device=dev)
+    _expect(out, "out", codes.shape, torch.bfloat16, dev)
+    n = codes.numel() // d if d else 0
+    _check("h2o_kv_dequantize", lib.h2o_kv_dequantize(int(n), int(d), _ptr(codes), _ptr(scales),
+                                                      _ptr(out), _stream(stream)))
+    return out
+
+
+def h2o_q8_workspace_size(dims: H2ODims) -> int:
+    lib = load()
+    n = ctypes.c_size_t(0)
+    _check("h2o_q8_workspace_size", lib.h2o_q8_workspace_size(ctypes.byref(dims), ctypes.byref(n)))
+    return n.value
+
+
+def _expect_q8(k_codes, k_scales, v_codes, v_scales, B, Hkv, M, d, dev):
+    _expect(k_codes, "k_codes", (B, Hkv, M, d), torch.int8, dev)
+    _expect(v_codes, "v_codes", (B, Hkv, M, d), torch.int8, dev)
+    _expect(k_scales, "k_scales", (B, Hkv, M), torch.float32, dev)
+    _expect(v_scales, "v_scales", (B, Hkv, M), torch.float32, dev)
+
+
+def h2o_update_q8(scores, slot_pos, score_inc, k_new, v_new, k_codes, k_scales, v_codes,
+                  v_scales, pos0: int, recent_window: int, policy: str = "h2o", evict_idx=None,
+                  budget: int | None = None, stream=None):
+    """h2o_update_policy on 8-bit buffers, in place.  Returns evict_idx (B,Hkv,S)."""
+    lib = load()
+    dev = scores.device
+    B, Hkv, M = scores.shape
+    S, d = k_new.shape[2], k_new.shape[3]
+    Hq = score_inc.shape[1]
+    if policy not in POLICY:
+        raise ValueError(f"unknown policy {policy!r}")
+    _expect(scores, "scores", (B, Hkv, M), torch.float32, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    _expect(score_inc, "score_inc", (B, Hq, M + S), torch.float32, dev)
+    _expect(k_new, "k_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect(v_new, "v_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect_q8(k_codes, k_scales, v_codes, v_scales, B, Hkv, M, d, dev)
+    if evict_idx is None:
+        evict_idx = torch.empty((B, Hkv, S), dtype=torch.int32, device=dev)
+    _expect(evict_idx, "evict_idx", (B, Hkv, S), torch.int32, dev)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    st = lib.h2o_update_q8(ctypes.byref(dims), int(pos0), _ptr(scores), _ptr(slot_pos),
+                           _ptr(score_inc), _ptr(k_new), _ptr(v_new), _ptr(k_codes),
+                           _ptr(k_scales), _ptr(v_codes), _ptr(v_scales),
+                           int(M if budget is None else budget), int(recent_window),
+                           POLICY[policy], _ptr(evict_idx), _stream(stream))
+    _check("h2o_update_q8", st)
+    return evict_idx
+
+
+def h2o_evict_insert_q8(scores, slot_pos, k_new, v_new, k_codes, k_scales, v_codes, v_scales,
+                        pos0: int, recent_window: int, policy: str = "h2o", evict_idx=None,
+                        budget: int | None = None, Hq: int | None = None, stream=None):
+    """h2o_evict_insert on 8-bit buffers, in place.  Returns evict_idx (B,Hkv,S)."""
+    lib = load()
+    dev = scores.device
+    B, Hkv, M = scores.shape
+    S, d = k_new.shape[2], k_new.shape[3]
+    if policy not in POLICY:
+        raise ValueError(f"unknown policy {policy!r}")
+    _expect(scores, "scores", (B, Hkv, M), torch.float32, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    _expect(k_new, "k_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect(v_new, "v_new", (B, Hkv, S, d), torch.bfloat16, dev)
+    _expect_q8(k_codes, k_scales, v_codes, v_scales, B, Hkv, M, d, dev)
+    if evict_idx is None:
+        evict_idx = torch.empty((B, Hkv, S), dtype=torch.int32, device=dev)
+    _expect(evict_idx, "evict_idx", (B, Hkv, S), torch.int32, dev)
+    dims = H2ODims(B, Hkv if Hq is None else Hq, Hkv, d, S, M)
+    st = lib.h2o_evict_insert_q8(ctypes.byref(dims), int(pos0), _ptr(scores), _ptr(slot_pos),
+                                 _ptr(k_new), _ptr(v_new), _ptr(k_codes), _ptr(k_scales),
+                                 _ptr(v_codes), _ptr(v_scales),
+                                 int(M if budget is None else budget), int(recent_window),
+                                 POLICY[policy], _ptr(evict_idx), _stream(stream))
+    _check("h2o_evict_insert_q8", st)
+    return evict_idx
+
+
+def _sdpa_q8(fn, q, k_codes, k_scales, v_codes, v_scales, k_new, v_new, slot_pos, pos0, scale,
+             out, score_inc, workspace, stream):
+    lib = load()
+    dev = q.device
+    B, Hq, S, d = q.shape
+    Hkv, M = k_codes.shape[1], k_codes.shape[2]
+    bf = torch.bfloat16
+    cache_only = k_new is None
+    nk = M if cache_only else M + S
+    _expect(q, "q", (B, Hq, S, d), bf, dev)
+    _expect_q8(k_codes, k_scales, v_codes, v_scales, B, Hkv, M, d, dev)
+    _expect(slot_pos, "slot_pos", (B, Hkv, M), torch.int32, dev)
+    if not cache_only:
+        _expect(k_new, "k_new", (B, Hkv, S, d), bf, dev)
+        _expect(v_new, "v_new", (B, Hkv, S, d), bf, dev)
+    if out is None:
+        out = torch.empty((B, Hq, S, d), dtype=bf, device=dev)
+    if score_inc is None:
+        score_inc = torch.empty((B, Hq, nk), dtype=torch.float32, device=dev)
+    _expect(out, "out", (B, Hq, S, d), bf, dev)
+    _expect(score_inc, "score_inc", (B, Hq, nk), torch.float32, dev)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    if workspace is None:
+        n = h2o_q8_workspace_size(dims)
+        if n:
+            workspace = torch.empty(n, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    head = [ctypes.byref(dims), int(pos0), float(scale), _ptr(q), _ptr(k_codes), _ptr(k_scales),
+            _ptr(v_codes), _ptr(v_scales)]
+    mid = [] if cache_only else [_ptr(k_new), _ptr(v_new)]
+    st = getattr(lib, fn)(*head, *mid, _ptr(slot_pos), _ptr(out), _ptr(score_inc),
+                          _ptr(workspace), ws_bytes, _stream(stream))
+    _check(fn, st)
+    return out, score_inc
+
+
+def h2o_sdpa_chunk_q8(q, k_codes, k_scales, v_codes, v_scales, k_new, v_new, slot_pos,
+                      pos0: int, scale: float = 0.0, out=None, score_inc=None, workspace=None,
+                      stream=None):
+    """h2o_sdpa_chunk with the cache read through 8-bit buffers (k_new / v_new
+    bf16).  Returns (out (B,Hq,S,d) bf16, score_inc (B,Hq,M+S) f32)."""
+    return _sdpa_q8("h2o_sdpa_chunk_q8", q, k_codes, k_scales, v_codes, v_scales, k_new, v_new,
+                    slot_pos, pos0, scale, out, score_inc, workspace, stream)
+
+
+def h2o_sdpa_cache_q8(q, k_codes, k_scales, v_codes, v_scales, slot_pos, pos0: int,
+                      scale: float = 0.0, out=None, score_inc=None, workspace=None, stream=None):
+    """h2o_sdpa_cache with the cache read through 8-bit buffers.  Returns
+    (out (B,Hq,S,d) bf16, score_inc (B,Hq,M) f32)."""
+    return _sdpa_q8("h2o_sdpa_cache_q8", q, k_codes, k_scales, v_codes, v_scales, None, None,
+                    slot_pos, pos0, scale, out, score_inc, workspace, stream)

@@ -118,11 +118,14 @@ int check_dims(const h2o_dims_t* d) {
 
 // h2o_sdpa_chunk (cache_only = false: keys are the M slots, then the chunk's
 // S tokens) and h2o_sdpa_cache (cache_only = true: the M slots only, the
-// chunk's keys already written there; k_new / v_new unused).
+// chunk's keys already written there; k_new / v_new unused).  With q8 (the
+// 8-bit buffer calls) k_cache / v_cache are q8's bf16 read-back rows, filled
+// from the codes on the stream just before the attention kernels.
 int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
               const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
               const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out, float* score_inc,
-              void* workspace, size_t workspace_bytes, void* stream, bool cache_only) {
+              void* workspace, size_t workspace_bytes, void* stream, bool cache_only,
+              const Q8Buffers* q8 = nullptr) {
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
@@ -145,6 +148,12 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   DeviceInfo* di = nullptr;
   if ((st = current_device(&di)) != H2O_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the 8-bit buffers' rows, read back to bf16 ahead of the attention kernels
+  auto read_back = [&]() -> cudaError_t {
+    if (!q8) return cudaSuccess;
+    return launch_kv_dequantize(q8->k_codes, q8->k_scales, q8->k_rows, q8->v_codes, q8->v_scales,
+                                q8->v_rows, static_cast<int64_t>(D.B) * D.Hkv * D.M, D.d, s);
+  };
 
   if (decode) {
     // one query token per sequence: split-K kernels (h2o_decode.cu)
@@ -160,7 +169,8 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
     a.n_split = n_split;
     a.with_new = cache_only ? 0 : 1;
     a.nk = nk;
-    const cudaError_t e = launch_decode(a, s);
+    cudaError_t e = read_back();
+    if (e == cudaSuccess) e = launch_decode(a, s);
     return e == cudaSuccess ? H2O_OK : cuda_fail(e);
   }
   if ((st = get_encoder()) != H2O_OK) return st;
@@ -214,7 +224,9 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
     }
   }
   const size_t inc_bytes = static_cast<size_t>(G) * qg * static_cast<size_t>(nk) * sizeof(float);
-  cudaError_t e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
+  cudaError_t e = read_back();
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
   if (e != cudaSuccess) return cuda_fail(e);
   e = launch_sdpa(a, s);
   if (e != cudaSuccess) return cuda_fail(e);
@@ -222,16 +234,20 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
 }
 
 // h2o_update_policy (insert = false) and h2o_evict_insert (insert = true:
-// score_inc is not read and may be NULL).
+// score_inc is not read and may be NULL).  With q8 (the 8-bit buffer calls)
+// k_cache / v_cache are NULL: the update kernel writes scores, positions and
+// evict_idx (set to -1 first), then kv_scatter_q8 quantises the chunk's rows
+// into the chosen slots.
 int update_impl(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
                 const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
                 h2o_bf16* k_cache, h2o_bf16* v_cache, int32_t budget, int32_t recent_window,
-                int32_t policy, int32_t* evict_idx, void* stream, bool insert) {
+                int32_t policy, int32_t* evict_idx, void* stream, bool insert,
+                const Q8Buffers* q8 = nullptr) {
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
-  if (!scores || !slot_pos || (!insert && !score_inc) || !k_new || !v_new || !k_cache ||
-      !v_cache)
+  if (!scores || !slot_pos || (!insert && !score_inc) || !k_new || !v_new ||
+      (!q8 && (!k_cache || !v_cache)) || (q8 && !evict_idx))
     return H2O_ERR_NULL;
   if (misaligned(scores) || misaligned(slot_pos) || misaligned(score_inc) || misaligned(k_new) ||
       misaligned(v_new) || misaligned(k_cache) || misaligned(v_cache) ||
@@ -255,9 +271,79 @@ int update_impl(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* sl
   a.W = recent_window;
   a.policy = policy;
   a.insert = insert ? 1 : 0;
-  const cudaError_t e = launch_update(a, static_cast<cudaStream_t>(stream));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t n_idx = static_cast<size_t>(D.B) * D.Hkv * D.S;
+  cudaError_t e = cudaSuccess;
+  if (q8) e = cudaMemsetAsync(evict_idx, 0xFF, n_idx * sizeof(int32_t), s);  // -1: no slot
+  if (e == cudaSuccess) e = launch_update(a, s);
+  if (e == cudaSuccess && q8) {
+    Q8ScatterArgs qa;
+    qa.evict_idx = evict_idx; qa.k_new = k_new; qa.v_new = v_new; qa.buf = *q8;
+    qa.err = di->err_word;
+    qa.B = D.B; qa.Hkv = D.Hkv; qa.d = D.d; qa.S = D.S; qa.M = D.M;
+    e = launch_kv_scatter_q8(qa, s);
+  }
   if (e != cudaSuccess) return cuda_fail(e);
   return H2O_OK;
+}
+
+// Bytes of one tensor of bf16 rows read back from 8-bit buffers (256-aligned).
+size_t q8_rows_bytes(const h2o_dims_t& D) {
+  const size_t b = static_cast<size_t>(D.B) * D.Hkv * static_cast<size_t>(D.M) * D.d * 2;
+  return (b + 255) / 256 * 256;
+}
+
+bool q8_null(const int8_t* kc, const float* ks, const int8_t* vc, const float* vs) {
+  return !kc || !ks || !vc || !vs;
+}
+
+bool q8_misaligned(const int8_t* kc, const float* ks, const int8_t* vc, const float* vs) {
+  return misaligned(kc) || misaligned(ks) || misaligned(vc) || misaligned(vs);
+}
+
+// h2o_sdpa_chunk_q8 / h2o_sdpa_cache_q8: the head of the workspace takes the K
+// and V rows read back to bf16, the rest is the attention's own workspace.
+int sdpa_q8_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
+                 const int8_t* k_codes, const float* k_scales, const int8_t* v_codes,
+                 const float* v_scales, const h2o_bf16* k_new, const h2o_bf16* v_new,
+                 const int32_t* slot_pos, h2o_bf16* out, float* score_inc, void* workspace,
+                 size_t workspace_bytes, void* stream, bool cache_only) {
+  int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  const h2o_dims_t& D = *dims;
+  if (D.M > 0 && q8_null(k_codes, k_scales, v_codes, v_scales)) return H2O_ERR_NULL;
+  if (D.M > 0 && q8_misaligned(k_codes, k_scales, v_codes, v_scales)) return H2O_ERR_ALIGN;
+  size_t base = 0;
+  if ((st = h2o_workspace_size(dims, &base)) != H2O_OK) return st;
+  const size_t rows = D.M > 0 ? q8_rows_bytes(D) : 0;
+  const size_t need = 2 * rows + base;
+  if (need > 0 && (!workspace || workspace_bytes < need)) return H2O_ERR_WORKSPACE;
+  if (need > 0 && misaligned(workspace)) return H2O_ERR_ALIGN;
+  uint8_t* w = static_cast<uint8_t*>(workspace);
+  Q8Buffers b;
+  b.k_codes = const_cast<int8_t*>(k_codes); b.k_scales = const_cast<float*>(k_scales);
+  b.v_codes = const_cast<int8_t*>(v_codes); b.v_scales = const_cast<float*>(v_scales);
+  b.k_rows = rows ? reinterpret_cast<uint16_t*>(w) : nullptr;
+  b.v_rows = rows ? reinterpret_cast<uint16_t*>(w + rows) : nullptr;
+  return sdpa_impl(dims, pos0, softmax_scale, q, b.k_rows, b.v_rows, k_new, v_new, slot_pos, out,
+                   score_inc, base ? w + 2 * rows : nullptr, base ? workspace_bytes - 2 * rows : 0,
+                   stream, cache_only, rows ? &b : nullptr);
+}
+
+int update_q8_impl(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+                   const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
+                   int8_t* k_codes, float* k_scales, int8_t* v_codes, float* v_scales,
+                   int32_t budget, int32_t recent_window, int32_t policy, int32_t* evict_idx,
+                   void* stream, bool insert) {
+  const int st = check_dims(dims);
+  if (st != H2O_OK) return st;
+  if (q8_null(k_codes, k_scales, v_codes, v_scales)) return H2O_ERR_NULL;
+  if (q8_misaligned(k_codes, k_scales, v_codes, v_scales)) return H2O_ERR_ALIGN;
+  Q8Buffers b;
+  b.k_codes = k_codes; b.k_scales = k_scales; b.v_codes = v_codes; b.v_scales = v_scales;
+  b.k_rows = nullptr; b.v_rows = nullptr;
+  return update_impl(dims, pos0, scores, slot_pos, score_inc, k_new, v_new, nullptr, nullptr,
+                     budget, recent_window, policy, evict_idx, stream, insert, &b);
 }
 
 // Waits on an mbarrier nothing completes, with the bounded wait every kernel
@@ -472,6 +558,83 @@ int h2o_kv_restore(const h2o_dims_t* dims, const int32_t* index, const h2o_bf16*
   a.restore = 1;
   const cudaError_t e = launch_kv_rows(a, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_kv_quantize(int64_t n_rows, int32_t d, const h2o_bf16* x, int8_t* codes, float* scales,
+                    void* stream) {
+  if (n_rows < 0) return H2O_ERR_SHAPE;
+  if (d != 64 && d != 128) return H2O_ERR_UNSUPPORTED;
+  if (n_rows == 0) return H2O_OK;
+  if (!x || !codes || !scales) return H2O_ERR_NULL;
+  if (misaligned(x) || misaligned(codes) || misaligned(scales)) return H2O_ERR_ALIGN;
+  DeviceInfo* di = nullptr;
+  const int st = current_device(&di);
+  if (st != H2O_OK) return st;
+  const cudaError_t e = launch_kv_quantize(x, codes, scales, n_rows, d,
+                                           static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_kv_dequantize(int64_t n_rows, int32_t d, const int8_t* codes, const float* scales,
+                      h2o_bf16* x, void* stream) {
+  if (n_rows < 0) return H2O_ERR_SHAPE;
+  if (d != 64 && d != 128) return H2O_ERR_UNSUPPORTED;
+  if (n_rows == 0) return H2O_OK;
+  if (!x || !codes || !scales) return H2O_ERR_NULL;
+  if (misaligned(x) || misaligned(codes) || misaligned(scales)) return H2O_ERR_ALIGN;
+  DeviceInfo* di = nullptr;
+  const int st = current_device(&di);
+  if (st != H2O_OK) return st;
+  const cudaError_t e = launch_kv_dequantize(codes, scales, x, nullptr, nullptr, nullptr, n_rows,
+                                             d, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_q8_workspace_size(const h2o_dims_t* dims, size_t* bytes) {
+  const int st = h2o_workspace_size(dims, bytes);
+  if (st != H2O_OK) return st;
+  if (dims->M > 0) *bytes += 2 * q8_rows_bytes(*dims);
+  return H2O_OK;
+}
+
+int h2o_sdpa_chunk_q8(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                      const h2o_bf16* q, const int8_t* k_codes, const float* k_scales,
+                      const int8_t* v_codes, const float* v_scales, const h2o_bf16* k_new,
+                      const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out,
+                      float* score_inc, void* workspace, size_t workspace_bytes, void* stream) {
+  return sdpa_q8_impl(dims, pos0, softmax_scale, q, k_codes, k_scales, v_codes, v_scales, k_new,
+                      v_new, slot_pos, out, score_inc, workspace, workspace_bytes, stream, false);
+}
+
+int h2o_sdpa_cache_q8(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                      const h2o_bf16* q, const int8_t* k_codes, const float* k_scales,
+                      const int8_t* v_codes, const float* v_scales, const int32_t* slot_pos,
+                      h2o_bf16* out, float* score_inc, void* workspace, size_t workspace_bytes,
+                      void* stream) {
+  if (dims && dims->M < 1) return H2O_ERR_SHAPE;
+  return sdpa_q8_impl(dims, pos0, softmax_scale, q, k_codes, k_scales, v_codes, v_scales,
+                      nullptr, nullptr, slot_pos, out, score_inc, workspace, workspace_bytes,
+                      stream, true);
+}
+
+int h2o_update_q8(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+                  const float* score_inc, const h2o_bf16* k_new, const h2o_bf16* v_new,
+                  int8_t* k_codes, float* k_scales, int8_t* v_codes, float* v_scales,
+                  int32_t budget, int32_t recent_window, int32_t policy, int32_t* evict_idx,
+                  void* stream) {
+  return update_q8_impl(dims, pos0, scores, slot_pos, score_inc, k_new, v_new, k_codes, k_scales,
+                        v_codes, v_scales, budget, recent_window, policy, evict_idx, stream,
+                        false);
+}
+
+int h2o_evict_insert_q8(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
+                        const h2o_bf16* k_new, const h2o_bf16* v_new, int8_t* k_codes,
+                        float* k_scales, int8_t* v_codes, float* v_scales, int32_t budget,
+                        int32_t recent_window, int32_t policy, int32_t* evict_idx,
+                        void* stream) {
+  return update_q8_impl(dims, pos0, scores, slot_pos, nullptr, k_new, v_new, k_codes, k_scales,
+                        v_codes, v_scales, budget, recent_window, policy, evict_idx, stream,
+                        true);
 }
 
 int h2o_backward_workspace_size(const h2o_dims_t* dims, size_t* bytes) {

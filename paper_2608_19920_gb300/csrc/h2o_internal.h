@@ -119,6 +119,34 @@ struct ReplayArgs {
 
 cudaError_t launch_kv_rows(const ReplayArgs& a, cudaStream_t stream);
 
+// 8-bit K/V buffers (h2o_quant.cu): per cache row d int8 codes and one fp32
+// scale.  The q8 calls pass the buffers and, for the SDPA, the bf16 rows the
+// codes are read back into.
+struct Q8Buffers {
+  int8_t* k_codes;           // (B, Hkv, M, d)
+  float* k_scales;           // (B, Hkv, M)
+  int8_t* v_codes;
+  float* v_scales;
+  uint16_t* k_rows;          // SDPA only: (B, Hkv, M, d) bf16 read-back of the codes
+  uint16_t* v_rows;
+};
+
+struct Q8ScatterArgs {
+  const int32_t* evict_idx;  // (B, Hkv, S): slot of token c, -1 = none (left as it is)
+  const uint16_t* k_new;     // (B, Hkv, S, d) bf16
+  const uint16_t* v_new;
+  Q8Buffers buf;
+  int* err;
+  int B, Hkv, d, S, M;
+};
+
+cudaError_t launch_kv_quantize(const uint16_t* x, int8_t* codes, float* scales, int64_t n_rows,
+                               int d, cudaStream_t stream);
+cudaError_t launch_kv_dequantize(const int8_t* codes, const float* scales, uint16_t* x,
+                                 const int8_t* codes2, const float* scales2, uint16_t* x2,
+                                 int64_t n_rows, int d, cudaStream_t stream);
+cudaError_t launch_kv_scatter_q8(const Q8ScatterArgs& a, cudaStream_t stream);
+
 // h2o_sdpa_chunk_backward (h2o_backward.cu)
 struct BackwardArgs {
   const uint16_t* q;         // (B, Hq, S, d) bf16

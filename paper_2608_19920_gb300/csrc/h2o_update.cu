@@ -117,6 +117,8 @@ __device__ __forceinline__ uint32_t block_scan_bit(bool f, uint32_t* warp_tot, u
 
 __device__ __forceinline__ void copy_row(const UpdateArgs& a, int grp, int c, int e, int lane) {
   // 32 lanes: lanes 0-15 copy the K row, 16-31 the V row, in 16-byte pieces.
+  // No cache pointers: the rows are written by another kernel (8-bit buffers).
+  if (a.k_cache == nullptr) return;
   const int vec = a.d / 8;  // uint4 per row
   const bool is_v = lane >= 16;
   const int l = lane & 15;
@@ -490,7 +492,7 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   // every batch entry the cluster owns, 16-byte pieces, four loads in flight
   // per thread before their stores.
   const int n_sel = min(static_cast<int>((tot & 0xFFFFu) + min(tot >> 16, take_eq)), S);
-  const int rows = n_sel > rank ? (n_sel - 1 - rank) / C + 1 : 0;
+  const int rows = a.k_cache != nullptr && n_sel > rank ? (n_sel - 1 - rank) / C + 1 : 0;
   const int vecs = a.d / 8;  // 16-byte pieces per row
   const int per_b = rows * 2 * vecs;
   const int pieces = nb * per_b;

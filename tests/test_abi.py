@@ -203,3 +203,65 @@ def test_backward_argument_checks(lib):
 def test_selftest_limit_is_checked_on_the_host(lib):
     assert lib.h2o_selftest_bounded_wait(10, None) == ARG          # below 1 us
     assert lib.h2o_selftest_bounded_wait(10 ** 9, None) == ARG     # above 100 ms
+
+
+def test_q8_argument_checks(lib):
+    """The 8-bit buffer calls refuse bad arguments on the host (through the
+    binding's declared argument types), before any device work."""
+    vp = ctypes.c_void_p
+    p = vp(0x1000)
+    d = _dims()
+    qz = lambda n, dd, ptrs: lib.h2o_kv_quantize(n, dd, *ptrs, None)
+    dq = lambda n, dd, ptrs: lib.h2o_kv_dequantize(n, dd, *ptrs, None)
+    for f in (qz, dq):
+        assert f(-1, 64, [p] * 3) == SHAPE
+        assert f(4, 96, [p] * 3) == UNSUP
+        assert f(0, 64, [None] * 3) == OK        # nothing to do
+        assert f(4, 64, [p, None, p]) == NULL
+        assert f(4, 128, [p, vp(0x1001), p]) == ALIGN
+    n = ctypes.c_size_t(0)
+    assert lib.h2o_q8_workspace_size(ctypes.byref(d), ctypes.byref(n)) == OK
+    assert n.value == 2 * 2 * 256 * 64 * 2                  # K and V rows read back to bf16
+    assert lib.h2o_q8_workspace_size(ctypes.byref(_dims(M=0)), ctypes.byref(n)) == OK
+    assert n.value == 0
+    base = ctypes.c_size_t(0)
+    dd = _dims(S=1, M=100)
+    assert lib.h2o_workspace_size(ctypes.byref(dd), ctypes.byref(base)) == OK
+    assert lib.h2o_q8_workspace_size(ctypes.byref(dd), ctypes.byref(n)) == OK
+    assert n.value == base.value + 2 * ((2 * 100 * 64 * 2 + 255) // 256 * 256)
+
+    up = lambda dims, ptrs, ev=p, budget=256, W=32, policy=0: lib.h2o_update_q8(
+        ctypes.byref(dims), 256, *ptrs, budget, W, policy, ev, None)
+    ok9 = [p] * 9
+    assert up(d, ok9, ev=None) == NULL                       # evict_idx is required
+    assert up(d, ok9[:5] + [None] + ok9[6:]) == NULL         # k_codes
+    assert up(d, ok9[:6] + [vp(0x1004)] + ok9[7:]) == ALIGN  # k_scales
+    assert up(d, ok9, budget=255) == ARG
+    assert up(d, ok9, policy=7) == ARG
+    assert up(_dims(d=96), ok9) == UNSUP
+    ei = lambda dims, ptrs, ev=p, W=32: lib.h2o_evict_insert_q8(
+        ctypes.byref(dims), 256, *ptrs, 256, W, 0, ev, None)
+    ok8 = [p] * 8
+    assert ei(d, ok8, ev=None) == NULL
+    assert ei(d, ok8[:7] + [None]) == NULL                   # v_scales
+    assert ei(d, ok8[:4] + [vp(0x1008)] + ok8[5:]) == ALIGN  # k_codes
+    assert ei(d, ok8, W=257) == ARG
+    assert ei(_dims(S=300), ok8) == SHAPE
+
+    ws = ctypes.c_size_t(0)
+    assert lib.h2o_q8_workspace_size(ctypes.byref(d), ctypes.byref(ws)) == OK
+    ch = lambda dims, ptrs, w=p, wb=ws.value, pos0=256: lib.h2o_sdpa_chunk_q8(
+        ctypes.byref(dims), pos0, 0.0, *ptrs, w, wb, None)
+    ok10 = [p] * 10
+    assert ch(d, ok10, w=None) == WORKSPACE
+    assert ch(d, ok10, wb=ws.value - 1) == WORKSPACE
+    assert ch(d, ok10, w=vp(0x1004)) == ALIGN
+    assert ch(d, [p, None] + ok10[2:]) == NULL               # k_codes
+    assert ch(d, ok10[:3] + [vp(0x100c)] + ok10[4:]) == ALIGN  # v_codes
+    assert ch(d, [None] + ok10[1:]) == NULL                  # q, checked by the attention
+    assert ch(d, ok10, pos0=-1) == ARG
+    ca = lambda dims, ptrs, w=p, wb=ws.value: lib.h2o_sdpa_cache_q8(
+        ctypes.byref(dims), 256, 0.0, *ptrs, w, wb, None)
+    assert ca(_dims(M=0), [p] * 8, w=None, wb=0) == SHAPE
+    assert ca(d, [p] * 8, w=None) == WORKSPACE
+    assert ca(d, [p] * 4 + [None] + [p] * 3) == NULL         # v_scales

@@ -402,7 +402,8 @@ def run_ours(args, w):
         "tflops_frac_of_peak": alg_tflops / pk["bf16_sus"],
         "chunk_step_ms_median": statistics.median(chunk_step_ms) if chunk_step_ms else None,
         "gpu_launches": args.steps * sum(launches_per_chunk(e - p, w.M, args.order,
-                                                            args.kv_bits) for p, e in plan),
+                                                            args.kv_bits, w.Hq // w.Hkv)
+                                         for p, e in plan),
         "clocks": clocks,
     }
     # the chunk SDPA is timed on its own (launch after launch, L2 flushed in
@@ -415,8 +416,8 @@ def run_ours(args, w):
         # decode: K and V read once per step, HBM bound
         line["roofline"] = {
             "bound": "hbm",
-            "kernel": ("kv_dequantize_kernel + " if args.kv_bits == 8 else "") +
-                      "decode_split_kernel + decode_combine_kernel (one step)",
+            "kernel": "decode_split_kernel" + ("<8-bit rows>" if args.kv_bits == 8 else "") +
+                      " + decode_combine_kernel (one step)",
             "achieved": kern["gbs"], "peak": pk["hbm"], "unit": "GB/s",
             "frac": kern["gbs"] / pk["hbm"], "traffic": traffic,
             "peak_source": f"{pk['source']} HBM copy bandwidth",
@@ -521,13 +522,16 @@ def decode_kv_bytes(w, kv_bits: int = 16):
     return 2.0 * w.B * w.Hkv * w.M * row
 
 
-def launches_per_chunk(S, M, order="chunk", kv_bits=16):
+def launches_per_chunk(S, M, order="chunk", kv_bits=16, qg=4):
     """Kernels of this library one chunk launches: the SDPA (split + combine
     when S = 1 and a cache exists) and the update (the paper's order: the
     eviction-insert, the SDPA and the score addition); 8-bit buffers add the
-    read-back before the SDPA and the quantising scatter after the update."""
-    sdpa = 2 if S == 1 and M > 0 else 1
-    return sdpa + (2 if order == "paper" else 1) + (2 if kv_bits == 8 else 0)
+    quantising scatter after the update and, where the chunk kernel runs, the
+    read-back before it (the decode kernels read the codes themselves)."""
+    decode = S == 1 and M > 0 and qg <= 8
+    sdpa = 2 if decode else 1
+    q8 = (1 + (0 if decode or M == 0 else 1)) if kv_bits == 8 else 0
+    return sdpa + (2 if order == "paper" else 1) + q8
 
 
 def executed_mma_flops(w, S):

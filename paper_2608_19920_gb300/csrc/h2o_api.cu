@@ -119,8 +119,9 @@ int check_dims(const h2o_dims_t* d) {
 // h2o_sdpa_chunk (cache_only = false: keys are the M slots, then the chunk's
 // S tokens) and h2o_sdpa_cache (cache_only = true: the M slots only, the
 // chunk's keys already written there; k_new / v_new unused).  With q8 (the
-// 8-bit buffer calls) k_cache / v_cache are q8's bf16 read-back rows, filled
-// from the codes on the stream just before the attention kernels.
+// 8-bit buffer calls) the decode kernels read the codes themselves; the chunk
+// kernel reads k_cache / v_cache = q8's bf16 read-back rows, filled from the
+// codes on the stream just before it.
 int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
               const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
               const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out, float* score_inc,
@@ -130,7 +131,8 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
   if (!q || !out || !score_inc || (!cache_only && (!k_new || !v_new))) return H2O_ERR_NULL;
-  if (D.M > 0 && (!k_cache || !v_cache || !slot_pos)) return H2O_ERR_NULL;
+  // (q8: the codes were checked by the caller; the decode kernels need no rows)
+  if (D.M > 0 && ((!q8 && (!k_cache || !v_cache)) || !slot_pos)) return H2O_ERR_NULL;
   if (misaligned(q) || misaligned(k_new) || misaligned(v_new) || misaligned(out) ||
       misaligned(score_inc) || (D.M > 0 && (misaligned(k_cache) || misaligned(v_cache) ||
                                             misaligned(slot_pos))))
@@ -157,7 +159,7 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
 
   if (decode) {
     // one query token per sequence: split-K kernels (h2o_decode.cu)
-    DecodeArgs a;
+    DecodeArgs a{};
     a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
     a.slot_pos = slot_pos; a.out = out; a.score_inc = score_inc;
     a.part = static_cast<float*>(workspace);
@@ -169,8 +171,12 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
     a.n_split = n_split;
     a.with_new = cache_only ? 0 : 1;
     a.nk = nk;
-    cudaError_t e = read_back();
-    if (e == cudaSuccess) e = launch_decode(a, s);
+    a.q8 = q8 ? 1 : 0;
+    a.k_codes = q8 ? q8->k_codes : nullptr;
+    a.k_scales = q8 ? q8->k_scales : nullptr;
+    a.v_codes = q8 ? q8->v_codes : nullptr;
+    a.v_scales = q8 ? q8->v_scales : nullptr;
+    const cudaError_t e = launch_decode(a, s);
     return e == cudaSuccess ? H2O_OK : cuda_fail(e);
   }
   if ((st = get_encoder()) != H2O_OK) return st;
@@ -287,8 +293,13 @@ int update_impl(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* sl
   return H2O_OK;
 }
 
-// Bytes of one tensor of bf16 rows read back from 8-bit buffers (256-aligned).
+// Bytes of one tensor of bf16 rows read back from 8-bit buffers (256-aligned);
+// none when the decode kernels run (they read the codes themselves).
 size_t q8_rows_bytes(const h2o_dims_t& D) {
+  int split_len = 0, n_split = 0;
+  size_t ws = 0;
+  if (D.M == 0 || decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws))
+    return 0;
   const size_t b = static_cast<size_t>(D.B) * D.Hkv * static_cast<size_t>(D.M) * D.d * 2;
   return (b + 255) / 256 * 256;
 }
@@ -315,7 +326,7 @@ int sdpa_q8_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, cons
   if (D.M > 0 && q8_misaligned(k_codes, k_scales, v_codes, v_scales)) return H2O_ERR_ALIGN;
   size_t base = 0;
   if ((st = h2o_workspace_size(dims, &base)) != H2O_OK) return st;
-  const size_t rows = D.M > 0 ? q8_rows_bytes(D) : 0;
+  const size_t rows = q8_rows_bytes(D);
   const size_t need = 2 * rows + base;
   if (need > 0 && (!workspace || workspace_bytes < need)) return H2O_ERR_WORKSPACE;
   if (need > 0 && misaligned(workspace)) return H2O_ERR_ALIGN;
@@ -327,7 +338,7 @@ int sdpa_q8_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, cons
   b.v_rows = rows ? reinterpret_cast<uint16_t*>(w + rows) : nullptr;
   return sdpa_impl(dims, pos0, softmax_scale, q, b.k_rows, b.v_rows, k_new, v_new, slot_pos, out,
                    score_inc, base ? w + 2 * rows : nullptr, base ? workspace_bytes - 2 * rows : 0,
-                   stream, cache_only, rows ? &b : nullptr);
+                   stream, cache_only, D.M > 0 ? &b : nullptr);
 }
 
 int update_q8_impl(const h2o_dims_t* dims, int64_t pos0, float* scores, int32_t* slot_pos,
@@ -448,7 +459,7 @@ int h2o_sdpa_decode_static(const h2o_dims_t* dims, int64_t pos0, float softmax_s
   if (ss.status != cudaSuccess) return cuda_fail(ss.status);
 
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
-  DecodeArgs a;
+  DecodeArgs a{};
   a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
   a.slot_pos = slot_pos; a.out = out; a.score_inc = score_inc;
   a.part = static_cast<float*>(ss.ptr);
@@ -593,7 +604,7 @@ int h2o_kv_dequantize(int64_t n_rows, int32_t d, const int8_t* codes, const floa
 int h2o_q8_workspace_size(const h2o_dims_t* dims, size_t* bytes) {
   const int st = h2o_workspace_size(dims, bytes);
   if (st != H2O_OK) return st;
-  if (dims->M > 0) *bytes += 2 * q8_rows_bytes(*dims);
+  *bytes += 2 * q8_rows_bytes(*dims);
   return H2O_OK;
 }
 

@@ -43,13 +43,41 @@ constexpr int kDecTileBytes = 16384;
 constexpr int kCombineThreads = 256;
 constexpr int kCombineCols = 4096;  // score_inc columns normalised per combine CTA
 
-template <int D>
+template <int D, bool Q8 = false>
 struct DecGeom {
-  static constexpr int kRowBytes = D * 2;
-  static constexpr int kTileKeys = kDecTileBytes / kRowBytes;  // 64 (d = 128) or 128
+  static constexpr int kRowBytes = Q8 ? D : D * 2;             // a cache row in the ring
+  static constexpr int kTileKeys = kDecTileBytes / kRowBytes;  // bf16: 64 (d = 128) or 128;
+                                                               // 8-bit: 128 or 256
+  // A ring slot holds kTileKeys rows, or (8-bit) up to kTileKeys - 1 code rows
+  // followed by the new token's bf16 row (2 D bytes) when that token ends the item.
+  static constexpr int kSlotBytes = kDecTileBytes + (Q8 ? D : 0);
   static constexpr int kCh = D / 64;                           // 16-byte chunks per lane in Q K^T
   static constexpr int kVe = D / 32;                           // value elements per lane in P V
 };
+
+// Two 8-bit codes of a cache row, read back as the 8-bit format defines:
+// bf16(code * scale), returned as fp32.  `wb` holds four codes with their sign
+// bits flipped (code + 128 as unsigned bytes); byte i of it is placed under the
+// exponent of 2^23, so the float is 2^23 + 128 + code exactly, and subtracting
+// 2^23 + 128 leaves the code.  The product and its rounding are those of the
+// read-back kernel (fp32 multiply, then round to nearest even bf16).
+__device__ __forceinline__ float2 q8_pair(uint32_t wb, int i, float2 s2) {
+  const float lo = __uint_as_float(__byte_perm(wb, 0x4B000000u, 0x7650u | i));
+  const float hi = __uint_as_float(__byte_perm(wb, 0x4B000000u, 0x7650u | (i + 1)));
+  const float2 c = __fadd2_rn(make_float2(lo, hi), make_float2(-8388736.f, -8388736.f));
+  const float2 x = __fmul2_rn(c, s2);
+  const uint32_t p = pack_bf16x2(x.x, x.y);
+  return make_float2(__uint_as_float(p << 16), __uint_as_float(p & 0xFFFF0000u));
+}
+
+// Floats of the region that holds the warps' partial outputs at the end of an
+// item and, with 8-bit buffers, the split's K and V scales before that.
+template <int D, int QG, bool Q8>
+__host__ __device__ constexpr int red_region_floats(int split_len) {
+  const int o = kDecWarps * QG * D;
+  const int sc = Q8 ? (2 * (split_len + 1) + 3) / 4 * 4 : 0;
+  return o > sc ? o : sc;
+}
 
 struct alignas(16) DecHead {  // 16-byte size: the logits after it are read as float4
   uint64_t full[kDecStages];
@@ -121,7 +149,7 @@ struct DecItem {
   bool last;
 };
 
-template <int D>
+template <int D, bool Q8>
 __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int it) {
   DecItem x;
   x.grp = it / a.n_split;
@@ -130,7 +158,7 @@ __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int it) {
   x.n_cache = min(a.split_len, a.M - x.j0);  // >= 1: n_split = ceil(M / split_len)
   x.last = x.s == a.n_split - 1 && a.with_new;  // this item also takes the new token
   x.n_loc = x.n_cache + (x.last ? 1 : 0);        // local key n_cache is the new token
-  x.n_tiles = (x.n_loc + DecGeom<D>::kTileKeys - 1) / DecGeom<D>::kTileKeys;
+  x.n_tiles = (x.n_loc + DecGeom<D, Q8>::kTileKeys - 1) / DecGeom<D, Q8>::kTileKeys;
   return x;
 }
 
@@ -154,18 +182,22 @@ __device__ __forceinline__ void block_reduce_qg(float (&v)[QG], float (*red)[kDe
     for (int g = 0; g < QG; ++g) red[warp][g] = v[g];
 }
 
-template <int D, int QG>
+template <int D, int QG, bool Q8>
 __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
     decode_split_kernel(const DecodeArgs a) {
-  using G = DecGeom<D>;
+  using G = DecGeom<D, Q8>;
   extern __shared__ __align__(128) uint8_t dsm[];
   uint8_t* ring = dsm;
-  DecHead& hd = *reinterpret_cast<DecHead*>(dsm + kDecStages * kDecTileBytes);
+  static_assert(G::kSlotBytes % 16 == 0, "ring slots must stay 16-byte aligned");
+  DecHead& hd = *reinterpret_cast<DecHead*>(dsm + kDecStages * G::kSlotBytes);
   static_assert(sizeof(DecHead) % 16 == 0, "logits must stay 16-byte aligned");
-  float* lg = reinterpret_cast<float*>(dsm + kDecStages * kDecTileBytes + sizeof(DecHead));
+  float* lg = reinterpret_cast<float*>(dsm + kDecStages * G::kSlotBytes + sizeof(DecHead));
   float* red_o = lg + (a.split_len + 1) * QG;  // [warp][g][D]
+  // 8-bit buffers: the item's K and V scales, in red_o's space until P V ends
+  float* ksc = red_o;
+  float* vsc = red_o + (a.split_len + 1);
   // q rows of the item whose first K tile sits in ring slot x: qbuf + x * QG * D
-  uint16_t* qbuf = reinterpret_cast<uint16_t*>(red_o + kDecWarps * QG * D);
+  uint16_t* qbuf = reinterpret_cast<uint16_t*>(red_o + red_region_floats<D, QG, Q8>(a.split_len));
 
   const int tid = threadIdx.x, warp = tid >> 5;
   const uint32_t lane = static_cast<uint32_t>(tid & 31);
@@ -185,7 +217,7 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
   int issued = 0;
   int p_it = blockIdx.x, p_t = 0;
   DecItem p_x;
-  if (p_it < n_items) p_x = dec_item<D>(a, p_it);
+  if (p_it < n_items) p_x = dec_item<D, Q8>(a, p_it);
   auto issue_next = [&]() {
     if (p_it >= n_items) return;
     const bool is_v = p_t >= p_x.n_tiles;
@@ -193,29 +225,34 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
     const int k1 = min(k0 + G::kTileKeys, p_x.n_loc);
     const int rows_c = max(0, min(k1, p_x.n_cache) - k0);
     const bool has_new = p_x.last && k1 > p_x.n_cache;
-    uint8_t* dst = ring + (issued % kDecStages) * kDecTileBytes;
+    uint8_t* dst = ring + (issued % kDecStages) * G::kSlotBytes;
     uint64_t* bar = &hd.full[issued % kDecStages];
     const uint32_t q_bytes = p_t == 0 ? static_cast<uint32_t>(a.qg * D * 2) : 0u;
-    bar_expect_tx(bar, static_cast<uint32_t>((rows_c + (has_new ? 1 : 0)) * G::kRowBytes) + q_bytes);
+    // the new token's row is bf16 (2 D bytes) in both layouts
+    bar_expect_tx(bar, static_cast<uint32_t>(rows_c * G::kRowBytes + (has_new ? 2 * D : 0)) +
+                           q_bytes);
     if (q_bytes) {
       const int pb = p_x.grp / a.Hkv, ph = p_x.grp % a.Hkv;
       bulk_load_once(qbuf + (issued % kDecStages) * QG * D,
                      a.q + static_cast<size_t>(pb * a.Hq + ph * a.qg) * D, q_bytes, bar);
     }
     if (rows_c > 0) {
-      const uint16_t* base = (is_v ? a.v_cache : a.k_cache) +
-                             (static_cast<size_t>(p_x.grp) * a.M + p_x.j0 + k0) * D;
+      const size_t row0 = static_cast<size_t>(p_x.grp) * a.M + p_x.j0 + k0;
+      const void* base;
+      if constexpr (Q8)
+        base = (is_v ? a.v_codes : a.k_codes) + row0 * D;
+      else
+        base = (is_v ? a.v_cache : a.k_cache) + row0 * D;
       bulk_load_once(dst, base, static_cast<uint32_t>(rows_c * G::kRowBytes), bar);
     }
     if (has_new)
       bulk_load_once(dst + rows_c * G::kRowBytes,
-                     (is_v ? a.v_new : a.k_new) + static_cast<size_t>(p_x.grp) * D, G::kRowBytes,
-                     bar);
+                     (is_v ? a.v_new : a.k_new) + static_cast<size_t>(p_x.grp) * D, 2 * D, bar);
     ++issued;
     if (++p_t == 2 * p_x.n_tiles) {
       p_t = 0;
       p_it += gridDim.x;
-      if (p_it < n_items) p_x = dec_item<D>(a, p_it);
+      if (p_it < n_items) p_x = dec_item<D, Q8>(a, p_it);
     }
   };
   if (tid == 0)
@@ -228,7 +265,7 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
   int g_t = 0;  // tiles consumed so far (ring slot and phase)
 
   for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
-    const DecItem x = dec_item<D>(a, it);
+    const DecItem x = dec_item<D, Q8>(a, it);
     const int b = x.grp / a.Hkv, h = x.grp % a.Hkv;
     const size_t row0 = static_cast<size_t>(b * a.Hq + h * a.qg);  // first query head's row
 
@@ -240,12 +277,20 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
       const int k = tid + u * kDecThreads;
       pos[u] = k < x.n_cache ? __ldg(sp + k) : 0;
     }
+    if constexpr (Q8) {  // the item's row scales, read in Q K^T and P V
+      const size_t sc0 = static_cast<size_t>(x.grp) * a.M + x.j0;
+      for (int k = tid; k < x.n_cache; k += kDecThreads) {
+        ksc[k] = __ldg(a.k_scales + sc0 + k);
+        vsc[k] = __ldg(a.v_scales + sc0 + k);
+      }
+      __syncthreads();
+    }
     // ---- Q K^T: raw dot products of the item's keys into lg
     float2 qr[QG][4 * G::kCh];  // this lane's slice of every head's query, element pairs
     for (int t = 0; t < x.n_tiles; ++t, ++g_t) {
       if (wait_bar(&hd.full[g_t % kDecStages], (g_t / kDecStages) & 1, abort_flag,
                    kWaitLimitNs)) {
-        const uint8_t* tile = ring + (g_t % kDecStages) * kDecTileBytes;
+        const uint8_t* tile = ring + (g_t % kDecStages) * G::kSlotBytes;
         if (t == 0) {  // the q rows arrived with this tile; read before its slot is reissued
           const uint16_t* qs = qbuf + (g_t % kDecStages) * QG * D;
 #pragma unroll
@@ -253,8 +298,11 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
 #pragma unroll
             for (int ch = 0; ch < G::kCh; ++ch) {
               float f[8];
+              // bf16 rows: chunks c0 and c0 + 8; 8-bit rows: the contiguous
+              // chunks kCh c0 .. kCh c0 + kCh - 1 (the lane's code bytes)
+              const int qc = Q8 ? G::kCh * c0 + ch : c0 + 8 * ch;
               if (g < a.qg) {
-                bf16x8_to_f32(reinterpret_cast<const uint4*>(qs + g * D)[c0 + 8 * ch], f);
+                bf16x8_to_f32(reinterpret_cast<const uint4*>(qs + g * D)[qc], f);
               } else {
 #pragma unroll
                 for (int e = 0; e < 8; ++e) f[e] = 0.f;
@@ -273,11 +321,36 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
           float2 d2[QG];
 #pragma unroll
           for (int g = 0; g < QG; ++g) d2[g] = make_float2(0.f, 0.f);
-          if (kl < x.n_loc) {
+          // the new token's row is bf16 in both layouts (8-bit: it follows the
+          // tile's code rows, at the offset its key index gives)
+          const bool code_row = Q8 && !(x.last && kl == x.n_cache);
+          if (kl < x.n_loc && code_row) {
+            const uint8_t* crow = tile + kk * G::kRowBytes;
+            const float sk = ksc[kl];
+            const float2 s2 = make_float2(sk, sk);
+            uint32_t w[2 * G::kCh];  // this lane's codes (elements kCh 8 c0 ..), sign-flipped
+            if constexpr (D == 128) {
+              const uint4 u = *reinterpret_cast<const uint4*>(crow + 16 * c0);
+              w[0] = u.x; w[1] = u.y; w[2] = u.z; w[3] = u.w;
+            } else {
+              const uint2 u = *reinterpret_cast<const uint2*>(crow + 8 * c0);
+              w[0] = u.x; w[1] = u.y;
+            }
+#pragma unroll
+            for (int x2 = 0; x2 < 2 * G::kCh; ++x2) w[x2] ^= 0x80808080u;
+#pragma unroll
+            for (int ch = 0; ch < G::kCh; ++ch)
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 kf = q8_pair(w[2 * ch + (e >> 1)], 2 * (e & 1), s2);
+#pragma unroll
+                for (int g = 0; g < QG; ++g) d2[g] = __ffma2_rn(qr[g][4 * ch + e], kf, d2[g]);
+              }
+          } else if (kl < x.n_loc) {
             const uint4* krow = reinterpret_cast<const uint4*>(tile + kk * G::kRowBytes);
 #pragma unroll
             for (int ch = 0; ch < G::kCh; ++ch) {
-              const uint4 u = krow[c0 + 8 * ch];
+              const uint4 u = krow[Q8 ? G::kCh * c0 + ch : c0 + 8 * ch];
               const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
@@ -370,7 +443,7 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
     for (int t = 0; t < x.n_tiles; ++t, ++g_t) {
       if (wait_bar(&hd.full[g_t % kDecStages], (g_t / kDecStages) & 1, abort_flag,
                    kWaitLimitNs)) {
-        const uint8_t* tile = ring + (g_t % kDecStages) * kDecTileBytes;
+        const uint8_t* tile = ring + (g_t % kDecStages) * G::kSlotBytes;
         const int k0 = t * G::kTileKeys;
         const int kend = min(G::kTileKeys, x.n_loc - k0);
 #pragma unroll 2
@@ -385,7 +458,23 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
             p[g4 + 3] = pv.w;
           }
           float2 vf[G::kVe / 2];
-          if constexpr (D == 128) {
+          if (Q8 && !(x.last && k0 + kk == x.n_cache)) {  // a code row (the warp's key)
+            const float sv = vsc[k0 + kk];
+            const float2 s2 = make_float2(sv, sv);
+            if constexpr (D == 128) {
+              const uint32_t wb =
+                  *reinterpret_cast<const uint32_t*>(tile + kk * G::kRowBytes + lane * 4) ^
+                  0x80808080u;
+              vf[0] = q8_pair(wb, 0, s2);
+              vf[G::kVe / 2 - 1] = q8_pair(wb, 2, s2);
+            } else {
+              const uint32_t wb =
+                  static_cast<uint32_t>(
+                      *reinterpret_cast<const uint16_t*>(tile + kk * G::kRowBytes + lane * 2)) ^
+                  0x8080u;
+              vf[0] = q8_pair(wb, 0, s2);
+            }
+          } else if constexpr (D == 128) {
             const uint2 uu = *reinterpret_cast<const uint2*>(tile + kk * G::kRowBytes + lane * 8);
             vf[0] = make_float2(__uint_as_float(uu.x << 16), __uint_as_float(uu.x & 0xFFFF0000u));
             vf[1] = make_float2(__uint_as_float(uu.y << 16), __uint_as_float(uu.y & 0xFFFF0000u));
@@ -521,30 +610,30 @@ __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const D
   for (int j = c0 + tid; j < c1; j += kCombineThreads) inc[j] = fast_exp2(inc[j] - lam);
 }
 
-template <int D, int QG>
+template <int D, int QG, bool Q8>
 constexpr size_t split_smem(int split_len) {
-  return kDecStages * kDecTileBytes + sizeof(DecHead) +
+  return kDecStages * DecGeom<D, Q8>::kSlotBytes + sizeof(DecHead) +
          static_cast<size_t>(split_len + 1) * QG * sizeof(float) +
-         static_cast<size_t>(kDecWarps) * QG * D * sizeof(float) +
+         static_cast<size_t>(red_region_floats<D, QG, Q8>(split_len)) * sizeof(float) +
          static_cast<size_t>(kDecStages) * QG * D * sizeof(uint16_t);
 }
 
-template <int D, int QG>
+template <int D, int QG, bool Q8>
 cudaError_t launch_split(const DecodeArgs& a, cudaStream_t stream) {
   // Persistent grid: as many CTAs as fit on the GPU at once (sized once per
   // device for the largest split), each taking every gridDim-th work item.
-  static int resident[64] = {};
+  static int resident[64] = {};  // one table per instantiation
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   int n_res = dev < 64 ? resident[dev] : 0;
   if (n_res == 0) {
-    const int smem_max = static_cast<int>(split_smem<D, QG>(kDecodeMaxSplitLen));
-    e = cudaFuncSetAttribute(decode_split_kernel<D, QG>,
+    const int smem_max = static_cast<int>(split_smem<D, QG, Q8>(kDecodeMaxSplitLen));
+    e = cudaFuncSetAttribute(decode_split_kernel<D, QG, Q8>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
     if (e != cudaSuccess) return e;
     int per_sm = 0, sms = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_split_kernel<D, QG>,
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_split_kernel<D, QG, Q8>,
                                                       kDecThreads, smem_max);
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -553,14 +642,18 @@ cudaError_t launch_split(const DecodeArgs& a, cudaStream_t stream) {
     if (dev < 64) resident[dev] = n_res;
   }
   const int n_items = a.n_split * a.B * a.Hkv;
-  const size_t smem = split_smem<D, QG>(a.split_len);
-  decode_split_kernel<D, QG><<<std::min(n_items, n_res), kDecThreads, smem, stream>>>(a);
+  const size_t smem = split_smem<D, QG, Q8>(a.split_len);
+  decode_split_kernel<D, QG, Q8><<<std::min(n_items, n_res), kDecThreads, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
 template <int D>
 cudaError_t launch_d(const DecodeArgs& a, cudaStream_t stream) {
-  cudaError_t e = a.qg <= 4 ? launch_split<D, 4>(a, stream) : launch_split<D, 8>(a, stream);
+  cudaError_t e;
+  if (a.q8)
+    e = a.qg <= 4 ? launch_split<D, 4, true>(a, stream) : launch_split<D, 8, true>(a, stream);
+  else
+    e = a.qg <= 4 ? launch_split<D, 4, false>(a, stream) : launch_split<D, 8, false>(a, stream);
   if (e != cudaSuccess) return e;
   const dim3 grid(static_cast<unsigned>(a.B * a.Hq),
                   static_cast<unsigned>((a.nk + kCombineCols - 1) / kCombineCols));

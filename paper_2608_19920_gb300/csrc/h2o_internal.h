@@ -86,6 +86,13 @@ struct DecodeArgs {
   int n_split;              // ceil(M / split_len); the last split also takes the new token
   int with_new;             // 1: the new token is key column M; 0: h2o_sdpa_cache (none)
   int nk;                   // score_inc row length: M + with_new
+  // 8-bit buffers (q8 = 1): the cache rows are int8 codes with a float32 scale
+  // per row, read as bf16(code * scale); k_cache / v_cache are then unused
+  int q8;
+  const int8_t* k_codes;    // (B, Hkv, M, d)
+  const float* k_scales;    // (B, Hkv, M)
+  const int8_t* v_codes;
+  const float* v_scales;
 };
 
 // Split of the M cache slots for the decode kernels (a function of the sizes

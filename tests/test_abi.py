@@ -228,7 +228,7 @@ def test_q8_argument_checks(lib):
     dd = _dims(S=1, M=100)
     assert lib.h2o_workspace_size(ctypes.byref(dd), ctypes.byref(base)) == OK
     assert lib.h2o_q8_workspace_size(ctypes.byref(dd), ctypes.byref(n)) == OK
-    assert n.value == base.value + 2 * ((2 * 100 * 64 * 2 + 255) // 256 * 256)
+    assert n.value == base.value       # S = 1: the decode kernels read the codes themselves
 
     up = lambda dims, ptrs, ev=p, budget=256, W=32, policy=0: lib.h2o_update_q8(
         ctypes.byref(dims), 256, *ptrs, budget, W, policy, ev, None)

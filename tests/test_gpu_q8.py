@@ -1,7 +1,8 @@
 """GPU parity of the 8-bit K/V buffer calls against the oracle (oracle/quant.py),
 through the C ABI, on the same seeded inputs: the quantiser, the read-back and
 the q8 updates bit for bit (codes, scales, scores, positions, evict_idx); the
-q8 SDPA calls within the SDPA tolerances of the bf16 calls."""
+q8 SDPA calls within the SDPA tolerances of the bf16 calls (S = 1: the decode
+kernels reading the codes; S > 1: the read-back, then the chunk kernel)."""
 import numpy as np
 import pytest
 import torch
@@ -154,6 +155,9 @@ SDPA_CASES = [
     (2, 8, 2, 128, 20, 300, 900, True),       # paper order: the cache only
     (1, 32, 8, 128, 512, 4096, 8192, True),
     (2, 6, 3, 64, 1, 130, 140, True),         # S = 1, d = 64
+    (1, 4, 1, 128, 1, 255, 300, False),       # S = 1: a ring slot of 127 code rows + the new bf16 row
+    (2, 16, 2, 64, 1, 777, 900, False),       # S = 1, q_g = 8, d = 64
+    (1, 8, 1, 128, 1, 1537, 1600, True),      # S = 1, q_g = 8, a last tile of one code row
 ]
 
 

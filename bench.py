@@ -270,6 +270,8 @@ def run_reference(args, w):
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d,
                        "T": w.T, "S": w.S, "M": w.M, "W": w.W,
+                       "kv_buffers": ("int8 codes + fp32 row scales" if args.kv_bits == 8
+                                      else "bf16"),
                        "step": "one steady-state chunk step per step (CPU sample)"},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(),
                              "kind": "oracle",

@@ -54,3 +54,24 @@ def test_flop_accounting():
     assert len(chunks) == 56
     assert abs(chunks[0] - 4 * 32 * 128 * 512 * (4096 + 256.5)) < 1
     assert abs(pre - 4 * 32 * 128 * 4096 * (4096 + 1) / 2) < 1
+
+
+def test_launch_and_byte_accounting():
+    """gpu_launches counts this library's kernels per chunk; decode bytes are
+    the K and V rows read once (8-bit rows: d codes + a 4-byte scale)."""
+    import bench
+    lpc = bench.launches_per_chunk
+    assert lpc(512, 4096) == 2                      # SDPA + update
+    assert lpc(512, 4096, "paper") == 3             # evict-insert + SDPA + scores_add
+    assert lpc(1, 4096) == 3                        # split + combine + update
+    assert lpc(1, 4096, "paper") == 4
+    assert lpc(1, 4096, "chunk", 16, 16) == 2       # q_g > 8: the chunk kernel
+    assert lpc(512, 4096, "chunk", 8) == 4          # + read-back + quantising scatter
+    assert lpc(4096, 4096, "chunk", 8) == 4         # the prefill
+    assert lpc(512, 4096, "paper", 8) == 5
+    assert lpc(1, 4096, "chunk", 8) == 4            # the decode kernels read the codes
+    assert lpc(1, 4096, "paper", 8) == 5
+    assert lpc(1, 4096, "chunk", 8, 16) == 4        # q_g > 8: read-back + chunk kernel
+    w = bench.wl.WORKLOADS["decode_64k"]
+    assert bench.decode_kv_bytes(w) == 2 * 8 * 8 * 65536 * 256
+    assert bench.decode_kv_bytes(w, 8) == 2 * 8 * 8 * 65536 * 132

@@ -80,7 +80,7 @@ enum {
   H2O_ERR_NULL = -1,        /* a required pointer is NULL */
   H2O_ERR_SHAPE = -2,       /* inconsistent or out-of-range sizes */
   H2O_ERR_ALIGN = -3,       /* a pointer is not 16-byte aligned */
-  H2O_ERR_UNSUPPORTED = -4, /* valid request this build does not handle (e.g. d) */
+  H2O_ERR_UNSUPPORTED = -4, /* valid request the library does not handle (e.g. d) */
   H2O_ERR_WORKSPACE = -5,   /* workspace NULL or smaller than h2o_workspace_size */
   H2O_ERR_ARG = -6,         /* bad scalar argument (window, budget, position) */
   H2O_ERR_CUDA = -7,        /* a CUDA runtime call failed; see h2o_last_cuda_error */

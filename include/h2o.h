@@ -310,12 +310,14 @@ H2O_API int h2o_kv_restore(const h2o_dims_t* dims, const int32_t* index,
  *   h2o_sdpa_chunk_q8, h2o_sdpa_cache_q8
  *                      h2o_sdpa_chunk / h2o_sdpa_cache with the cache read
  *                      through the 8-bit buffers (the chunk's own k_new /
- *                      v_new stay bf16 in h2o_sdpa_chunk_q8).  The workspace
- *                      (h2o_q8_workspace_size bytes, 16-byte aligned) holds
- *                      the K and V rows read back to bf16 (2 B d per slot
- *                      each; 8 MiB each for B = 1, Hkv = 8, M = 4096, d = 128,
- *                      which stays in L2) ahead of the attention's own
- *                      workspace.  Errors as h2o_sdpa_chunk / h2o_sdpa_cache.
+ *                      v_new stay bf16 in h2o_sdpa_chunk_q8).  S = 1 (the
+ *                      decode kernels) reads the codes directly.  Otherwise
+ *                      the workspace (h2o_q8_workspace_size bytes, 16-byte
+ *                      aligned) holds the K and V rows read back to bf16
+ *                      (2 B d per slot each; 8 MiB each for B = 1, Hkv = 8,
+ *                      M = 4096, d = 128, which stays in L2) ahead of the
+ *                      attention's own workspace.  Errors as h2o_sdpa_chunk /
+ *                      h2o_sdpa_cache.
  */
 H2O_API int h2o_kv_quantize(int64_t n_rows, int32_t d, const h2o_bf16* x, int8_t* codes,
                    float* scales, void* stream);

@@ -265,3 +265,41 @@ def test_q8_argument_checks(lib):
     assert ca(_dims(M=0), [p] * 8, w=None, wb=0) == SHAPE
     assert ca(d, [p] * 8, w=None) == WORKSPACE
     assert ca(d, [p] * 4 + [None] + [p] * 3) == NULL         # v_scales
+
+
+def test_q8_binding_marshals_to_the_host_checks(lib):
+    """The Python q8 wrappers reject wrong tensors themselves and hand the rest
+    to the C checks in the declared order (no GPU: a valid call ends at the
+    device lookup)."""
+    import types
+
+    import torch
+    bf16, i8, f32 = torch.bfloat16, torch.int8, torch.float32
+    st = types.SimpleNamespace(cuda_stream=0)            # the legacy default stream
+    with pytest.raises(ValueError):
+        b.h2o_kv_quantize(torch.zeros((4, 64), dtype=f32), stream=st)
+    with pytest.raises(b.H2OError) as e:
+        b.h2o_kv_quantize(torch.zeros((4, 96), dtype=bf16), stream=st)
+    assert e.value.status == UNSUP                       # d reached the C side as d
+    with pytest.raises(b.H2OError) as e:
+        b.h2o_kv_dequantize(torch.zeros((4, 64), dtype=i8), torch.zeros(4, dtype=f32), stream=st)
+    assert e.value.status == -10                         # no device: past every argument check
+    B, Hq, Hkv, d, S, M = 1, 4, 2, 64, 8, 32
+    codes = torch.zeros((B, Hkv, M, d), dtype=i8)
+    scales = torch.zeros((B, Hkv, M), dtype=f32)
+    scores = torch.zeros((B, Hkv, M), dtype=f32)
+    pos = torch.zeros((B, Hkv, M), dtype=torch.int32)
+    kn = torch.zeros((B, Hkv, S, d), dtype=bf16)
+    with pytest.raises(ValueError):                      # scales given as codes
+        b.h2o_evict_insert_q8(scores, pos, kn, kn, codes, codes, codes, scales, 100, 8, stream=st)
+    with pytest.raises(b.H2OError) as e:                 # budget != M, checked in C
+        b.h2o_evict_insert_q8(scores, pos, kn, kn, codes, scales, codes, scales, 100, 8,
+                              budget=M - 1, stream=st)
+    assert e.value.status == ARG
+    q = torch.zeros((B, Hq, S, d), dtype=bf16)
+    with pytest.raises(ValueError):                      # v_scales of the wrong shape
+        b.h2o_sdpa_chunk_q8(q, codes, scales, codes, scales[:, :, :-1], kn, kn, pos, 100, stream=st)
+    with pytest.raises(b.H2OError) as e:
+        b.h2o_sdpa_cache_q8(q, codes, scales, codes, scales, pos, -1,
+                            workspace=torch.zeros(1 << 20, dtype=torch.uint8), stream=st)
+    assert e.value.status == ARG                         # pos0 < 0

@@ -5,12 +5,11 @@ import numpy as np
 import pytest
 import torch
 
-from oracle import sdpa_chunk as ref_sdpa
 from paper_2608_19920_gb300 import build, h2o_device_errors, h2o_sdpa_chunk
 from paper_2608_19920_gb300._binding import h2o_selftest_bounded_wait
 from paper_2608_19920_gb300 import workloads as wl
 
-from test_gpu_parity import bf, check_sdpa
+from test_gpu_parity import bf, check_sdpa, oracle_sdpa
 
 pytestmark = pytest.mark.gpu
 
@@ -34,5 +33,6 @@ def test_bounded_wait_runs_out_and_is_reported():
                               pos0)
     torch.cuda.synchronize()
     assert h2o_device_errors() == 0
-    ref_out, ref_inc, _ = ref_sdpa(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"], pos0)
-    check_sdpa(out, inc, ref_out, ref_inc)
+    ref_out, ref_inc, w = oracle_sdpa(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"],
+                                      pos0)
+    check_sdpa(out, inc, ref_out, ref_inc, w)

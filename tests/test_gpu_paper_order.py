@@ -14,7 +14,7 @@ from paper_2608_19920_gb300 import (H2OLayer, build, h2o_device_errors, h2o_evic
 from paper_2608_19920_gb300 import workloads as wl
 from paper_2608_19920_gb300.runner import chunk_bounds
 
-from test_gpu_parity import bf, check_out, check_sdpa, f32
+from test_gpu_parity import bf, check_out, check_sdpa, f32, with_abs_values
 
 pytestmark = pytest.mark.gpu
 
@@ -94,8 +94,9 @@ def test_sdpa_cache_matches_oracle(dev, case):
                               torch.from_numpy(ins["slot_pos"]).to(dev), pos0)
     torch.cuda.synchronize()
     assert h2o_device_errors() == 0
-    ref_out, ref_inc, _ = ref_sdpa_cache(q, ins["k_cache"], ins["v_cache"], ins["slot_pos"], pos0)
-    check_sdpa(out, inc, ref_out, ref_inc)
+    ref_out, ref_inc, w = with_abs_values(ref_sdpa_cache, (q, ins["k_cache"], ins["v_cache"],
+                                                           ins["slot_pos"], pos0), (2,))
+    check_sdpa(out, inc, ref_out, ref_inc, w)
     np.testing.assert_allclose(inc.sum(-1).cpu().numpy(), S, rtol=1e-4)
 
 
@@ -122,8 +123,9 @@ def _paper_step_teacher_forced(layer, q, kn, vn, p, W, policy="h2o"):
     np.testing.assert_array_equal(ev.cpu().numpy(), ins["evict_idx"])
     np.testing.assert_array_equal(layer.slot_pos.cpu().numpy(), ins["slot_pos"])
     np.testing.assert_array_equal(f32(layer.k_cache), ins["k_cache"])
-    ref_out, ref_inc, _ = ref_sdpa_cache(qn, ins["k_cache"], ins["v_cache"], ins["slot_pos"], p)
-    check_sdpa(out, inc, ref_out, ref_inc)
+    ref_out, ref_inc, w = with_abs_values(ref_sdpa_cache, (qn, ins["k_cache"], ins["v_cache"],
+                                                           ins["slot_pos"], p), (2,))
+    check_sdpa(out, inc, ref_out, ref_inc, w)
     ref_scores = ref_scores_add(ins["scores"], inc.cpu().numpy(), "fp32")
     np.testing.assert_array_equal(layer.scores.cpu().numpy().view(np.uint32),
                                   ref_scores.view(np.uint32))
@@ -156,10 +158,10 @@ def test_full_size_paper_order_sampled(dev, name, check):
         if n == 0:
             out, inc, _ = layer.step(gq, gk, gv, p)
             rows = np.unique(np.concatenate([np.arange(4), np.linspace(0, e - 1, 12).astype(int)]))
-            ref_out, _, _ = ref_sdpa_cache(q[:1, :w.q_g], k[:1, :1], v[:1, :1],
-                                           np.arange(e, dtype=np.int32)[None, None], 0,
-                                           rows=rows)
-            check_out(f32(out[:1, :w.q_g])[:, :, rows], ref_out)
+            ref_out, _, wr = with_abs_values(
+                ref_sdpa_cache, (q[:1, :w.q_g], k[:1, :1], v[:1, :1],
+                                 np.arange(e, dtype=np.int32)[None, None], 0), (2,), rows=rows)
+            check_out(f32(out[:1, :w.q_g])[:, :, rows], ref_out, wr)
             np.testing.assert_allclose(inc.sum(-1).cpu().numpy(), e, rtol=1e-4)
         elif n in check:
             _paper_step_teacher_forced(layer, gq, gk, gv, p, w.W)

@@ -14,7 +14,7 @@ from paper_2608_19920_gb300 import (build, h2o_device_errors, h2o_evict_insert_q
 from paper_2608_19920_gb300._binding import H2O_DEVERR_CANDIDATES
 from paper_2608_19920_gb300 import workloads as wl
 
-from test_gpu_parity import bf, check_sdpa
+from test_gpu_parity import bf, check_sdpa, with_abs_values
 
 pytestmark = pytest.mark.gpu
 
@@ -175,14 +175,17 @@ def test_q8_sdpa_matches_oracle(dev, case):
         g = _gpu_q8(ins["k_codes"], ins["k_scales"], ins["v_codes"], ins["v_scales"], dev)
         sp = ins["slot_pos"]
         out, inc = h2o_sdpa_cache_q8(bf(q, dev), *g, torch.from_numpy(sp).to(dev), pos0)
-        ref_out, ref_inc, _ = oracle.sdpa_cache_q8(q, ins["k_codes"], ins["k_scales"],
-                                                   ins["v_codes"], ins["v_scales"], sp, pos0)
+        ref_out, ref_inc, w = with_abs_values(
+            oracle.sdpa_cache_q8, (q, ins["k_codes"], ins["k_scales"], ins["v_codes"],
+                                   ins["v_scales"], sp, pos0), (3,))
     else:
         sp = st["slot_pos"]
         out, inc = h2o_sdpa_chunk_q8(bf(q, dev), *g, bf(kn, dev), bf(vn, dev),
                                      torch.from_numpy(sp).to(dev), pos0)
-        ref_out, ref_inc, _ = oracle.sdpa_chunk_q8(q, kc, ks, vc, vs, kn, vn, sp, pos0)
+        # |codes| give |bf16(c s)| (the rounding is symmetric, scales >= 0)
+        ref_out, ref_inc, w = with_abs_values(oracle.sdpa_chunk_q8,
+                                              (q, kc, ks, vc, vs, kn, vn, sp, pos0), (3, 6))
     torch.cuda.synchronize()
     assert h2o_device_errors() == 0
-    check_sdpa(out, inc, ref_out, ref_inc)
+    check_sdpa(out, inc, ref_out, ref_inc, w)
     np.testing.assert_allclose(inc.sum(-1).cpu().numpy(), S, rtol=1e-4)

@@ -87,7 +87,7 @@ def peaks():
 
 # ---------------------------------------------------------------- clocks --
 class ClockSampler:
-    """nvidia-smi clocks / throttle reasons, sampled every 20 ms; only samples
+    """nvidia-smi clocks / throttle reasons, sampled every 10 ms; only samples
     whose timestamps fall inside [mark_start, mark_end] are summarised."""
     FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -104,7 +104,7 @@ class ClockSampler:
             self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "20"],
+                 "--format=csv,noheader,nounits", "-lms", "10"],
                 stdout=self.file, stderr=subprocess.DEVNULL)
             # sampling must be running before the timed region starts
             deadline = time.time() + 5.0
@@ -382,7 +382,7 @@ def run_ours(args, w):
         raise SystemExit("device-side error during the timed region")
 
     # ---- dominant kernel: the chunk SDPA alone, timed on the same stream
-    kern = time_sdpa_kernel(w, layer, inputs, plan, stream, reps=max(3, args.steps))
+    kern = time_sdpa_kernel(w, layer, inputs, plan, stream, reps=args.roofline_reps)
 
     value = tokens_per_step * world / (step_ms / 1e3)
     in_bytes = sum(x.numel() * x.element_size() for c in inputs for x in c)
@@ -430,7 +430,9 @@ def run_ours(args, w):
             "achieved": kern["gbs"], "peak": pk["hbm"], "unit": "GB/s",
             "frac": kern["gbs"] / pk["hbm"], "traffic": traffic,
             "peak_source": f"{pk['source']} HBM copy bandwidth",
-            "avg_launch_us": kern["avg_us"], "bytes_per_launch": kern["bytes"],
+            "avg_launch_us": kern["avg_us"], "median_launch_us": kern["median_us"],
+            "launches_timed": kern["launches"], "bytes_per_launch": kern["bytes"],
+            "clocks": kern["clocks"],
         }
     else:
         line["roofline"] = {
@@ -442,8 +444,10 @@ def run_ours(args, w):
             "frac": kern["alg_tflops"] / pk["bf16"], "traffic": traffic,
             "peak_source": f"{pk['source']} bf16 dense, burst",
             "frac_of_sustained": kern["alg_tflops"] / pk["bf16_sus"],
-            "avg_launch_us": kern["avg_us"], "flops_per_launch": kern["flops"],
+            "avg_launch_us": kern["avg_us"], "median_launch_us": kern["median_us"],
+            "launches_timed": kern["launches"], "flops_per_launch": kern["flops"],
             "executed_tflops": kern["alg_tflops"] * kern["exec_ratio"],
+            "clocks": kern["clocks"],
         }
     if args.e2e:
         line["e2e"] = run_e2e(w, layer, plan, outs, dev, args, world)
@@ -501,27 +505,32 @@ def time_sdpa_kernel(w, layer, inputs, plan, stream, reps, idx=None, prepare=Tru
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph):
         call()
-    times = []
-    for _ in range(reps + 2):
-        # Evict the previous launch's data from L2 by writing a buffer twice
-        # its size, then read another one so that the write-back of those
-        # dirty lines happens here, not inside the timed launch.
-        flush.zero_()
-        clean.sum()
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        graph.replay()
-        b.record(stream)
+    evs = []
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        clk.mark_start()
+        for _ in range(reps + 2):
+            # Evict the previous launch's data from L2 by writing a buffer
+            # twice its size, then read another one so that the write-back of
+            # those dirty lines happens here, not inside the timed launch.
+            flush.zero_()
+            clean.sum()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            graph.replay()
+            b.record(stream)
+            evs.append((a, b))
         torch.cuda.synchronize()
-        times.append(a.elapsed_time(b))
-    times = times[2:]
+        clk.mark_end()
+    times = [a.elapsed_time(b) for a, b in evs][2:]
     avg_ms = sum(times) / len(times)
     flops = chunk_flops(w.B, w.Hq, w.d, e - p, visible_old(w, e - p, layer.order))
     exec_flops = executed_mma_flops(w, e - p)
     kv_bytes = decode_kv_bytes(w, layer.kv_bits)
-    return dict(avg_us=avg_ms * 1e3, flops=flops, alg_tflops=flops / (avg_ms / 1e3) / 1e12,
-                exec_ratio=exec_flops / flops, bytes=kv_bytes, gbs=kv_bytes / (avg_ms / 1e3) / 1e9)
+    return dict(avg_us=avg_ms * 1e3, median_us=statistics.median(times) * 1e3, launches=len(times),
+                flops=flops, alg_tflops=flops / (avg_ms / 1e3) / 1e12,
+                exec_ratio=exec_flops / flops, bytes=kv_bytes, gbs=kv_bytes / (avg_ms / 1e3) / 1e9,
+                clocks=clk.summary())
 
 
 def decode_kv_bytes(w, kv_bits: int = 16):
@@ -646,6 +655,9 @@ def main():
                     help="kernel: only repeat the steady-state chunk SDPA launch (for profiling); "
                          "backward: time the gradient of that chunk (h2o_sdpa_chunk_backward)")
     ap.add_argument("--reps", type=int, default=5)
+    ap.add_argument("--roofline-reps", type=int, default=500,
+                    help="launches of the dominant kernel timed for the roofline (after 2 "
+                         "untimed ones), independent of --steps")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

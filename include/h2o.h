@@ -32,12 +32,21 @@
  *
  * Conventions for every call:
  *  - All array arguments are DEVICE pointers, allocated and owned by the
- *    caller; the library allocates no device memory of its own (the scratch
- *    of h2o_sdpa_decode_static and the error word are static device arrays;
- *    h2o_sdpa_chunk_backward uses cuBLASLt in the caller's workspace) and
- *    keeps no per-call state.
+ *    caller.  The forward, update, replay and 8-bit calls allocate no device
+ *    memory (the scratch of h2o_sdpa_decode_static and the error word are
+ *    static device arrays) and keep no per-call state.  The exception is
+ *    h2o_sdpa_chunk_backward: its GEMMs run on cuBLASLt, and its first call
+ *    on a device creates one cuBLASLt handle there that lives until exit; the
+ *    handle's own allocations belong to the library (the matrices themselves
+ *    go to the caller's workspace).
  *    Every array is dense, row-major (C order) with the shape given, and must
  *    be 16-byte aligned.
+ *  - The library resolves some per-device state on its first call on a
+ *    device (the error word's and the static scratch's addresses, kernel
+ *    shared-memory limits, resident CTA counts) and keeps it until exit.
+ *    A cudaDeviceReset() destroys the context that state belongs to: after
+ *    one, no call of this library may be made on that device in the same
+ *    process.
  *  - bf16 arrays hold IEEE bfloat16 bit patterns (h2o_bf16 = uint16_t).
  *  - Calls only enqueue work on `stream` (a cudaStream_t; NULL = legacy
  *    default stream) and return without synchronising.  Arguments are

@@ -20,7 +20,6 @@ __device__ int g_device_errors;
 
 namespace {
 
-constexpr int kMaxDevices = 64;
 thread_local int t_last_cuda_error = 0;
 
 struct DeviceInfo {

@@ -622,25 +622,28 @@ template <int D, int QG, bool Q8>
 cudaError_t launch_split(const DecodeArgs& a, cudaStream_t stream) {
   // Persistent grid: as many CTAs as fit on the GPU at once (sized once per
   // device for the largest split), each taking every gridDim-th work item.
-  static int resident[64] = {};  // one table per instantiation
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  int n_res = dev < 64 ? resident[dev] : 0;
-  if (n_res == 0) {
+  // One table per instantiation.
+  static OncePerDevice once;
+  static int resident[kMaxDevices];
+  cudaError_t e = once.run([](int d) {
     const int smem_max = static_cast<int>(split_smem<D, QG, Q8>(kDecodeMaxSplitLen));
-    e = cudaFuncSetAttribute(decode_split_kernel<D, QG, Q8>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
-    if (e != cudaSuccess) return e;
+    cudaError_t r = cudaFuncSetAttribute(decode_split_kernel<D, QG, Q8>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
+    if (r != cudaSuccess) return r;
     int per_sm = 0, sms = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_split_kernel<D, QG, Q8>,
+    r = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_split_kernel<D, QG, Q8>,
                                                       kDecThreads, smem_max);
-    if (e != cudaSuccess) return e;
-    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-    n_res = std::max(1, per_sm) * sms;
-    if (dev < 64) resident[dev] = n_res;
-  }
+    if (r != cudaSuccess) return r;
+    r = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, d);
+    if (r != cudaSuccess) return r;
+    resident[d] = std::max(1, per_sm) * sms;
+    return cudaSuccess;
+  });
+  if (e != cudaSuccess) return e;
+  int dev = 0;
+  e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const int n_res = resident[dev];
   const int n_items = a.n_split * a.B * a.Hkv;
   const size_t smem = split_smem<D, QG, Q8>(a.split_len);
   decode_split_kernel<D, QG, Q8><<<std::min(n_items, n_res), kDecThreads, smem, stream>>>(a);

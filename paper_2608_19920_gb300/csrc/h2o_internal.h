@@ -5,10 +5,30 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <mutex>
 
 #include "../../include/h2o.h"
 
 namespace h2o {
+
+constexpr int kMaxDevices = 64;
+
+// Runs a set-up step (a kernel attribute, an occupancy query) once per device,
+// the first time any host thread needs it there, and remembers its status.
+// The function receives the device ordinal and returns a cudaError_t.
+struct OncePerDevice {
+  std::once_flag once[kMaxDevices];
+  cudaError_t status[kMaxDevices] = {};
+  template <typename F>
+  cudaError_t run(F&& f) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::call_once(once[dev], [&] { status[dev] = f(dev); });
+    return status[dev];
+  }
+};
 
 constexpr int kTileM = 128;        // query rows per CTA (tcgen05 M)
 constexpr int kTileN = 128;        // keys per tile (tcgen05 N of Q K^T, K of P V)

@@ -716,16 +716,12 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
     const size_t per = (static_cast<size_t>(a.M) + C - 1) / C;
     const size_t stash = per * (a.policy == H2O_POLICY_ORIG ? a.B : 1) * sizeof(float);
     const int stash_ok = stash <= kDStashBytes ? 1 : 0;
-    static bool dconf[64] = {};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    static OncePerDevice dconf;
+    cudaError_t e = dconf.run([](int) {
+      return cudaFuncSetAttribute(update_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(kDStashBytes));
+    });
     if (e != cudaSuccess) return e;
-    if (dev >= 64 || !dconf[dev]) {
-      e = cudaFuncSetAttribute(update_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               static_cast<int>(kDStashBytes));
-      if (e != cudaSuccess) return e;
-      if (dev < 64) dconf[dev] = true;
-    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(groups * C));
     cfg.blockDim = dim3(kDThreads);
@@ -745,16 +741,12 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
     update_kernel<<<groups, kUpdThreads, 0, stream>>>(a);
     return cudaGetLastError();
   }
-  static bool configured[64] = {};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  static OncePerDevice configured;
+  cudaError_t e = configured.run([](int) {
+    return cudaFuncSetAttribute(update_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(kMaxClusterSmem));
+  });
   if (e != cudaSuccess) return e;
-  if (dev < 64 && !configured[dev]) {
-    e = cudaFuncSetAttribute(update_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kMaxClusterSmem));
-    if (e != cudaSuccess) return e;
-    configured[dev] = true;
-  }
   int C = (a.S + 63) / 64;
   C = C < 1 ? 1 : (C > 8 ? 8 : C);
   cudaLaunchConfig_t cfg = {};

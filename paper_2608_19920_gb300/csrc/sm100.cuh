@@ -68,6 +68,12 @@ __device__ __forceinline__ bool bar_try_wait(uint64_t* bar, uint32_t parity,
   return done != 0;
 }
 
+// Longest time one try_wait may keep a thread suspended.  The thread wakes as
+// soon as the phase completes, so this only bounds how late the abort flag and
+// the time limit below are looked at; in between, a waiting warp issues
+// nothing and leaves its scheduler's issue slots to the warps doing work.
+constexpr uint32_t kSuspendHintNs = 200000;
+
 // Waits for the phase with the given parity to complete.  Gives up after
 // `limit_ns` or as soon as *abort becomes non-zero; returns false then.
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort,
@@ -75,7 +81,7 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatil
   if (bar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   while (true) {
-    if (bar_try_wait(bar, parity)) return true;
+    if (bar_try_wait(bar, parity, kSuspendHintNs)) return true;
     if (*abort) return false;
     if (global_timer_ns() - t0 > limit_ns) {
       *abort = 1;
@@ -555,6 +561,18 @@ __device__ __forceinline__ float fast_exp2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+
+// Three-input maximum (one instruction on the sm_100 family).
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Packed pairs of fp32 operations (one instruction for two lanes of data on
+// the sm_100 family), round to nearest even like their scalar forms.
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) { return __fadd2_rn(a, b); }
 
 __device__ __forceinline__ void red_add_f32(float* addr, float v) {
   asm volatile("red.global.add.f32 [%0], %1;" ::"l"(addr), "f"(v) : "memory");

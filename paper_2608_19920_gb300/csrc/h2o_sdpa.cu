@@ -570,6 +570,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     }
     float m_run = -INFINITY, l_run = 0.f;
     float lam4[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+    float2 nl4[4];  // (-lam, -lam) of the four rows, for the packed FMAs
+#pragma unroll
+    for (int x = 0; x < 4; ++x) nl4[x] = make_float2(-INFINITY, -INFINITY);
     bool ok = true;
     bool have_lambda = false;
     int k2 = 0;  // pass-2 tiles this warp has processed (column-sum buffer phase)
@@ -600,6 +603,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           for (int w = 0; w < kNumWG; ++w)
             l += sm.rowstat[w][r][1] * fast_exp2(sm.rowstat[w][r][0] - mm);
           lam4[x] = (v4[x] && mm > -INFINITY) ? mm + fast_log2(l) : INFINITY;
+          nl4[x] = make_float2(-lam4[x], -lam4[x]);
         }
         have_lambda = true;
       }
@@ -633,24 +637,31 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
             if (lane == 0) arrive_issuer<kPair>(&sm.bar_sread[buf]);  // S buffer may be overwritten
           }
           if (!partial) {
-            float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
+            // maximum: four chains of three-input max (16 instructions for 32
+            // values); then exp2(s c - m) and the sum with packed fp32 pairs
+            float c0 = max3f(v[0], v[1], v[2]), c1 = max3f(v[3], v[4], v[5]);
+            float c2 = max3f(v[6], v[7], v[8]), c3 = max3f(v[9], v[10], v[11]);
 #pragma unroll
-            for (int k = 4; k < 32; k += 4) {
-              mx0 = fmaxf(mx0, v[k]);
-              mx1 = fmaxf(mx1, v[k + 1]);
-              mx2 = fmaxf(mx2, v[k + 2]);
-              mx3 = fmaxf(mx3, v[k + 3]);
+            for (int k = 12; k < 28; k += 8) {
+              c0 = max3f(c0, v[k], v[k + 1]);
+              c1 = max3f(c1, v[k + 2], v[k + 3]);
+              c2 = max3f(c2, v[k + 4], v[k + 5]);
+              c3 = max3f(c3, v[k + 6], v[k + 7]);
             }
-            const float m_new = fmaxf(m_run, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2);
-            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+            c0 = max3f(c0, v[28], v[29]);
+            c1 = max3f(c1, v[30], v[31]);
+            const float m_new = fmaxf(m_run, max3f(c0, c1, fmaxf(c2, c3)) * sl2);
+            const float2 sc = make_float2(sl2, sl2), nm = make_float2(-m_new, -m_new);
+            float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
 #pragma unroll
             for (int k = 0; k < 32; k += 4) {
-              s0 += fast_exp2(fmaf(v[k], sl2, -m_new));
-              s1 += fast_exp2(fmaf(v[k + 1], sl2, -m_new));
-              s2 += fast_exp2(fmaf(v[k + 2], sl2, -m_new));
-              s3 += fast_exp2(fmaf(v[k + 3], sl2, -m_new));
+              const float2 x = ffma2(make_float2(v[k], v[k + 1]), sc, nm);
+              const float2 y = ffma2(make_float2(v[k + 2], v[k + 3]), sc, nm);
+              a0 = fadd2(a0, make_float2(fast_exp2(x.x), fast_exp2(x.y)));
+              a1 = fadd2(a1, make_float2(fast_exp2(y.x), fast_exp2(y.y)));
             }
-            l_run = l_run * fast_exp2(m_run - m_new) + ((s0 + s1) + (s2 + s3));
+            const float2 s = fadd2(a0, a1);
+            l_run = l_run * fast_exp2(m_run - m_new) + (s.x + s.y);
             m_run = m_new;
           } else {
             uint32_t vis = 0u;  // bit k: column col0 + k visible to this row
@@ -708,10 +719,23 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
             }
           }
           if (!partial) {
+            // registers 4k, 4k+1 hold row A (pa) / C (pb), 4k+2, 4k+3 row B / D,
+            // each a pair of adjacent columns: one packed FMA per pair
+            const float2 sc = make_float2(sl2, sl2);
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-              pa[k] = fast_exp2(fmaf(pa[k], sl2, -lam4[(k >> 1) & 1]));
-              pb[k] = fast_exp2(fmaf(pb[k], sl2, -lam4[2 + ((k >> 1) & 1)]));
+            for (int k = 0; k < 4; ++k) {
+              const float2 xa = ffma2(make_float2(pa[4 * k], pa[4 * k + 1]), sc, nl4[0]);
+              const float2 xb = ffma2(make_float2(pa[4 * k + 2], pa[4 * k + 3]), sc, nl4[1]);
+              const float2 xc = ffma2(make_float2(pb[4 * k], pb[4 * k + 1]), sc, nl4[2]);
+              const float2 xd = ffma2(make_float2(pb[4 * k + 2], pb[4 * k + 3]), sc, nl4[3]);
+              pa[4 * k] = fast_exp2(xa.x);
+              pa[4 * k + 1] = fast_exp2(xa.y);
+              pa[4 * k + 2] = fast_exp2(xb.x);
+              pa[4 * k + 3] = fast_exp2(xb.y);
+              pb[4 * k] = fast_exp2(xc.x);
+              pb[4 * k + 1] = fast_exp2(xc.y);
+              pb[4 * k + 2] = fast_exp2(xd.x);
+              pb[4 * k + 3] = fast_exp2(xd.y);
             }
           } else {
 #pragma unroll
@@ -756,8 +780,11 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           float v[8];
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            v[2 * k] = (pa[4 * k] + pa[4 * k + 2]) + (pb[4 * k] + pb[4 * k + 2]);
-            v[2 * k + 1] = (pa[4 * k + 1] + pa[4 * k + 3]) + (pb[4 * k + 1] + pb[4 * k + 3]);
+            const float2 cs =
+                fadd2(fadd2(make_float2(pa[4 * k], pa[4 * k + 1]), make_float2(pa[4 * k + 2], pa[4 * k + 3])),
+                      fadd2(make_float2(pb[4 * k], pb[4 * k + 1]), make_float2(pb[4 * k + 2], pb[4 * k + 3])));
+            v[2 * k] = cs.x;
+            v[2 * k + 1] = cs.y;
           }
           rs_step<8, 16>(v, lane);
           rs_step<4, 8>(v, lane);
@@ -855,16 +882,12 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
 template <int D, bool kPair>
 cudaError_t launch_d(const SdpaArgs& a, cudaStream_t stream) {
   const size_t smem = sizeof(SdpaSmem<D, kPair>) + 1024;
-  static bool configured[64] = {};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  static OncePerDevice configured;
+  cudaError_t e = configured.run([smem](int) {
+    return cudaFuncSetAttribute(sdpa_chunk_kernel<D, kPair>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  });
   if (e != cudaSuccess) return e;
-  if (dev < 64 && !configured[dev]) {
-    e = cudaFuncSetAttribute(sdpa_chunk_kernel<D, kPair>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    configured[dev] = true;
-  }
   const int ctas = kPair ? 2 * ((a.n_row_tiles + 1) / 2) : a.n_row_tiles;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(ctas), static_cast<unsigned>(a.B * a.Hkv));

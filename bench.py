@@ -545,9 +545,11 @@ def launches_per_chunk(S, M, order="chunk", kv_bits=16, qg=4):
     when S = 1 and a cache exists) and the update (the paper's order: the
     eviction-insert, the SDPA and the score addition); 8-bit buffers add the
     quantising scatter after the update and, where the chunk kernel runs, the
-    read-back before it (the decode kernels read the codes themselves)."""
+    read-back before it (the decode kernels read the codes themselves).  With
+    three or more 128-row tiles per query head (S > 256) the chunk kernel is
+    followed by the kernel that adds its per-tile column sums in order."""
     decode = S == 1 and M > 0 and qg <= 8
-    sdpa = 2 if decode else 1
+    sdpa = 2 if decode else (2 if (S + 127) // 128 >= 3 and S > 128 else 1)
     q8 = (1 + (0 if decode or M == 0 else 1)) if kv_bits == 8 else 0
     return sdpa + (2 if order == "paper" else 1) + q8
 

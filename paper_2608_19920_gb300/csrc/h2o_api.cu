@@ -144,8 +144,9 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   int split_len = 0, n_split = 0;
   size_t ws_need = 0;
   const bool decode = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
-  if (decode && (!workspace || workspace_bytes < ws_need)) return H2O_ERR_WORKSPACE;
-  if (decode && misaligned(workspace)) return H2O_ERR_ALIGN;
+  if (!decode) ws_need = sdpa_colpart_bytes(D.B, D.Hq, D.S, D.M);
+  if (ws_need > 0 && (!workspace || workspace_bytes < ws_need)) return H2O_ERR_WORKSPACE;
+  if (ws_need > 0 && misaligned(workspace)) return H2O_ERR_ALIGN;
   DeviceInfo* di = nullptr;
   if ((st = current_device(&di)) != H2O_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -203,6 +204,7 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   a.out = out;
   a.score_inc = score_inc;
   a.err = di->err_word;
+  a.colpart = ws_need > 0 ? static_cast<float*>(workspace) : nullptr;
 
   const uint64_t G = static_cast<uint64_t>(D.B) * D.Hkv;
   {
@@ -231,10 +233,16 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   const size_t inc_bytes = static_cast<size_t>(G) * qg * static_cast<size_t>(nk) * sizeof(float);
   cudaError_t e = read_back();
   if (e != cudaSuccess) return cuda_fail(e);
-  e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
-  if (e != cudaSuccess) return cuda_fail(e);
+  if (a.colpart == nullptr) {
+    e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
   e = launch_sdpa(a, s);
   if (e != cudaSuccess) return cuda_fail(e);
+  if (a.colpart != nullptr) {
+    e = launch_colsum_reduce(a.colpart, score_inc, D.B * D.Hq, a.tiles_per_head, nk, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
   return H2O_OK;
 }
 
@@ -408,7 +416,9 @@ int h2o_workspace_size(const h2o_dims_t* dims, size_t* bytes) {
   int split_len = 0, n_split = 0;
   size_t ws = 0;
   const h2o_dims_t& D = *dims;
-  *bytes = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws) ? ws : 0;
+  *bytes = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws)
+               ? ws
+               : sdpa_colpart_bytes(D.B, D.Hq, D.S, D.M);
   return H2O_OK;
 }
 

@@ -55,7 +55,27 @@ struct SdpaArgs {
   int n_cache_tiles;       // ceil(M / 128)
   int n_chunk_tiles;       // ceil(S / 128); 0 for h2o_sdpa_cache (keys in the cache only)
   int nk;                  // key columns of a score_inc row: M + S, or M for h2o_sdpa_cache
+  // Column-sum partials, one row per (b, query head, row tile of that head):
+  // (B * Hq, tiles_per_head, nk) fp32 in the caller's workspace, or null.
+  // With three or more row tiles per head the kernel stores each tile's
+  // column sums here (zeros for tiles it skips) and colsum_reduce adds them
+  // in row-tile order, so score_inc does not depend on the order the CTAs
+  // finish in; otherwise it adds into the zeroed score_inc directly (at most
+  // two addends per element onto an exact zero, which commute).
+  float* colpart;
 };
+
+// Row tiles per query head above which the column sums go through colpart.
+constexpr int kColpartMinTiles = 3;
+
+// Bytes of colpart for a chunk of S queries against M slots (0 when the
+// column sums are added into score_inc directly).
+size_t sdpa_colpart_bytes(int B, int Hq, int S, int M);
+
+// score_inc[row, j] = sum over r = 0 .. tph-1 (in that order) of
+// colpart[row, r, j], for rows = B * Hq and j < nk.
+cudaError_t launch_colsum_reduce(const float* colpart, float* score_inc, int rows, int tph, int nk,
+                                 cudaStream_t stream);
 
 struct UpdateArgs {
   float* scores;

@@ -568,6 +568,23 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       }
       warp_head[w] = (gw >= 0 && gw < a.qg) ? gw : -1;
     }
+    // this CTA's row of column-sum partials (three or more row tiles per
+    // head: all 128 rows belong to query head g_first, row tile rt % tph);
+    // the columns of tiles neither CTA of the pair visits are zeroed here,
+    // the others are stored by the combine after each pass-2 tile
+    float* prow = nullptr;
+    if (a.colpart != nullptr && has_rows) {
+      prow = a.colpart + (static_cast<size_t>(b * a.Hq + hkv * a.qg + g_first) * a.tiles_per_head +
+                          rt % a.tiles_per_head) * NK;
+      const int total = a.n_cache_tiles + a.n_chunk_tiles;
+      for (int tt = sw; tt < total; tt += kSoftmaxWarps) {
+        if (sm.cls[tt] != 0) continue;
+        const bool ch = tt >= a.n_cache_tiles;
+        const int c0 = (ch ? tt - a.n_cache_tiles : tt) * kTileN;
+        const int c1 = min(c0 + kTileN, ch ? a.S : a.M);
+        for (int c = c0 + static_cast<int>(lane); c < c1; c += 32) prow[(ch ? a.M : 0) + c] = 0.f;
+      }
+    }
     float m_run = -INFINITY, l_run = 0.f;
     float lam4[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
     float2 nl4[4];  // (-lam, -lam) of the four rows, for the packed FMAs
@@ -813,7 +830,14 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           for (int hh = 0; hh < 2; ++hh) {
             const int c = 32 * hh + static_cast<int>(lane);
             const int col = colb + c;
-            if (chunk ? col < a.S : col < a.M) {
+            if (prow != nullptr && (chunk ? col < a.S : col < a.M)) {
+              // one head: the four quarters in order, stored (rows past S
+              // have p = 0)
+              float acc = 0.f;
+#pragma unroll
+              for (int w = 0; w < 4; ++w) acc += sm.colsum[cb][wg][w][c];
+              prow[(chunk ? a.M : 0) + col] = acc;
+            } else if (chunk ? col < a.S : col < a.M) {
               float* dst = inc_base + (chunk ? a.M + col : col);
               float acc = 0.f;
 #pragma unroll
@@ -908,6 +932,48 @@ cudaError_t launch_d(const SdpaArgs& a, cudaStream_t stream) {
 
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream) {
   return a.d == 64 ? launch_d<64, false>(a, stream) : launch_d<128, true>(a, stream);
+}
+
+namespace {
+
+constexpr int kReduceThreads = 256;
+
+// One thread per score_inc element: the row tiles' partials in row-tile order
+// (all loads issued before the adds).
+__global__ void __launch_bounds__(kReduceThreads) colsum_reduce_kernel(
+    const float* __restrict__ part, float* __restrict__ score_inc, int rows, int tph, int nk) {
+  const int col = blockIdx.x * kReduceThreads + static_cast<int>(threadIdx.x);
+  if (col >= nk) return;
+  for (int row = blockIdx.y; row < rows; row += gridDim.y) {
+  const float* p = part + static_cast<size_t>(row) * tph * nk + col;
+  float acc = __ldg(p);
+  int r = 1;
+  for (; r + 4 <= tph; r += 4) {
+    const float x0 = __ldg(p + static_cast<size_t>(r) * nk);
+    const float x1 = __ldg(p + static_cast<size_t>(r + 1) * nk);
+    const float x2 = __ldg(p + static_cast<size_t>(r + 2) * nk);
+    const float x3 = __ldg(p + static_cast<size_t>(r + 3) * nk);
+    acc = (((acc + x0) + x1) + x2) + x3;
+  }
+  for (; r < tph; ++r) acc += __ldg(p + static_cast<size_t>(r) * nk);
+  score_inc[static_cast<size_t>(row) * nk + col] = acc;
+  }
+}
+
+}  // namespace
+
+size_t sdpa_colpart_bytes(int B, int Hq, int S, int M) {
+  const int tph = S > kTileM ? (S + kTileM - 1) / kTileM : 0;
+  if (tph < kColpartMinTiles) return 0;
+  return static_cast<size_t>(B) * Hq * tph * (static_cast<size_t>(M) + S) * sizeof(float);
+}
+
+cudaError_t launch_colsum_reduce(const float* colpart, float* score_inc, int rows, int tph, int nk,
+                                 cudaStream_t stream) {
+  const dim3 grid(static_cast<unsigned>((nk + kReduceThreads - 1) / kReduceThreads),
+                  static_cast<unsigned>(rows < 65535 ? rows : 65535));
+  colsum_reduce_kernel<<<grid, kReduceThreads, 0, stream>>>(colpart, score_inc, rows, tph, nk);
+  return cudaGetLastError();
 }
 
 }  // namespace h2o

@@ -91,6 +91,27 @@ def test_decode_workspace(lib):
                               None) == ALIGN
 
 
+def test_chunk_workspace(lib):
+    """With three or more 128-row tiles per query head (S > 256) the chunk
+    kernel stores per-row-tile column sums in the workspace, (B, Hq, tiles,
+    M + S) fp32, and a second kernel adds them in row-tile order; one or two
+    tiles per head add into score_inc directly and need no workspace."""
+    n = ctypes.c_size_t(0)
+    for S, tiles in ((32, 0), (128, 0), (256, 0), (257, 3), (512, 4), (4096, 32)):
+        dims = _dims(B=2, Hq=8, Hkv=2, d=128, S=S, M=4096)
+        assert lib.h2o_workspace_size(ctypes.byref(dims), ctypes.byref(n)) == OK
+        assert n.value == 2 * 8 * tiles * (4096 + S) * 4, (S, n.value)
+    vp = ctypes.c_void_p
+    ptrs = [vp(0x1000)] * 8
+    big = _dims(B=1, Hq=4, Hkv=2, d=128, S=512, M=1024)
+    need = 1 * 4 * 4 * (1024 + 512) * 4
+    assert lib.h2o_sdpa_chunk(ctypes.byref(big), 2048, 0.0, *ptrs, None, 0, None) == WORKSPACE
+    assert lib.h2o_sdpa_chunk(ctypes.byref(big), 2048, 0.0, *ptrs, vp(0x2000), need - 1,
+                              None) == WORKSPACE
+    assert lib.h2o_sdpa_chunk(ctypes.byref(big), 2048, 0.0, *ptrs, vp(0x2008), need,
+                              None) == ALIGN
+
+
 def _upd(lib, dims, budget=256, W=32, pos0=256, ptrs=None, evict=None):
     p = ptrs or [0x1000] * 7
     vp = ctypes.c_void_p

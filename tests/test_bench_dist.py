@@ -61,14 +61,15 @@ def test_launch_and_byte_accounting():
     the K and V rows read once (8-bit rows: d codes + a 4-byte scale)."""
     import bench
     lpc = bench.launches_per_chunk
-    assert lpc(512, 4096) == 2                      # SDPA + update
-    assert lpc(512, 4096, "paper") == 3             # evict-insert + SDPA + scores_add
+    assert lpc(512, 4096) == 3                      # SDPA + column-sum reduction + update
+    assert lpc(256, 2048) == 2                      # two row tiles per head: no reduction
+    assert lpc(512, 4096, "paper") == 4             # evict-insert + SDPA + reduction + scores_add
     assert lpc(1, 4096) == 3                        # split + combine + update
     assert lpc(1, 4096, "paper") == 4
     assert lpc(1, 4096, "chunk", 16, 16) == 2       # q_g > 8: the chunk kernel
-    assert lpc(512, 4096, "chunk", 8) == 4          # + read-back + quantising scatter
-    assert lpc(4096, 4096, "chunk", 8) == 4         # the prefill
-    assert lpc(512, 4096, "paper", 8) == 5
+    assert lpc(512, 4096, "chunk", 8) == 5          # + read-back + quantising scatter
+    assert lpc(4096, 4096, "chunk", 8) == 5         # the prefill
+    assert lpc(512, 4096, "paper", 8) == 6
     assert lpc(1, 4096, "chunk", 8) == 4            # the decode kernels read the codes
     assert lpc(1, 4096, "paper", 8) == 5
     assert lpc(1, 4096, "chunk", 8, 16) == 4        # q_g > 8: read-back + chunk kernel

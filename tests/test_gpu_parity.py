@@ -106,6 +106,9 @@ SDPA_CASES = [
     (1, 8, 8, 64, 64, 128, 128, 0, 0),        # empty cache (prefill against empty slots)
     (2, 16, 4, 128, 130, 1000, 40, 30, 2000), # mixed: empties, future slots, ragged tiles
     (1, 32, 8, 128, 512, 4096, 0, 0, 8192),   # the Llama-3-8B-shaped chunk
+    (2, 8, 2, 128, 300, 700, 11, 20, 3000),   # 3 row tiles per head (the last of 44 rows):
+                                              # column sums through the workspace
+    (1, 4, 1, 64, 520, 130, 0, 40, 600),      # d = 64, 5 row tiles per head, future slots
 ]
 
 

@@ -246,6 +246,9 @@ constexpr int kCWarps = kCThreads / 32;
 // which the packed 16-bit counts of phase 3 need)
 constexpr size_t kMaxClusterSmem = 200 * 1024;
 
+// Keys a thread keeps in registers during the selection (M <= 16 * 512).
+constexpr int kRegKeys = 16;
+
 // Exclusive prefix sum over the block of one value per thread.
 __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_tot,
                                                     uint32_t* total) {
@@ -274,14 +277,13 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_t
   return base + incl - v;
 }
 
-// Loads of up to kQgBatch query heads are in flight before their sums.
-constexpr int kQgBatch = 4;
-// Slots a thread handles per batch of loads in phase 1.
-constexpr int kBatch = 8;
 
-__global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const UpdateArgs a, int C) {
-  extern __shared__ uint32_t dyn[];
-  __shared__ uint32_t hist[256];
+__global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const UpdateArgs a, int C,
+                                                                      int prefetch) {
+  extern __shared__ __align__(16) uint32_t dyn[];
+  __shared__ __align__(16) uint32_t hist[3][256];
+  __shared__ uint64_t rows_bar;
+  __shared__ int abort_flag;
   __shared__ uint32_t warp_tot[kCWarps];
   __shared__ uint32_t bcast[4];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -297,6 +299,27 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   float* accs = reinterpret_cast<float*>(dyn + M);               // [M] scores of (b0, h)
   float* nscore = reinterpret_cast<float*>(dyn + 2 * M);         // [S] score of new token c
   int* elist = reinterpret_cast<int*>(dyn + 2 * M + S);          // [S] evicted slot of rank c
+  // prefetch: this CTA copies the ranks [c_lo, c_lo + n_rows); their K rows
+  // then V rows are bulk-loaded here at the start and stored in phase 5
+  const int c_per = (S + C - 1) / C;
+  const int c_lo = min(S, rank * c_per), n_rows = min(S, c_lo + c_per) - c_lo;
+  uint16_t* rowbuf = reinterpret_cast<uint16_t*>(
+      reinterpret_cast<uint8_t*>(dyn) + ((2 * static_cast<size_t>(M) + 2 * S) * 4 + 15) / 16 * 16);
+  if (tid == 0) {
+    abort_flag = 0;
+    if (prefetch && n_rows > 0) {
+      bar_init(&rows_bar, 1);
+      fence_bar_init();
+      const uint32_t bytes = static_cast<uint32_t>(n_rows) * a.d * 2u;
+      bar_expect_tx(&rows_bar, 2 * bytes);
+      const size_t src = ((static_cast<size_t>(b0) * a.Hkv + h) * S + c_lo) * a.d;
+      bulk_load_once(rowbuf, a.k_new + src, bytes, &rows_bar);
+      bulk_load_once(rowbuf + static_cast<size_t>(c_per) * a.d, a.v_new + src, bytes, &rows_bar);
+    }
+  }
+  // histograms of passes 0 and 1 (the cluster barrier below orders the clears
+  // before any count)
+  for (int x = tid; x < 2 * 256; x += kCThreads) hist[x >> 8][x & 255] = 0u;
   auto scores_of = [&](int b) { return a.scores + (static_cast<size_t>(b) * a.Hkv + h) * M; };
   auto pos_of = [&](int b) { return a.slot_pos + (static_cast<size_t>(b) * a.Hkv + h) * M; };
   auto inc_of = [&](int b) { return a.score_inc + static_cast<size_t>(b * a.Hq + h * qg) * NK; };
@@ -307,131 +330,159 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   // 16-byte loads need every row start (b, h rows of M and NK) and j0 aligned
   const bool vec = R % 4 == 0 && M % 4 == 0 && NK % 4 == 0;
 
-  // acc_j = scores_j + (inc_0j + inc_1j + ...) of batch entry b for the n
-  // slots from jb, fp32, heads in order (Eq. 3); tot_j := acc_j (first) or
-  // tot_j + acc_j.  Loads of up to four heads are in flight before their sums.
-  auto add_acc = [&](int b, int jb, int n, float (&tot)[kBatch], bool first) {
-    const float* sc = scores_of(b);
-    const float* inc = inc_of(b);
-    float sv[kBatch], tv[kBatch];
-    if (a.insert) {  // scores as they are
-      for (int k = 0; k < n; ++k) {
-        sv[k] = sc[jb + k];
-        tv[k] = 0.f;
-      }
-    } else if (vec && n == kBatch) {
-      float4 s4[2];
-#pragma unroll
-      for (int q = 0; q < 2; ++q) s4[q] = *reinterpret_cast<const float4*>(sc + jb + 4 * q);
-      for (int g0 = 0; g0 < qg; g0 += kQgBatch) {
-        float4 i4[kQgBatch][2];
-#pragma unroll
-        for (int gg = 0; gg < kQgBatch; ++gg)
-          if (g0 + gg < qg)
-#pragma unroll
-            for (int q = 0; q < 2; ++q)
-              i4[gg][q] = __ldg(reinterpret_cast<const float4*>(
-                                    inc + static_cast<size_t>(g0 + gg) * NK + jb) + q);
-#pragma unroll
-        for (int gg = 0; gg < kQgBatch; ++gg)
-          if (g0 + gg < qg)
-#pragma unroll
-            for (int q = 0; q < 2; ++q) {
-              const float x[4] = {i4[gg][q].x, i4[gg][q].y, i4[gg][q].z, i4[gg][q].w};
-#pragma unroll
-              for (int e = 0; e < 4; ++e)
-                tv[4 * q + e] = (g0 + gg == 0) ? x[e] : __fadd_rn(tv[4 * q + e], x[e]);
-            }
-      }
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        sv[4 * q] = s4[q].x; sv[4 * q + 1] = s4[q].y; sv[4 * q + 2] = s4[q].z; sv[4 * q + 3] = s4[q].w;
-      }
-    } else {
-      for (int k = 0; k < n; ++k) {
-        sv[k] = sc[jb + k];
-        tv[k] = inc_group(a, inc, NK, jb + k);
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < kBatch; ++k)
-      if (k < n) {
-        const float acc = __fadd_rn(sv[k], tv[k]);
-        tot[k] = first ? acc : __fadd_rn(tot[k], acc);
-      }
-  };
-
   // Phase 1: scores and selection keys of every slot (positions of b0).
-  for (int jb = j0; jb < j1; jb += kBatch) {
-    const int n = min(kBatch, j1 - jb);
-    float tot[kBatch];
-    int pv[kBatch];
+  // CTA r of the cluster computes the slots of its share [r share, (r + 1)
+  // share) and stores each key into every CTA's key array, so that every CTA
+  // ends up with all M keys while each loads only its share of the old
+  // state; the accumulated scores stay with the share's CTA, which also
+  // writes the share's new state in phase 4.  acc_j = scores_j + (inc_0j +
+  // inc_1j + ...) in fp32, heads in order (Eq. 3); h2o_orig adds the batch
+  // entries' accumulated scores in ascending b.  (share is a multiple of R,
+  // so each thread's run of slots lies in one share.)
+  const int share = ((M + C - 1) / C + R - 1) / R * R;
+  const int lo = min(M, rank * share), hi = min(M, lo + share);
+  {
     const int* sp = pos_of(b0);
-    if (vec && n == kBatch) {
-      const int4 p0 = *reinterpret_cast<const int4*>(sp + jb);
-      const int4 p1 = *reinterpret_cast<const int4*>(sp + jb + 4);
-      pv[0] = p0.x; pv[1] = p0.y; pv[2] = p0.z; pv[3] = p0.w;
-      pv[4] = p1.x; pv[5] = p1.y; pv[6] = p1.z; pv[7] = p1.w;
-    } else {
-      for (int k = 0; k < n; ++k) pv[k] = sp[jb + k];
+    uint32_t key_dst[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) key_dst[r] = r < C ? cluster_addr(keys, r) : 0u;
+    for (int j = lo + tid; j < hi; j += kCThreads) {
+      const int pos = sp[j];
+      float tot = 0.f;
+      for (int bi = 0; bi < nb; ++bi) {
+        const float acc = __fadd_rn(scores_of(b0 + bi)[j], inc_group(a, inc_of(b0 + bi), NK, j));
+        tot = bi == 0 ? acc : __fadd_rn(tot, acc);
+      }
+      const uint32_t key = make_key(tot, pos, thr, a.policy, t_choice(a));
+      const uint32_t off = static_cast<uint32_t>(j) * 4u;
+#pragma unroll
+      for (int r = 0; r < 8; ++r)
+        if (r < C) st_cluster_u32(key_dst[r] + off, key);
+      if (!orig) accs[j] = tot;
     }
-    // h2o_orig sums the batch entries in ascending b
-    for (int bi = 0; bi < nb; ++bi) add_acc(b0 + bi, jb, n, tot, bi == 0);
-    for (int k = 0; k < n; ++k) {
-      keys[jb + k] = make_key(tot[k], pv[k], thr, a.policy, t_choice(a));
-      if (!orig) accs[jb + k] = tot[k];
+    // scores of the new tokens (their own columns M + c, summed over the
+    // group), 1/C of them here, into every CTA
+    if (!orig) {
+      const int cs = (S + C - 1) / C;
+      uint32_t ns_dst[8];
+#pragma unroll
+      for (int r = 0; r < 8; ++r) ns_dst[r] = r < C ? cluster_addr(nscore, r) : 0u;
+      for (int c = rank * cs + tid; c < min(S, rank * cs + cs); c += kCThreads) {
+        const uint32_t v = __float_as_uint(inc_group(a, inc_of(b0) + M, NK, c));
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+          if (r < C) st_cluster_u32(ns_dst[r] + static_cast<uint32_t>(c) * 4u, v);
+      }
     }
   }
-  // scores of the new tokens: their own columns M + c, summed over the group
-  if (!orig)
-    for (int c = tid; c < S; c += kCThreads) nscore[c] = inc_group(a, inc_of(b0) + M, NK, c);
-  // Every CTA of the cluster has read the old state before CTA 0 rewrites it.
+  // Every CTA of the cluster has read the old state before CTA 0 rewrites it,
+  // and every CTA's keys (and CTA 0's scores) are in place.
   cluster_sync_all();
 
+  // This thread's keys, slots j0 .. j1 - 1, are held in registers for the
+  // selection passes (16-byte loads: a run of R slots read one key at a time
+  // would hit the same shared-memory banks from every lane); long runs
+  // (M > 8192) are read from shared memory.
+  const int nR = j1 - j0;
+  const bool in_regs = R <= kRegKeys;
+  uint32_t kr[kRegKeys];
+#pragma unroll
+  for (int k = 0; k < kRegKeys; ++k) kr[k] = 0u;
+  if (in_regs) {
+    if (R % 4 == 0) {
+#pragma unroll
+      for (int q = 0; q < kRegKeys / 4; ++q)
+        if (4 * q < nR) {
+          const uint4 v = *reinterpret_cast<const uint4*>(keys + j0 + 4 * q);
+          kr[4 * q] = v.x; kr[4 * q + 1] = v.y; kr[4 * q + 2] = v.z; kr[4 * q + 3] = v.w;
+        }
+    } else {
+#pragma unroll
+      for (int k = 0; k < kRegKeys; ++k)
+        if (k < nR) kr[k] = keys[j0 + k];
+    }
+  }
+  // body(key, j) for this thread's slots in slot order
+  auto for_keys = [&](auto&& body) {
+    if (in_regs) {
+#pragma unroll
+      for (int k = 0; k < kRegKeys; ++k)
+        if (k < nR) body(kr[k], j0 + k);
+    } else {
+      for (int j = j0; j < j1; ++j) body(keys[j], j);
+    }
+  };
+
   // Phase 2: radix select of the S-th smallest key T, and how many keys equal
-  // to T are taken (the lowest slots first).
+  // to T are taken (the lowest slots first).  One barrier per pass: every
+  // warp scans the pass's histogram itself, and the histograms rotate over
+  // three buffers: pass p counts into buffer p % 3 and clears buffer
+  // (p + 1) % 3, which the warps last read in pass p - 2, before barrier
+  // p - 1 that every warp has passed.
   uint32_t prefix = 0, mask = 0, kth = static_cast<uint32_t>(S);
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
-    for (int x = tid; x < 256; x += kCThreads) hist[x] = 0u;
-    __syncthreads();
-    for (int j = j0; j < j1; ++j) {
-      const uint32_t key = keys[j];
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
-    }
-    __syncthreads();
-    if (pass == 0 && static_cast<uint32_t>(M) - hist[255] < static_cast<uint32_t>(S)) {
-      if (tid == 0 && rank == 0) atomicOr(a.err, 2);
-      return;  // uniform over the cluster: every CTA computed the same histogram
-    }
-    if (warp == 0) {
-      uint32_t c[8], s = 0;
-#pragma unroll
-      for (int x = 0; x < 8; ++x) {
-        c[x] = hist[8 * lane + x];
-        s += c[x];
-      }
-      uint32_t incl = s;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      uint32_t run = incl - s;
-#pragma unroll
-      for (int x = 0; x < 8; ++x) {
-        if (run < kth && kth <= run + c[x]) {
-          bcast[0] = static_cast<uint32_t>(8 * lane + x);
-          bcast[1] = kth - run;
+    uint32_t* hp = hist[pass % 3];
+    // neighbouring slots mostly share a digit (the high digits of similar
+    // scores): a thread adds runs of equal digits with one atomic each
+    {
+      uint32_t run_bin = 256u, run = 0u;
+      for_keys([&](uint32_t key, int) {
+        if ((key & mask) != prefix) return;
+        const uint32_t bin = (key >> shift) & 255u;
+        if (bin != run_bin) {
+          if (run) atomicAdd(&hp[run_bin], run);
+          run_bin = bin;
+          run = 0u;
         }
-        run += c[x];
-      }
+        ++run;
+      });
+      if (run) atomicAdd(&hp[run_bin], run);
     }
+    if (pass > 0)
+      for (int x = tid; x < 256; x += kCThreads) hist[(pass + 1) % 3][x] = 0u;
     __syncthreads();
-    prefix |= bcast[0] << shift;
+    if (pass == 0 && static_cast<uint32_t>(M) - hp[255] < static_cast<uint32_t>(S)) {
+      if (tid == 0 && rank == 0) atomicOr(a.err, 2);
+      // uniform over the cluster: every CTA computed the same histogram; the
+      // rows loaded for the copies land before the CTA's shared memory goes
+      if (prefetch && n_rows > 0) {
+        volatile int never = 0;
+        wait_bar(&rows_bar, 0, &never, kWaitLimitNs);
+      }
+      return;
+    }
+    // the bin holding the kth key: lane l sums bins 8l .. 8l + 7, a warp
+    // scan of the sums, and the lane whose range holds kth finds the bin
+    uint32_t c[8], sum = 0;
+    const uint4 v0 = reinterpret_cast<const uint4*>(hp)[2 * lane];
+    const uint4 v1 = reinterpret_cast<const uint4*>(hp)[2 * lane + 1];
+    c[0] = v0.x; c[1] = v0.y; c[2] = v0.z; c[3] = v0.w;
+    c[4] = v1.x; c[5] = v1.y; c[6] = v1.z; c[7] = v1.w;
+#pragma unroll
+    for (int x = 0; x < 8; ++x) sum += c[x];
+    uint32_t incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    uint32_t run = incl - sum, bin = 0u, rem = 0u;
+    const bool here = run < kth && kth <= incl;
+#pragma unroll
+    for (int x = 0; x < 8; ++x) {
+      if (run < kth && kth <= run + c[x]) {
+        bin = static_cast<uint32_t>(8 * lane + x);
+        rem = kth - run;
+      }
+      run += c[x];
+    }
+    const int src = __ffs(__ballot_sync(0xffffffffu, here)) - 1;
+    bin = __shfl_sync(0xffffffffu, bin, src);
+    rem = __shfl_sync(0xffffffffu, rem, src);
+    prefix |= bin << shift;
     mask |= 255u << shift;
-    kth = bcast[1];
-    __syncthreads();
+    kth = rem;
   }
   const uint32_t T = prefix, take_eq = kth;
 
@@ -439,19 +490,20 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   // halves (M < 65536), gives each slot's eviction rank: the slots below T
   // before it plus the taken slots equal to T before it.
   uint32_t n_lt = 0, n_eq = 0;
-  for (int j = j0; j < j1; ++j) {
-    n_lt += keys[j] < T;
-    n_eq += keys[j] == T;
-  }
+  for_keys([&](uint32_t key, int) {
+    n_lt += key < T;
+    n_eq += key == T;
+  });
   uint32_t tot;
   const uint32_t before = block_excl_scan(n_lt | (n_eq << 16), warp_tot, &tot);
 
-  // Phase 4: evicted slots get ranks 0..S-1; CTA 0 writes the new state of
-  // every batch entry the cluster owns.
+  // Phase 4: evicted slots get ranks 0..S-1 (every CTA needs all of them for
+  // its share of the row copies); the CTA whose share holds a thread's slots
+  // writes their new state for every batch entry the cluster owns.
   {
+    const bool mine = j0 >= lo && j0 < hi;
     uint32_t lt_b = before & 0xFFFFu, eq_b = before >> 16;
-    for (int j = j0; j < j1; ++j) {
-      const uint32_t key = keys[j];
+    for_keys([&](uint32_t key, int j) {
       const bool eq = key == T;
       const bool sel0 = key < T || (eq && eq_b < take_eq);
       const uint32_t c = lt_b + min(eq_b, take_eq);
@@ -459,7 +511,7 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
       lt_b += key < T;
       eq_b += eq;
       if (sel) elist[c] = j;
-      if (rank == 0) {
+      if (mine) {
         for (int bi = 0; bi < nb; ++bi) {
           const int b = b0 + bi;
           const size_t g = static_cast<size_t>(b) * a.Hkv + h;
@@ -475,23 +527,53 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
           }
         }
       }
-    }
-  }
-  if (rank == 0 && !orig) {
-    float* sc = scores_of(b0);
-    if (vec) {
-      for (int j = j0; j < j1; j += 4)
-        *reinterpret_cast<float4*>(sc + j) = *reinterpret_cast<const float4*>(accs + j);
-    } else {
-      for (int j = j0; j < j1; ++j) sc[j] = accs[j];
+    });
+    if (mine && !orig) {
+      float* sc = scores_of(b0);
+      if (vec) {
+        for (int j = j0; j < j1; j += 4)
+          *reinterpret_cast<float4*>(sc + j) = *reinterpret_cast<const float4*>(accs + j);
+      } else {
+        for (int j = j0; j < j1; ++j) sc[j] = accs[j];
+      }
     }
   }
   __syncthreads();
 
+  const int n_sel = min(static_cast<int>((tot & 0xFFFFu) + min(tot >> 16, take_eq)), S);
+  if (prefetch) {
+    // Phase 5 (rows in shared memory): the ranks [c_lo, c_lo + n_rows) of
+    // batch entry b0, 16-byte pieces from the rows loaded at the start
+    if (n_rows <= 0) return;
+    const bool landed = wait_bar(&rows_bar, 0, &abort_flag, kWaitLimitNs);
+    if (!landed) {
+      // the copies may still be in flight: give them time before the CTA's
+      // shared memory goes away, and report
+      const uint64_t t0 = global_timer_ns();
+      while (global_timer_ns() - t0 < 1000000ull) {
+      }
+      if (tid == 0) atomicOr(a.err, H2O_DEVERR_TIMEOUT);
+      return;
+    }
+    const int vecs = a.d / 8;  // 16-byte pieces per row
+    const int n_cp = min(n_rows, n_sel - c_lo);
+    const int pieces = n_cp * 2 * vecs;
+    const size_t g = static_cast<size_t>(b0) * a.Hkv + h;
+    for (int x = tid; x < pieces; x += kCThreads) {
+      const int piece = x % vecs;
+      const int rv = x / vecs;  // row * 2 + (0 = K, 1 = V)
+      const int r = rv >> 1;
+      const bool is_v = rv & 1;
+      const uint4 v = reinterpret_cast<const uint4*>(
+          rowbuf + (static_cast<size_t>(is_v ? c_per : 0) + r) * a.d)[piece];
+      uint16_t* d = (is_v ? a.v_cache : a.k_cache) + (g * M + elist[c_lo + r]) * a.d;
+      reinterpret_cast<uint4*>(d)[piece] = v;
+    }
+    return;
+  }
   // Phase 5: this CTA's share of the K/V row copies (ranks c = rank mod C) of
   // every batch entry the cluster owns, 16-byte pieces, four loads in flight
   // per thread before their stores.
-  const int n_sel = min(static_cast<int>((tot & 0xFFFFu) + min(tot >> 16, take_eq)), S);
   const int rows = a.k_cache != nullptr && n_sel > rank ? (n_sel - 1 - rank) / C + 1 : 0;
   const int vecs = a.d / 8;  // 16-byte pieces per row
   const int per_b = rows * 2 * vecs;
@@ -749,11 +831,17 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   int C = (a.S + 63) / 64;
   C = C < 1 ? 1 : (C > 8 ? 8 : C);
+  // the chunk rows a CTA writes are loaded into shared memory at its start
+  // when they fit (one batch entry per cluster, rows to copy)
+  const size_t rows_off = (smem + 15) / 16 * 16;
+  const size_t rows_bytes = 2 * static_cast<size_t>((a.S + C - 1) / C) * a.d * sizeof(uint16_t);
+  const int prefetch = a.k_cache != nullptr && a.policy != H2O_POLICY_ORIG &&
+                       rows_off + rows_bytes <= kMaxClusterSmem;
   cudaLaunchConfig_t cfg = {};
   const int groups = a.policy == H2O_POLICY_ORIG ? a.Hkv : a.B * a.Hkv;
   cfg.gridDim = dim3(static_cast<unsigned>(groups * C));
   cfg.blockDim = dim3(kCThreads);
-  cfg.dynamicSmemBytes = smem;
+  cfg.dynamicSmemBytes = prefetch ? rows_off + rows_bytes : smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -762,7 +850,7 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, update_cluster_kernel, a, C);
+  return cudaLaunchKernelEx(&cfg, update_cluster_kernel, a, C, prefetch);
 }
 
 }  // namespace h2o

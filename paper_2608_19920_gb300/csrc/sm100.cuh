@@ -110,6 +110,12 @@ __device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t cta) {
   return r;
 }
 
+// 32-bit store to a shared::cluster address (this CTA's shared memory or
+// another CTA's of the cluster, from cluster_addr).
+__device__ __forceinline__ void st_cluster_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
 // Arrive on an mbarrier given by shared::cluster address (possibly in another
 // CTA of the cluster).  Default semantics (release at CTA scope): enough to
 // order this thread's tcgen05 operations (after tcgen05.fence::before_thread_sync)

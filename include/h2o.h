@@ -32,13 +32,9 @@
  *
  * Conventions for every call:
  *  - All array arguments are DEVICE pointers, allocated and owned by the
- *    caller.  The forward, update, replay and 8-bit calls allocate no device
- *    memory (the scratch of h2o_sdpa_decode_static and the error word are
- *    static device arrays) and keep no per-call state.  The exception is
- *    h2o_sdpa_chunk_backward: its GEMMs run on cuBLASLt, and its first call
- *    on a device creates one cuBLASLt handle there that lives until exit; the
- *    handle's own allocations belong to the library (the matrices themselves
- *    go to the caller's workspace).
+ *    caller.  No call allocates device memory (the scratch of
+ *    h2o_sdpa_decode_static and the error word are static device arrays) or
+ *    keeps per-call state; every kernel is this library's own (no cuBLAS).
  *    Every array is dense, row-major (C order) with the shape given, and must
  *    be 16-byte aligned.
  *  - The library resolves some per-device state on its first call on a
@@ -96,7 +92,7 @@ enum {
   H2O_ERR_TIMEOUT = -8,     /* device: a bounded wait ran out (reported by h2o_device_errors) */
   H2O_ERR_DEVICE = -9,      /* device: fewer eviction candidates than S, etc. */
   H2O_ERR_NODEVICE = -10,   /* no usable sm_100-family GPU is current */
-  H2O_ERR_BLAS = -11        /* a cuBLASLt call failed; its cublasStatus_t in h2o_last_cuda_error */
+  H2O_ERR_BLAS = -11        /* reserved: no call returns it */
 };
 
 /* Device error bits reported by h2o_device_errors(). */
@@ -372,13 +368,17 @@ H2O_API int h2o_sdpa_cache_q8(const h2o_dims_t* dims, int64_t pos0, float softma
  *   dq         (B, Hq, S, d) f32, written
  *   dk_cache, dv_cache (B, Hkv, M, d) f32, written (may be NULL when M == 0)
  *   dk_new, dv_new     (B, Hkv, S, d) f32, written
- *   workspace  at least h2o_backward_workspace_size(dims) bytes: 32 MiB for
- *              cuBLASLt plus the materialised (B Hkv) x (q_g S) x (M + S)
- *              score matrices (fp32 scores, bf16 P and dS)
+ *   workspace  at least h2o_backward_workspace_size(dims) bytes: two floats
+ *              per query row (each group's q_g S rows padded to a multiple
+ *              of 128), the rows' log-sum-exp and D
  *
- * The five contractions run on cuBLASLt (bf16 operands, fp32 accumulation);
- * a failure there returns H2O_ERR_BLAS.  Cache slots no row sees get zero
- * gradient.
+ * Three kernels on the stream: the chunk SDPA's first pass (the rows'
+ * log-sum-exp), D per row, and one fused tcgen05 kernel whose CTAs form
+ * either 128 rows of dq or 128 keys of dk and dv.  Neither P nor dS is
+ * stored: each is rebuilt tile by tile in tensor memory, rounded to bf16 for
+ * the contractions (fp32 accumulation); no atomics, so results do not depend
+ * on scheduling.  Cache slots no row sees get zero gradient.  A group may
+ * hold at most 128 x 4096 query rows (q_g S), else H2O_ERR_UNSUPPORTED.
  */
 H2O_API int h2o_backward_workspace_size(const h2o_dims_t* dims, size_t* bytes);
 H2O_API int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,

@@ -66,9 +66,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     with open(os.path.join(BUILD, "ptxas.log"), "w") as f:
         f.write("\n".join(log))
     tmp = LIB + ".tmp"
-    cuda_lib = os.path.join(os.path.dirname(os.path.dirname(cc)), "lib64")
-    cmd = [cc, *ARCH, "-shared", "-o", tmp, *[o for _, o, _ in results], "-lcublasLt",
-           "-Xlinker", f"-rpath={cuda_lib}"]
+    cmd = [cc, *ARCH, "-shared", "-o", tmp, *[o for _, o, _ in results]]
     p = subprocess.run(cmd, capture_output=True, text=True)
     if p.returncode != 0:
         raise RuntimeError(f"link failed:\n{p.stdout}{p.stderr}")

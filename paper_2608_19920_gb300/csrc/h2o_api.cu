@@ -125,11 +125,14 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
               const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
               const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out, float* score_inc,
               void* workspace, size_t workspace_bytes, void* stream, bool cache_only,
-              const Q8Buffers* q8 = nullptr) {
+              const Q8Buffers* q8 = nullptr, float* lse = nullptr, int lse_stride = 0) {
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
-  if (!q || !out || !score_inc || (!cache_only && (!k_new || !v_new))) return H2O_ERR_NULL;
+  // lse (the backward's recomputation): the chunk kernel's pass 1 alone,
+  // which writes the rows' log-sum-exp and neither out nor score_inc
+  if (!q || (!lse && (!out || !score_inc)) || (!cache_only && (!k_new || !v_new)))
+    return H2O_ERR_NULL;
   // (q8: the codes were checked by the caller; the decode kernels need no rows)
   if (D.M > 0 && ((!q8 && (!k_cache || !v_cache)) || !slot_pos)) return H2O_ERR_NULL;
   if (misaligned(q) || misaligned(k_new) || misaligned(v_new) || misaligned(out) ||
@@ -143,8 +146,9 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
   int split_len = 0, n_split = 0;
   size_t ws_need = 0;
-  const bool decode = decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
-  if (!decode) ws_need = sdpa_colpart_bytes(D.B, D.Hq, D.S, D.M);
+  const bool decode =
+      !lse && decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
+  if (!decode) ws_need = lse ? 0 : sdpa_colpart_bytes(D.B, D.Hq, D.S, D.M);
   if (ws_need > 0 && (!workspace || workspace_bytes < ws_need)) return H2O_ERR_WORKSPACE;
   if (ws_need > 0 && misaligned(workspace)) return H2O_ERR_ALIGN;
   DeviceInfo* di = nullptr;
@@ -205,6 +209,8 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   a.score_inc = score_inc;
   a.err = di->err_word;
   a.colpart = ws_need > 0 ? static_cast<float*>(workspace) : nullptr;
+  a.lse = lse;
+  a.lse_stride = lse_stride;
 
   const uint64_t G = static_cast<uint64_t>(D.B) * D.Hkv;
   {
@@ -233,7 +239,7 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   const size_t inc_bytes = static_cast<size_t>(G) * qg * static_cast<size_t>(nk) * sizeof(float);
   cudaError_t e = read_back();
   if (e != cudaSuccess) return cuda_fail(e);
-  if (a.colpart == nullptr) {
+  if (a.colpart == nullptr && !lse) {
     e = cudaMemsetAsync(score_inc, 0, inc_bytes, s);
     if (e != cudaSuccess) return cuda_fail(e);
   }
@@ -402,7 +408,7 @@ const char* h2o_status_string(int s) {
     case H2O_ERR_TIMEOUT: return "a device-side bounded wait ran out";
     case H2O_ERR_DEVICE: return "device-side error (fewer eviction candidates than S)";
     case H2O_ERR_NODEVICE: return "no usable sm_100-family GPU is current";
-    case H2O_ERR_BLAS: return "a cuBLASLt call failed (status in h2o_last_cuda_error)";
+    case H2O_ERR_BLAS: return "reserved (no call returns it)";
     default: return "unknown status";
   }
 }
@@ -685,26 +691,50 @@ int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_
     return H2O_ERR_ALIGN;
   if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
   if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
+  const int qg = D.Hq / D.Hkv;
+  const int R = qg * D.S;                        // stacked query rows of a group
+  if ((R + kTileM - 1) / kTileM > kMaxKeyTiles) return H2O_ERR_UNSUPPORTED;
   if (!workspace || workspace_bytes < backward_workspace_bytes(D.B, D.Hq, D.Hkv, D.S, D.M))
     return H2O_ERR_WORKSPACE;
   DeviceInfo* di = nullptr;
   if ((st = current_device(&di)) != H2O_OK) return st;
+  if ((st = get_encoder()) != H2O_OK) return st;
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
-  BackwardArgs a = {};
+  BackwardArgs a;
+  std::memset(&a, 0, sizeof(a));
   a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
   a.slot_pos = slot_pos; a.out = out; a.dout = dout;
   a.dq = dq; a.dk_cache = dk_cache; a.dv_cache = dv_cache; a.dk_new = dk_new; a.dv_new = dv_new;
-  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = D.Hq / D.Hkv;
+  a.err = di->err_word;
+  a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = qg;
   a.pos0 = static_cast<int>(pos0);
   a.scale = scale;
   a.scale_log2 = scale * 1.4426950408889634f;
-  const BackwardStatus bs = launch_backward(a, workspace, static_cast<cudaStream_t>(stream));
-  if (bs.cuda != cudaSuccess) return cuda_fail(bs.cuda);
-  if (bs.blas != 0) {
-    t_last_cuda_error = bs.blas;
-    return H2O_ERR_BLAS;
+  const int Rp = backward_row_stride(qg, D.S);
+  const uint64_t G = static_cast<uint64_t>(D.B) * D.Hkv;
+  a.lse = static_cast<float*>(workspace);
+  a.drow = a.lse + G * Rp;
+  {
+    // 128-row boxes of the stacked query rows and of the key / value rows
+    const uint32_t box[3] = {64, static_cast<uint32_t>(kTileM), 1};
+    const uint64_t dr[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(R), G};
+    const uint64_t dn[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.S), G};
+    if ((st = encode(&a.tm_q, q, 3, dr, box)) != H2O_OK) return st;
+    if ((st = encode(&a.tm_do, dout, 3, dr, box)) != H2O_OK) return st;
+    if ((st = encode(&a.tm_kn, k_new, 3, dn, box)) != H2O_OK) return st;
+    if ((st = encode(&a.tm_vn, v_new, 3, dn, box)) != H2O_OK) return st;
+    if (D.M > 0) {
+      const uint64_t dc[3] = {static_cast<uint64_t>(D.d), static_cast<uint64_t>(D.M), G};
+      if ((st = encode(&a.tm_kc, k_cache, 3, dc, box)) != H2O_OK) return st;
+      if ((st = encode(&a.tm_vc, v_cache, 3, dc, box)) != H2O_OK) return st;
+    }
   }
-  return H2O_OK;
+  // each row's log-sum-exp, from the forward kernel's first pass
+  st = sdpa_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, k_new, v_new, slot_pos, nullptr,
+                 nullptr, nullptr, 0, stream, false, nullptr, a.lse, Rp);
+  if (st != H2O_OK) return st;
+  const cudaError_t e = launch_backward(a, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? H2O_OK : cuda_fail(e);
 }
 
 int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores, void* stream) {

@@ -1,28 +1,35 @@
-// Gradient of the chunk SDPA under the position mask (§3.1 Eq. 2, mask of
-// §3.3.1), the backward pass the paper's fine-tuning runs through every chunk.
+// Gradient of the chunk SDPA (§3.1 Eq. 2 under the position mask of §3.3.1):
+// the backward pass the paper's fine-tuning runs through every chunk (§3.2,
+// §A.4).  For L = sum(out * dout), with m_ij the attention weights of the
+// forward, per (b, kv head) group with the q_g heads' rows stacked:
 //
-// For the loss sum(out * dout), per (b, kv head) group with its q_g query heads'
-// rows stacked (R = q_g S rows, the layout of q) and the keys [k_cache; k_new]
-// (N_k = M + S columns):
+//   D_i    = sum_d dout_id out_id
+//   dP_ij  = dout_i . v_j,   dS_ij = m_ij (dP_ij - D_i)
+//   dq_i   = scale sum_j dS_ij k_j
+//   dk_j   = scale sum_i dS_ij q_i,   dv_j = sum_i m_ij dout_i
 //
-//   S  = Q K^T                      (GEMM)
-//   P  = softmax(mask(scale S))     (masked row softmax, recomputed; bf16)
-//   D  = rowsum(dout * out)         (per row)
-//   dP = dout V^T                   (GEMM)
-//   dS = P * (dP - D)               (elementwise; bf16)
-//   dQ = scale dS K,  dK = scale dS^T Q,  dV = P^T dout   (GEMMs)
+// with m_ij = exp2(scale log2e q_i . k_j - lambda_i) rebuilt from each row's
+// log-sum-exp lambda (log2 units), which the forward kernel's pass 1 writes.
+// Hidden (i, j) pairs have m_ij = 0, so cache slots no row sees get zero
+// gradients.
 //
-// dK and dV of a KV head sum over its q_g heads because Q, dS and P stack the
-// heads' rows.  The five contractions are plain dense GEMMs, so they run on
-// cuBLASLt (bf16 operands, fp32 accumulation and outputs), batched over the
-// groups, in the caller's workspace; the mask, the softmax and dS run in the
-// kernels below.  The S x N_k matrices are materialised (fp32 S / dP, bf16 P
-// and dS), so the pass is bandwidth heavy; a fused kernel is future work.
-#include <cublasLt.h>
-
-#include <algorithm>
-#include <cstdint>
-#include <mutex>
+// Two tcgen05 kernels, neither materialising a score matrix and neither
+// using atomics (so the result does not depend on scheduling):
+//  * bwd_dq_kernel: one CTA per 128 stacked rows; per key tile, S = Q K^T and
+//    dP = dO V^T into TMEM, the softmax warps (one row per thread) form dS in
+//    bf16 over S's columns, and dQ += dS K accumulates in TMEM.
+//  * bwd_dkv_kernel: one CTA per 128-key tile; per tile of stacked rows,
+//    S^T = K Q^T and dP^T = V dO^T into TMEM (one key per lane), the softmax
+//    warps form P^T and dS^T in bf16 over those columns, and dV += P^T dO,
+//    dK += dS^T Q accumulate in TMEM (A from TMEM, B = the row tile in
+//    shared memory).
+// Row and key tiles that no (row, key) pair of which is visible are skipped;
+// tiles every pair of which is visible take no mask.  Products whose B
+// operand is a row or key tile read along d (N = d) run as one MMA per
+// 64-column panel.  Every wait is bounded; on expiry a CTA drains its MMAs,
+// frees TMEM and reports H2O_DEVERR_TIMEOUT.
+#include <climits>
+#include <cmath>
 
 #include "h2o_internal.h"
 #include "sm100.cuh"
@@ -30,441 +37,778 @@
 namespace h2o {
 namespace {
 
-constexpr int kRowThreads = 256;
-constexpr size_t kLtWorkspace = size_t(32) << 20;
+constexpr int kBT = 128;               // rows or keys per tile
+constexpr int kBwdSoftmaxWarps = 8;    // two teams of four warps (one per TMEM lane quarter)
+constexpr int kBwdFirstSoftmax = 2;    // warp 0 TMA, warp 1 MMA issue
+constexpr int kBwdThreads = 32 * (kBwdFirstSoftmax + kBwdSoftmaxWarps);  // 320
+constexpr int kBwdStages = 2;          // shared-memory ring of streamed tile pairs
+constexpr int kBwdBufs = 3;            // S / dP buffer pairs in TMEM
+constexpr uint8_t kBClsSkip = 0, kBClsFull = 1, kBClsPartial = 2;
+constexpr uint16_t kBPartial = 0x8000;  // tile-list entry: masked tile
+constexpr uint16_t kBIdxMask = 0x7FFF;
+constexpr int kDqStep = 64;            // keys per dq step (two steps per key tile)
 
-__device__ __forceinline__ uint16_t to_bf16(float x) {
-  return static_cast<uint16_t>(pack_bf16x2(x, 0.f) & 0xFFFFu);
+template <int D>
+struct BwdGeom {
+  static constexpr int kPanels = D / 64;
+  static constexpr int kTileBytes = kPanels * kBT * 128;  // 128 rows of D bf16
+  // dkv: stacked rows per step.  TMEM holds dV and dK (D columns each) and
+  // three buffers of S^T and dP^T (W columns each): 2D + 6W <= 512.
+  static constexpr int kW = D == 128 ? 32 : 64;
+  static constexpr int kStepsPerTile = kBT / kW;
+};
+
+// Shared memory of both kernels: two resident tiles (dq: Q and dO; dkv: K and
+// V), a ring of kBwdStages pairs of streamed tiles (dq: K_j, V_j; dkv: Q_i,
+// dO_i), per stage the streamed rows' lambda and D (dkv), the tile list.
+template <int D>
+struct __align__(1024) BwdSmem {
+  uint8_t res[2][BwdGeom<D>::kTileBytes];
+  uint8_t ring[kBwdStages][2][BwdGeom<D>::kTileBytes];
+  float rowv[kBwdStages][2][kBT];  // dkv: lambda and D of the stage's rows
+  uint64_t bar_res, bar_full[kBwdStages], bar_empty[kBwdStages];
+  uint64_t bar_sfull[kBwdBufs], bar_pfull[kBwdBufs], bar_done[kBwdBufs];
+  uint64_t bar_acc, bar_drain;
+  uint32_t taddr;
+  int abort_flag;
+  int n_tiles;
+  uint16_t tiles[kMaxKeyTiles];  // kBPartial | tile index
+  uint8_t cls[kMaxKeyTiles];
+};
+
+__device__ __forceinline__ bool bwait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  return wait_bar(bar, parity, abort, kWaitLimitNs);
 }
 
-__device__ __forceinline__ float from_bf16(uint16_t x) {
-  return __uint_as_float(static_cast<uint32_t>(x) << 16);
+// Stacked row r of a group -> (head within the group, chunk row i).
+__device__ __forceinline__ void split_row(int r, int S, int& g, int& i) {
+  g = r / S;
+  i = r - g * S;
 }
 
-__device__ __forceinline__ float block_reduce(float v, float* sh, bool is_max) {
+// D_i = dout_i . out_i (fp32) for every stacked row: one warp per row; row
+// r of group grp (memory row grp R + r) goes to drow[grp R_pad + r].
+template <int D>
+__global__ void __launch_bounds__(256) bwd_drow_kernel(const uint16_t* __restrict__ out,
+                                                      const uint16_t* __restrict__ dout,
+                                                      float* __restrict__ drow, int rows, int R,
+                                                      int R_pad) {
+  const int r = blockIdx.x * 8 + static_cast<int>(threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  constexpr int kPer = D / 32;  // elements per lane: 4 or 2
+  float s = 0.f;
+  if constexpr (kPer == 4) {
+    const uint2 o = reinterpret_cast<const uint2*>(out + static_cast<size_t>(r) * D)[lane];
+    const uint2 g = reinterpret_cast<const uint2*>(dout + static_cast<size_t>(r) * D)[lane];
+    const uint32_t ow[2] = {o.x, o.y}, gw[2] = {g.x, g.y};
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float y = __shfl_xor_sync(0xffffffffu, v, o);
-    v = is_max ? fmaxf(v, y) : v + y;
-  }
-  const int w = threadIdx.x >> 5;
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh[w] = v;
-  __syncthreads();
-  float r = sh[0];
-  for (int x = 1; x < kRowThreads / 32; ++x) r = is_max ? fmaxf(r, sh[x]) : r + sh[x];
-  return r;
-}
-
-// One CTA per stacked row: P (bf16) from the S row, and D.  (Measured against a
-// register-resident one-read variant and a warp-per-row online variant: this
-// plain three-pass form was the fastest of the three.)
-__global__ void __launch_bounds__(kRowThreads) bwd_softmax_kernel(const BackwardArgs a) {
-  __shared__ float sh[kRowThreads / 32];
-  const size_t row = blockIdx.x;  // g * R + r
-  const int R = a.qg * a.S;
-  const size_t g = row / R;
-  const int r = static_cast<int>(row % R);
-  const int gg = r / a.S, i = r % a.S;
-  const int NK = a.M + a.S;
-  const float* srow = a.sbuf + row * NK;
-  uint16_t* prow = a.pbuf + row * NK;
-  const int32_t* sp = a.slot_pos + g * a.M;
-  const int qpos = a.pos0 + i;
-  auto visible = [&](int j) -> bool {
-    if (j < a.M) {
-      const int pos = __ldg(sp + j);
-      return pos >= 0 && pos <= qpos;
-    }
-    return j - a.M <= i;
-  };
-  float mx = -INFINITY;
-  for (int j = threadIdx.x; j < NK; j += kRowThreads)
-    if (visible(j)) mx = fmaxf(mx, srow[j] * a.scale_log2);
-  mx = block_reduce(mx, sh, true);
-  float sum = 0.f;
-  for (int j = threadIdx.x; j < NK; j += kRowThreads)
-    if (visible(j)) sum += fast_exp2(srow[j] * a.scale_log2 - mx);
-  sum = block_reduce(sum, sh, false);
-  const float lam = mx + fast_log2(sum);  // every row sees its own token
-  for (int j = threadIdx.x; j < NK; j += kRowThreads)
-    prow[j] = to_bf16(visible(j) ? fast_exp2(srow[j] * a.scale_log2 - lam) : 0.f);
-  // D = dout . out of this row (query head h q_g + gg, token i)
-  const int b = static_cast<int>(g / a.Hkv), h = static_cast<int>(g % a.Hkv);
-  const size_t orow = (static_cast<size_t>(b * a.Hq + h * a.qg + gg) * a.S + i) * a.d;
-  float dsum = 0.f;
-  for (int e = threadIdx.x; e < a.d; e += kRowThreads)
-    dsum += from_bf16(a.dout[orow + e]) * from_bf16(a.out[orow + e]);
-  dsum = block_reduce(dsum, sh, false);
-  if (threadIdx.x == 0) a.drow[row] = dsum;
-}
-
-// dS = P * (dP - D), bf16, over every stacked row and key column; CTAs take
-// whole rows.
-__global__ void __launch_bounds__(kRowThreads) bwd_ds_kernel(const BackwardArgs a) {
-  const int NK = a.M + a.S;
-  const size_t rows = static_cast<size_t>(a.B) * a.Hkv * a.qg * a.S;
-  for (size_t row = blockIdx.x; row < rows; row += gridDim.x) {
-    const float dr = a.drow[row];
-    const size_t base = row * NK;
-    for (int j = threadIdx.x; j < NK; j += kRowThreads) {
-      const float p = from_bf16(a.pbuf[base + j]);
-      a.dsbuf[base + j] = to_bf16(p * (a.sbuf[base + j] - dr));
-    }
-  }
-}
-
-// ---- vectorised forms: N_k and M multiples of 4, 16-byte aligned buffers ----
-// A row of N_k fp32 scores is then a run of float4s, and no group of four
-// columns straddles the cache / chunk boundary.  Each thread keeps four 16-byte
-// loads in flight: one 4-byte load per thread (the scalar kernels above) holds
-// too few bytes in flight per SM to cover the HBM latency.
-constexpr int kVecUnroll = 4;
-
-// Visibility of columns 4v .. 4v+3 of row (query i, position qpos) as a 4-bit
-// mask: cache slots by their positions p (§3.3.1), chunk columns causally.
-__device__ __forceinline__ unsigned vis_mask4(int v, int mv, int4 p, int qpos, int i, int M) {
-  if (v < mv)
-    return static_cast<unsigned>(p.x >= 0 && p.x <= qpos) |
-           static_cast<unsigned>(p.y >= 0 && p.y <= qpos) << 1 |
-           static_cast<unsigned>(p.z >= 0 && p.z <= qpos) << 2 |
-           static_cast<unsigned>(p.w >= 0 && p.w <= qpos) << 3;
-  const int n = i - (4 * v - M) + 1;  // chunk columns t .. t+3 visible while t <= i
-  return n <= 0 ? 0u : n >= 4 ? 15u : (1u << n) - 1u;
-}
-
-// (m, l) <- the pair whose sum of 2^(y - m) covers both sets: the online
-// softmax merge; an empty set is (-inf, 0).
-__device__ __forceinline__ void merge_ml(float& m, float& l, float m2, float l2) {
-  const float mn = fmaxf(m, m2);
-  if (mn == -INFINITY) return;
-  l = l * fast_exp2(m - mn) + l2 * fast_exp2(m2 - mn);
-  m = mn;
-}
-
-// The softmax pass with one DRAM read of the S row, one CTA of kVecThreads per
-// stacked row: a per-thread online (max, sum) over base-2 logits and D's dot
-// product, merged across the CTA at one barrier.  kKeep (the row fits one trip
-// of kVecUnroll float4s per thread, N_k <= 4096): the write pass takes the
-// values still held in registers; otherwise it reads the row again while it is
-// in L2 (streaming, its last use).  Four CTAs per SM: 512-thread CTAs (one trip
-// up to N_k = 8192, two per SM) measured slower, having fewer rows in flight.
-constexpr int kVecThreads = 256;
-
-__device__ __forceinline__ void online4(float4 x, unsigned vm, float c, float& m, float& l) {
-  if (vm == 0) return;
-  const float y0 = (vm & 1u) ? x.x * c : -INFINITY;
-  const float y1 = (vm & 2u) ? x.y * c : -INFINITY;
-  const float y2 = (vm & 4u) ? x.z * c : -INFINITY;
-  const float y3 = (vm & 8u) ? x.w * c : -INFINITY;
-  const float mx = fmaxf(fmaxf(y0, y1), fmaxf(y2, y3));
-  if (mx > m) {
-    l *= fast_exp2(m - mx);
-    m = mx;
-  }
-  l += (fast_exp2(y0 - m) + fast_exp2(y1 - m)) + (fast_exp2(y2 - m) + fast_exp2(y3 - m));
-}
-
-__device__ __forceinline__ uint2 probs4(float4 x, unsigned vm, float c, float lam) {
-  const float e0 = (vm & 1u) ? fast_exp2(x.x * c - lam) : 0.f;
-  const float e1 = (vm & 2u) ? fast_exp2(x.y * c - lam) : 0.f;
-  const float e2 = (vm & 4u) ? fast_exp2(x.z * c - lam) : 0.f;
-  const float e3 = (vm & 8u) ? fast_exp2(x.w * c - lam) : 0.f;
-  return make_uint2(pack_bf16x2(e0, e1), pack_bf16x2(e2, e3));
-}
-
-template <bool kKeep>
-__global__ void __launch_bounds__(kVecThreads, 4) bwd_softmax_vec_kernel(const BackwardArgs a) {
-  constexpr int T = kVecThreads, U = kVecUnroll, W = kVecThreads / 32;
-  __shared__ float sh_m[W], sh_l[W], sh_d[W];
-  const size_t row = blockIdx.x;
-  const int R = a.qg * a.S;
-  const size_t g = row / R;
-  const int r = static_cast<int>(row % R);
-  const int gg = r / a.S, i = r % a.S;
-  const int nv = (a.M + a.S) >> 2, mv = a.M >> 2;
-  const float4* s4 = reinterpret_cast<const float4*>(a.sbuf) + row * nv;
-  uint2* p4 = reinterpret_cast<uint2*>(a.pbuf) + row * nv;
-  const int4* sp4 = reinterpret_cast<const int4*>(a.slot_pos + g * a.M);
-  const int qpos = a.pos0 + i;
-  const float c = a.scale_log2;
-
-  // D = dout . out of this row (query head h q_g + gg, token i), d <= T: the
-  // two loads go out ahead of the row's and are used after them
-  const int b = static_cast<int>(g / a.Hkv), h = static_cast<int>(g % a.Hkv);
-  const size_t orow = (static_cast<size_t>(b * a.Hq + h * a.qg + gg) * a.S + i) * a.d;
-  uint16_t dv = 0, ov = 0;
-  if (static_cast<int>(threadIdx.x) < a.d) {
-    dv = a.dout[orow + threadIdx.x];
-    ov = a.out[orow + threadIdx.x];
-  }
-
-  float m = -INFINITY, l = 0.f;
-  float4 x[U];
-  unsigned vm[U];
-#pragma unroll
-  for (int u = 0; u < U; ++u) vm[u] = 0u;
-  for (int v0 = threadIdx.x; v0 < nv; v0 += U * T) {
-    int4 p[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int v = v0 + u * T;
-      x[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-      p[u] = make_int4(-1, -1, -1, -1);
-      if (v < nv) x[u] = s4[v];
-      if (v < mv) p[u] = __ldg(sp4 + v);
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int v = v0 + u * T;
-      vm[u] = v < nv ? vis_mask4(v, mv, p[u], qpos, i, a.M) : 0u;
-      online4(x[u], vm[u], c, m, l);
-    }
-  }
-  float dsum = from_bf16(dv) * from_bf16(ov);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    merge_ml(m, l, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, l, o));
-    dsum += __shfl_xor_sync(0xffffffffu, dsum, o);
-  }
-  if ((threadIdx.x & 31) == 0) {
-    sh_m[threadIdx.x >> 5] = m;
-    sh_l[threadIdx.x >> 5] = l;
-    sh_d[threadIdx.x >> 5] = dsum;
-  }
-  __syncthreads();
-  m = sh_m[0];
-  l = sh_l[0];
-  for (int w = 1; w < W; ++w) merge_ml(m, l, sh_m[w], sh_l[w]);
-  const float lam = m + fast_log2(l);  // every row sees its own token
-  if (threadIdx.x == 0) {
-    float dr = 0.f;
-    for (int w = 0; w < W; ++w) dr += sh_d[w];
-    a.drow[row] = dr;
-  }
-
-  if constexpr (kKeep) {  // nv <= U T: x and vm hold this thread's whole share
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int v = threadIdx.x + u * T;
-      if (v < nv) p4[v] = probs4(x[u], vm[u], c, lam);
+    for (int x = 0; x < 2; ++x) {
+      s = fmaf(__uint_as_float(ow[x] << 16), __uint_as_float(gw[x] << 16), s);
+      s = fmaf(__uint_as_float(ow[x] & 0xFFFF0000u), __uint_as_float(gw[x] & 0xFFFF0000u), s);
     }
   } else {
-    for (int v0 = threadIdx.x; v0 < nv; v0 += U * T) {
-      int4 p[U];
+    const uint32_t o = reinterpret_cast<const uint32_t*>(out + static_cast<size_t>(r) * D)[lane];
+    const uint32_t g = reinterpret_cast<const uint32_t*>(dout + static_cast<size_t>(r) * D)[lane];
+    s = fmaf(__uint_as_float(o << 16), __uint_as_float(g << 16), s);
+    s = fmaf(__uint_as_float(o & 0xFFFF0000u), __uint_as_float(g & 0xFFFF0000u), s);
+  }
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int v = v0 + u * T;
-        x[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        p[u] = make_int4(-1, -1, -1, -1);
-        if (v < nv) x[u] = __ldcs(s4 + v);
-        if (v < mv) p[u] = __ldg(sp4 + v);
-      }
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane == 0) drow[static_cast<size_t>(r / R) * R_pad + r % R] = s;
+}
+
+// K-major 128-byte-swizzled operand descriptors of a 128-row tile (kPanels
+// panels of 64 columns): the eight K-steps of 16 elements along D.
+template <int D>
+__device__ __forceinline__ void kmajor_steps(uint32_t base, uint64_t (&d)[D / 16]) {
+  const uint64_t d0 = sdesc_sw128(base, 16, 1024);
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int v = v0 + u * T;
-        if (v < nv) p4[v] = probs4(x[u], vis_mask4(v, mv, p[u], qpos, i, a.M), c, lam);
-      }
-    }
+  for (int kk = 0; kk < D / 16; ++kk)
+    d[kk] = d0 + static_cast<uint64_t>((kBT * 128 >> 4) * (kk / 4) + 2 * (kk % 4));
+}
+
+// MN-major descriptor of panel p of a 128-row tile read with K = rows and
+// N = the panel's 64 columns; K-step kk covers rows 16 kk .. 16 kk + 15.
+__device__ __forceinline__ uint64_t mn_step(uint32_t base, int p, int kk) {
+  return sdesc_sw128(base + p * kBT * 128, kBT * 128, 1024) + static_cast<uint64_t>(128 * kk);
+}
+
+// Warp-uniform bounded wait: every lane waits, and the warp goes on only if
+// all of them saw the phase complete (so that the .sync.aligned TMEM
+// instructions after it are reached by the whole warp or by none of it).
+__device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const bool r = bwait(bar, parity, abort);
+  return __all_sync(0xffffffffu, r) != 0;
+}
+
+// Smallest and largest chunk row i among the valid stacked rows r0 .. r0+127
+// of a group (R = q_g S rows, row r = head r / S, chunk row r % S); a tile that
+// crosses a head boundary holds both i = S - 1 and i = 0.
+__device__ __forceinline__ void row_tile_range(int r0, int R, int S, int& i_min, int& i_max) {
+  const int r1 = min(r0 + kBT, R) - 1;
+  const int g0 = r0 / S, g1 = r1 / S;
+  if (g0 == g1) {
+    i_min = r0 - g0 * S;
+    i_max = r1 - g0 * S;
+  } else {
+    i_min = 0;
+    i_max = S - 1;
   }
 }
 
-// dS = P * (dP - D), one CTA per stacked row, four float4 / 8-byte loads in
-// flight per thread; dP is read for the last time (streaming).
-__global__ void __launch_bounds__(kRowThreads, 4) bwd_ds_vec_kernel(const BackwardArgs a) {
-  const size_t row = blockIdx.x;
-  const int nv = (a.M + a.S) >> 2;
-  const float dr = a.drow[row];
-  const float4* s4 = reinterpret_cast<const float4*>(a.sbuf) + row * nv;
-  const uint2* p4 = reinterpret_cast<const uint2*>(a.pbuf) + row * nv;
-  uint2* ds4 = reinterpret_cast<uint2*>(a.dsbuf) + row * nv;
-  for (int v0 = threadIdx.x; v0 < nv; v0 += kVecUnroll * kRowThreads) {
-    float4 x[kVecUnroll];
-    uint2 p[kVecUnroll];
+// Compacts the classes in sm.cls[0 .. total) into the ordered list of tiles
+// to visit (one warp).
+template <int D>
+__device__ __forceinline__ void build_tile_list(BwdSmem<D>& sm, int total, uint32_t lane) {
+  int n = 0;
+  for (int base = 0; base < total; base += 32) {
+    const int t = base + static_cast<int>(lane);
+    const uint8_t cl = t < total ? sm.cls[t] : kBClsSkip;
+    const uint32_t m = __ballot_sync(0xffffffffu, cl != kBClsSkip);
+    if (cl != kBClsSkip)
+      sm.tiles[n + __popc(m & ((1u << lane) - 1u))] =
+          static_cast<uint16_t>(t | (cl == kBClsPartial ? kBPartial : 0));
+    n += __popc(m);
+  }
+  if (lane == 0) sm.n_tiles = n;
+}
+
+template <int D>
+__device__ __forceinline__ void init_barriers(BwdSmem<D>& sm) {
+  bar_init(&sm.bar_res, 1);
+  for (int s = 0; s < kBwdStages; ++s) {
+    bar_init(&sm.bar_full[s], 1);
+    bar_init(&sm.bar_empty[s], 1);
+  }
+  for (int b = 0; b < kBwdBufs; ++b) {
+    bar_init(&sm.bar_sfull[b], 1);
+    bar_init(&sm.bar_pfull[b], kBwdSoftmaxWarps / 2);  // the four warps of one team
+    bar_init(&sm.bar_done[b], 1);
+  }
+  bar_init(&sm.bar_acc, 1);
+  bar_init(&sm.bar_drain, 1);
+  sm.abort_flag = 0;
+  fence_bar_init();
+}
+
+// After an abort: lets the copies still in flight land before the CTA's
+// shared memory goes away (at most the latest load of each stage).
+template <int D>
+__device__ void drain_loads(BwdSmem<D>& sm, const int (&uses)[kBwdStages], bool res_issued) {
+  volatile int never = 0;
+  if (res_issued) wait_bar(&sm.bar_res, 0, &never, 100000000ull);
+  for (int s = 0; s < kBwdStages; ++s)
+    if (uses[s] > 0) wait_bar(&sm.bar_full[s], (uses[s] - 1) & 1, &never, 100000000ull);
+}
+
+// Issuer epilogue: no MMA may still be running when TMEM is freed.
+template <int D>
+__device__ __forceinline__ void drain_mmas(BwdSmem<D>& sm) {
+  mma_commit(&sm.bar_drain);
+  volatile int never = 0;
+  wait_bar(&sm.bar_drain, 0, &never, kWaitLimitNs);
+}
+
+// ------------------------------------------------------------------ dq ------
+// One CTA per 128 stacked rows r0 .. r0+127 of a group.  The key
+// tiles (cache tiles, then chunk tiles) run as steps of 64 keys, step n in
+// TMEM buffer n % 3: S at columns 128 + 128 b, dP 64 columns after it; the
+// softmax writes bf16 dS over S's first 32 columns, dQ (D columns from 0)
+// accumulates dS K.  The issuer puts step n+1's S and dP ahead of step n's
+// dQ, so the tensor pipe has work while the softmax runs; a buffer is
+// refilled only after the dQ that read it has completed (MMAs into
+// different accumulators are not ordered by issue).
+template <int D>
+__device__ __forceinline__ void bwd_dq(const BackwardArgs& a, BwdSmem<D>& sm, int rt, int grp) {
+  using G = BwdGeom<D>;
+  constexpr int P = G::kPanels;
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const uint32_t lane = tid & 31;
+  const int R = a.qg * a.S;
+  const int r0 = rt * kBT;
+  const int n_ct = (a.M + kBT - 1) / kBT;
+  const int n_nt = (a.S + kBT - 1) / kBT;
+  int i_min, i_max;
+  row_tile_range(r0, R, a.S, i_min, i_max);
+
+  if (tid == 0) init_barriers(sm);
+  if (warp == 1) {
+    tmem_alloc(&sm.taddr, 512);
+    tmem_relinquish();
+  }
+  // key tiles against this CTA's rows: skipped when no row sees a key of
+  // it, unmasked when every row sees every key (rows past R have lambda =
+  // +inf, so their weights are 0 either way)
+  if (warp >= kBwdFirstSoftmax) {
+    const int sw = warp - kBwdFirstSoftmax;
+    const int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
+    for (int ct = sw; ct < n_ct; ct += kBwdSoftmaxWarps) {
+      bool any = false, all = true;
 #pragma unroll
-    for (int u = 0; u < kVecUnroll; ++u) {
-      const int v = v0 + u * kRowThreads;
-      if (v < nv) {
-        x[u] = __ldcs(s4 + v);
-        p[u] = p4[v];
+      for (int x = 0; x < 4; ++x) {
+        const int j = ct * kBT + 32 * x + static_cast<int>(lane);
+        const int pos = j < a.M ? __ldg(sp + j) : -1;
+        any |= pos >= 0 && pos <= a.pos0 + i_max;
+        all &= pos >= 0 && pos <= a.pos0 + i_min;
+      }
+      any = __any_sync(0xffffffffu, any);
+      all = __all_sync(0xffffffffu, all);
+      if (lane == 0) sm.cls[ct] = any ? (all ? kBClsFull : kBClsPartial) : kBClsSkip;
+    }
+    for (int c = sw; c < n_nt; c += kBwdSoftmaxWarps) {
+      const int c0 = c * kBT;
+      const uint8_t cl = c0 > i_max ? kBClsSkip
+                         : (c0 + kBT - 1 <= i_min && c0 + kBT <= a.S) ? kBClsFull
+                                                                       : kBClsPartial;
+      if (lane == 0) sm.cls[n_ct + c] = cl;
+    }
+  }
+  __syncthreads();
+  if (warp == kBwdFirstSoftmax) build_tile_list(sm, n_ct + n_nt, lane);
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+
+  const uint32_t tmem = sm.taddr;
+  const uint32_t tdQ = tmem;
+  const int n_t = sm.n_tiles;
+  const int n_steps = 2 * n_t;
+  volatile int* abort_flag = &sm.abort_flag;
+
+  if (warp == 0) {
+    // --------------------------------------------------------- TMA producer --
+    if (lane == 0 && n_t > 0) {
+      tma_prefetch_desc(&a.tm_q);
+      tma_prefetch_desc(&a.tm_do);
+      tma_prefetch_desc(&a.tm_kn);
+      tma_prefetch_desc(&a.tm_vn);
+      if (n_ct > 0) {
+        tma_prefetch_desc(&a.tm_kc);
+        tma_prefetch_desc(&a.tm_vc);
+      }
+      bar_expect_tx(&sm.bar_res, 2 * G::kTileBytes);
+      for (int p = 0; p < P; ++p) {
+        tma_load_3d(sm.res[0] + p * kBT * 128, &a.tm_q, &sm.bar_res, 64 * p, r0, grp);
+        tma_load_3d(sm.res[1] + p * kBT * 128, &a.tm_do, &sm.bar_res, 64 * p, r0, grp);
+      }
+      int uses[kBwdStages] = {};
+      for (int t = 0; t < n_t; ++t) {
+        const int s = t % kBwdStages;
+        if (uses[s] > 0 && !bwait(&sm.bar_empty[s], (uses[s] - 1) & 1, abort_flag)) break;
+        const int idx = sm.tiles[t] & kBIdxMask;
+        const bool chunk = idx >= n_ct;
+        const int key0 = (chunk ? idx - n_ct : idx) * kBT;
+        const CUtensorMap* mk = chunk ? &a.tm_kn : &a.tm_kc;
+        const CUtensorMap* mv = chunk ? &a.tm_vn : &a.tm_vc;
+        bar_expect_tx(&sm.bar_full[s], 2 * G::kTileBytes);
+        for (int p = 0; p < P; ++p) {
+          tma_load_3d(sm.ring[s][0] + p * kBT * 128, mk, &sm.bar_full[s], 64 * p, key0, grp);
+          tma_load_3d(sm.ring[s][1] + p * kBT * 128, mv, &sm.bar_full[s], 64 * p, key0, grp);
+        }
+        ++uses[s];
+      }
+      if (*abort_flag) drain_loads(sm, uses, true);
+    }
+  } else if (warp == 1) {
+    // ----------------------------------------------------------- MMA issue --
+    if (lane == 0 && n_t > 0) {
+      constexpr uint32_t kIdS = idesc_bf16_f32(kBT, kDqStep, false);  // S, dP: N = 64 keys
+      constexpr uint32_t kIdQ = idesc_bf16_f32(kBT, 64, true);        // dQ: one 64-column panel
+      uint64_t qd[D / 16], od[D / 16];
+      kmajor_steps<D>(smem_addr(sm.res[0]), qd);
+      kmajor_steps<D>(smem_addr(sm.res[1]), od);
+      // S = Q K^T and dP = dO V^T of step m (keys 64 h .. of tile m / 2)
+      auto issue_sdp = [&](int m) -> bool {
+        const int b = m % kBwdBufs, t = m >> 1, h = m & 1, s = t % kBwdStages;
+        if (m >= kBwdBufs && !bwait(&sm.bar_done[b], (m / kBwdBufs - 1) & 1, abort_flag))
+          return false;
+        if (h == 0 && !bwait(&sm.bar_full[s], (t / kBwdStages) & 1, abort_flag)) return false;
+        tc_fence_after_sync();
+        uint64_t kd[D / 16], vd[D / 16];
+        kmajor_steps<D>(smem_addr(sm.ring[s][0]) + h * kDqStep * 128, kd);
+        kmajor_steps<D>(smem_addr(sm.ring[s][1]) + h * kDqStep * 128, vd);
+        const uint32_t tSb = tmem + 128 + 128 * b;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) mma_ss(tSb, qd[kk], kd[kk], kIdS, kk > 0 ? 1u : 0u);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk)
+          mma_ss(tSb + kDqStep, od[kk], vd[kk], kIdS, kk > 0 ? 1u : 0u);
+        mma_commit(&sm.bar_sfull[b]);
+        return true;
+      };
+      // dQ += dS K_step (A = dS from TMEM, 4 K-steps of 16 keys; B = the
+      // step's 64 key rows, MN-major, one MMA per 64-column panel)
+      auto issue_dq = [&](int n) -> bool {
+        const int b = n % kBwdBufs, t = n >> 1, h = n & 1, s = t % kBwdStages;
+        if (!bwait(&sm.bar_pfull[b], (n / kBwdBufs) & 1, abort_flag)) return false;
+        tc_fence_after_sync();
+        const uint32_t tSb = tmem + 128 + 128 * b;
+        const uint32_t kb = smem_addr(sm.ring[s][0]);
+#pragma unroll
+        for (int p = 0; p < P; ++p)
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            mma_ts(tdQ + 64 * p, tSb + 8 * kk, mn_step(kb, p, 4 * h + kk), kIdQ,
+                   (n > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&sm.bar_done[b]);
+        if (h == 1) mma_commit(&sm.bar_empty[s]);  // both halves of K_t, V_t read
+        return true;
+      };
+      bool ok = bwait(&sm.bar_res, 0, abort_flag) && issue_sdp(0);
+      for (int n = 0; ok && n < n_steps; ++n) {
+        if (n + 1 < n_steps) ok = issue_sdp(n + 1);
+        if (ok) ok = issue_dq(n);
+      }
+      if (ok) mma_commit(&sm.bar_acc);
+      drain_mmas(sm);
+    }
+  } else {
+    // ---------------------------------------------------- dS = P (dP - D) --
+    // Team t (warps 2-5 or 6-9) takes steps n = t, t + 2, ...; each thread
+    // owns one stacked row (the 32x32b layout: lane quarter warp % 4).
+    const int sw = warp - kBwdFirstSoftmax;
+    const int team = sw >> 2;
+    const int q4 = warp & 3;
+    const int row = q4 * 32 + static_cast<int>(lane);
+    const int r = r0 + row;
+    const bool valid = r < R;
+    int g = 0, i = 0;
+    if (valid) split_row(r, a.S, g, i);
+    const size_t ri = static_cast<size_t>(grp) * backward_row_stride(a.qg, a.S) + r;
+    const float nlam = valid ? -__ldg(a.lse + ri) : -INFINITY;
+    const float drow = valid ? __ldg(a.drow + ri) : 0.f;
+    const float sl2 = a.scale_log2;
+    const int qpos = a.pos0 + i;
+    const int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
+    const uint32_t lane_addr = static_cast<uint32_t>(q4 * 32) << 16;
+    bool ok = true;
+    for (int n = team; n < n_steps; n += 2) {
+      const int b = n % kBwdBufs, t = n >> 1, h = n & 1;
+      if (!wwait(&sm.bar_sfull[b], (n / kBwdBufs) & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after_sync();
+      const uint16_t e = sm.tiles[t];
+      const int idx = e & kBIdxMask;
+      const bool partial = (e & kBPartial) != 0;
+      const bool chunk = idx >= n_ct;
+      const int key0 = (chunk ? idx - n_ct : idx) * kBT + h * kDqStep;
+      const uint32_t tSb = tmem + 128 + 128 * b + lane_addr;
+#pragma unroll 1
+      for (int hh = 0; hh < 2; ++hh) {
+        uint32_t sr[32], pr[32];
+        tmem_ld32_async(tSb + 32 * hh, sr);
+        tmem_ld32_async(tSb + kDqStep + 32 * hh, pr);
+        uint32_t vis = 0xffffffffu;  // bit k: key key0 + 32 hh + k visible to this row
+        if (partial) {
+          vis = 0u;
+          const int j0 = key0 + 32 * hh;
+          if (valid) {
+            if (chunk) {
+#pragma unroll
+              for (int k = 0; k < 32; ++k)
+                if (j0 + k <= i && j0 + k < a.S) vis |= 1u << k;
+            } else {
+              for (int k = 0; k < 32; ++k) {
+                const int j = j0 + k;
+                const int pos = j < a.M ? __ldg(sp + j) : -1;
+                if (pos >= 0 && pos <= qpos) vis |= 1u << k;
+              }
+            }
+          }
+        }
+        tmem_wait_ld(sr);
+        tmem_wait_ld(pr);
+        uint32_t ds[16];
+        const float2 sc = make_float2(sl2, sl2), nl = make_float2(nlam, nlam);
+        const float2 nd = make_float2(-drow, -drow);
+#pragma unroll
+        for (int k = 0; k < 32; k += 2) {
+          const float2 x = ffma2(make_float2(__uint_as_float(sr[k]), __uint_as_float(sr[k + 1])), sc, nl);
+          const float2 p = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+          const float2 dp = fadd2(make_float2(__uint_as_float(pr[k]), __uint_as_float(pr[k + 1])), nd);
+          float d0 = p.x * dp.x, d1 = p.y * dp.y;
+          if (partial) {
+            d0 = (vis >> k) & 1u ? d0 : 0.f;
+            d1 = (vis >> (k + 1)) & 1u ? d1 : 0.f;
+          }
+          ds[k / 2] = pack_bf16x2(d0, d1);
+        }
+        // keys 32 hh .. 32 hh + 31 as bf16 pairs over columns 16 hh .. of S
+        // (columns this thread has already loaded)
+        tmem_st16_async(tSb + 16 * hh, ds);
+      }
+      tmem_wait_st();
+      tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) bar_arrive(&sm.bar_pfull[b]);
+    }
+    // ------------------------------------------------------------ epilogue --
+    // dq = scale dQ: team t stores columns t D / 2 .. of its rows
+    if (ok && n_steps > 0) ok = wwait(&sm.bar_acc, 0, abort_flag);
+    if (ok) {
+      tc_fence_after_sync();
+      float* dst = a.dq + (static_cast<size_t>(grp) * R + r) * D + team * (D / 2);
+#pragma unroll 1
+      for (int c = 0; c < D / 2; c += 32) {
+        uint32_t v[32];
+        if (n_steps > 0) {
+          tmem_ld32(tdQ + lane_addr + team * (D / 2) + c, v);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) v[k] = 0u;
+        }
+        if (valid) {
+          float4* d4 = reinterpret_cast<float4*>(dst + c);
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            d4[k] = make_float4(a.scale * __uint_as_float(v[4 * k]), a.scale * __uint_as_float(v[4 * k + 1]),
+                                a.scale * __uint_as_float(v[4 * k + 2]), a.scale * __uint_as_float(v[4 * k + 3]));
+        }
       }
     }
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ----------------------------------------------------------------- dkv ------
+// One CTA per key tile kt of a group (cache tiles, then chunk tiles), K and V
+// resident.  The row tiles of the group's stacked rows stream through the
+// ring with their lambda and D and run as steps of W rows, step n in TMEM
+// buffer n % 3: S^T at columns 2D + 2W b, dP^T W columns after it; the
+// softmax writes bf16 P^T over S^T's first W/2 columns and dS^T over
+// dP^T's, dV (columns 0 ..) accumulates P^T dO and dK (columns D ..) dS^T Q.
+// The issue order is that of the dq kernel.
+template <int D>
+__device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, int kt, int grp) {
+  using G = BwdGeom<D>;
+  constexpr int P = G::kPanels;
+  constexpr int W = G::kW;
+  constexpr int SPT = G::kStepsPerTile;
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const uint32_t lane = tid & 31;
+  const int R = a.qg * a.S;
+  const int Rp = backward_row_stride(a.qg, a.S);
+  const int n_ct = (a.M + kBT - 1) / kBT;
+  const bool chunk = kt >= n_ct;
+  const int key0 = (chunk ? kt - n_ct : kt) * kBT;
+  const int n_keys = min(kBT, (chunk ? a.S : a.M) - key0);
+  const int n_rt = (R + kBT - 1) / kBT;
+  const int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
+  // key j of the tile is seen by chunk row i iff thr(j) <= i (cache slot:
+  // occupied and pos - pos0 <= i; chunk token c: c <= i); keys that do not
+  // exist or are empty never are
+  auto key_thr = [&](int kl) -> int {
+    const int j = key0 + kl;
+    if (chunk) return kl < n_keys ? j : INT_MAX;
+    const int pos = kl < n_keys ? __ldg(sp + j) : -1;
+    return pos >= 0 ? pos - a.pos0 : INT_MAX;
+  };
+
+  if (tid == 0) init_barriers(sm);
+  if (warp == 1) {
+    tmem_alloc(&sm.taddr, 512);
+    tmem_relinquish();
+  }
+  if (warp == kBwdFirstSoftmax) {
+    // row tiles against this key tile: skipped when no row sees a key,
+    // unmasked when every row exists and sees every key
+    int tmin = INT_MAX, tmax = INT_MIN;
 #pragma unroll
-    for (int u = 0; u < kVecUnroll; ++u) {
-      const int v = v0 + u * kRowThreads;
-      if (v >= nv) continue;
-      const float d0 = __uint_as_float(p[u].x << 16) * (x[u].x - dr);
-      const float d1 = __uint_as_float(p[u].x & 0xFFFF0000u) * (x[u].y - dr);
-      const float d2 = __uint_as_float(p[u].y << 16) * (x[u].z - dr);
-      const float d3 = __uint_as_float(p[u].y & 0xFFFF0000u) * (x[u].w - dr);
-      ds4[v] = make_uint2(pack_bf16x2(d0, d1), pack_bf16x2(d2, d3));
+    for (int x = 0; x < 4; ++x) {
+      const int th = key_thr(32 * x + static_cast<int>(lane));
+      tmin = min(tmin, th);
+      tmax = max(tmax, th);
+    }
+    tmin = __reduce_min_sync(0xffffffffu, tmin);
+    tmax = __reduce_max_sync(0xffffffffu, tmax);  // INT_MAX when a key is never seen
+    for (int rt = static_cast<int>(lane); rt < n_rt; rt += 32) {
+      int i_min, i_max;
+      row_tile_range(rt * kBT, R, a.S, i_min, i_max);
+      const bool all_rows = rt * kBT + kBT <= R;
+      sm.cls[rt] = tmin > i_max                              ? kBClsSkip
+                   : (all_rows && tmax != INT_MAX && tmax <= i_min) ? kBClsFull
+                                                              : kBClsPartial;
+    }
+    __syncwarp();
+    build_tile_list(sm, n_rt, lane);
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+
+  const uint32_t tmem = sm.taddr;
+  const uint32_t tdV = tmem, tdK = tmem + D;
+  const int n_t = sm.n_tiles;
+  const int n_steps = n_t * SPT;
+  volatile int* abort_flag = &sm.abort_flag;
+
+  if (warp == 0) {
+    // --------------------------------------------------------- TMA producer --
+    if (lane == 0 && n_t > 0) {
+      const CUtensorMap* mk = chunk ? &a.tm_kn : &a.tm_kc;
+      const CUtensorMap* mv = chunk ? &a.tm_vn : &a.tm_vc;
+      tma_prefetch_desc(mk);
+      tma_prefetch_desc(mv);
+      tma_prefetch_desc(&a.tm_q);
+      tma_prefetch_desc(&a.tm_do);
+      bar_expect_tx(&sm.bar_res, 2 * G::kTileBytes);
+      for (int p = 0; p < P; ++p) {
+        tma_load_3d(sm.res[0] + p * kBT * 128, mk, &sm.bar_res, 64 * p, key0, grp);
+        tma_load_3d(sm.res[1] + p * kBT * 128, mv, &sm.bar_res, 64 * p, key0, grp);
+      }
+      int uses[kBwdStages] = {};
+      for (int t = 0; t < n_t; ++t) {
+        const int s = t % kBwdStages;
+        if (uses[s] > 0 && !bwait(&sm.bar_empty[s], (uses[s] - 1) & 1, abort_flag)) break;
+        const int row0 = (sm.tiles[t] & kBIdxMask) * kBT;
+        const size_t ro = static_cast<size_t>(grp) * Rp + row0;
+        bar_expect_tx(&sm.bar_full[s], 2 * G::kTileBytes + 2 * kBT * 4);
+        for (int p = 0; p < P; ++p) {
+          tma_load_3d(sm.ring[s][0] + p * kBT * 128, &a.tm_q, &sm.bar_full[s], 64 * p, row0, grp);
+          tma_load_3d(sm.ring[s][1] + p * kBT * 128, &a.tm_do, &sm.bar_full[s], 64 * p, row0, grp);
+        }
+        bulk_load_once(sm.rowv[s][0], a.lse + ro, kBT * 4, &sm.bar_full[s]);
+        bulk_load_once(sm.rowv[s][1], a.drow + ro, kBT * 4, &sm.bar_full[s]);
+        ++uses[s];
+      }
+      if (*abort_flag) drain_loads(sm, uses, true);
+    }
+  } else if (warp == 1) {
+    // ----------------------------------------------------------- MMA issue --
+    if (lane == 0 && n_t > 0) {
+      constexpr uint32_t kIdS = idesc_bf16_f32(kBT, W, false);  // S^T, dP^T: N = W rows
+      constexpr uint32_t kIdG = idesc_bf16_f32(kBT, 64, true);  // dV, dK: one 64-column panel
+      uint64_t kd[D / 16], vd[D / 16];
+      kmajor_steps<D>(smem_addr(sm.res[0]), kd);
+      kmajor_steps<D>(smem_addr(sm.res[1]), vd);
+      // S^T = K Q_w^T and dP^T = V dO_w^T of step m (rows W w .. of row tile m / SPT)
+      auto issue_sdp = [&](int m) -> bool {
+        const int b = m % kBwdBufs, t = m / SPT, w = m % SPT, s = t % kBwdStages;
+        if (m >= kBwdBufs && !bwait(&sm.bar_done[b], (m / kBwdBufs - 1) & 1, abort_flag))
+          return false;
+        if (w == 0 && !bwait(&sm.bar_full[s], (t / kBwdStages) & 1, abort_flag)) return false;
+        tc_fence_after_sync();
+        uint64_t qd[D / 16], od[D / 16];
+        kmajor_steps<D>(smem_addr(sm.ring[s][0]) + w * W * 128, qd);
+        kmajor_steps<D>(smem_addr(sm.ring[s][1]) + w * W * 128, od);
+        const uint32_t tSb = tmem + 2 * D + 2 * W * b;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) mma_ss(tSb, kd[kk], qd[kk], kIdS, kk > 0 ? 1u : 0u);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) mma_ss(tSb + W, vd[kk], od[kk], kIdS, kk > 0 ? 1u : 0u);
+        mma_commit(&sm.bar_sfull[b]);
+        return true;
+      };
+      // dV += P^T dO_w, dK += dS^T Q_w (A from TMEM, W / 16 K-steps of 16
+      // rows; B = the step's rows, MN-major, one MMA per 64-column panel)
+      auto issue_kv = [&](int n) -> bool {
+        const int b = n % kBwdBufs, t = n / SPT, w = n % SPT, s = t % kBwdStages;
+        if (!bwait(&sm.bar_pfull[b], (n / kBwdBufs) & 1, abort_flag)) return false;
+        tc_fence_after_sync();
+        const uint32_t tSb = tmem + 2 * D + 2 * W * b;
+        const uint32_t qb = smem_addr(sm.ring[s][0]), ob = smem_addr(sm.ring[s][1]);
+#pragma unroll
+        for (int p = 0; p < P; ++p)
+#pragma unroll
+          for (int kk = 0; kk < W / 16; ++kk)
+            mma_ts(tdV + 64 * p, tSb + 8 * kk, mn_step(ob, p, (W / 16) * w + kk), kIdG,
+                   (n > 0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+        for (int p = 0; p < P; ++p)
+#pragma unroll
+          for (int kk = 0; kk < W / 16; ++kk)
+            mma_ts(tdK + 64 * p, tSb + W + 8 * kk, mn_step(qb, p, (W / 16) * w + kk), kIdG,
+                   (n > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&sm.bar_done[b]);
+        if (w == SPT - 1) mma_commit(&sm.bar_empty[s]);  // the row tile's last step
+        return true;
+      };
+      bool ok = bwait(&sm.bar_res, 0, abort_flag) && issue_sdp(0);
+      for (int n = 0; ok && n < n_steps; ++n) {
+        if (n + 1 < n_steps) ok = issue_sdp(n + 1);
+        if (ok) ok = issue_kv(n);
+      }
+      if (ok) mma_commit(&sm.bar_acc);
+      drain_mmas(sm);
+    }
+  } else {
+    // ------------------------------------ P^T and dS^T = P^T (dP^T - D) --
+    // Team t takes steps n = t, t + 2, ...; each thread owns one key (the
+    // 32x32b layout: lane quarter warp % 4), the columns are stacked rows.
+    const int sw = warp - kBwdFirstSoftmax;
+    const int team = sw >> 2;
+    const int q4 = warp & 3;
+    const int kl = q4 * 32 + static_cast<int>(lane);
+    const int thr = key_thr(kl);
+    const float sl2 = a.scale_log2;
+    const float2 sc = make_float2(sl2, sl2);
+    const uint32_t lane_addr = static_cast<uint32_t>(q4 * 32) << 16;
+    bool ok = true;
+    for (int n = team; n < n_steps; n += 2) {
+      const int b = n % kBwdBufs, t = n / SPT, w = n % SPT, s = t % kBwdStages;
+      // the S^T buffer, and the stage's lambda and D (complete with its tiles)
+      if (!wwait(&sm.bar_sfull[b], (n / kBwdBufs) & 1, abort_flag) ||
+          !wwait(&sm.bar_full[s], (t / kBwdStages) & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after_sync();
+      const uint16_t e = sm.tiles[t];
+      const bool partial = (e & kBPartial) != 0;
+      const int rs0 = (e & kBIdxMask) * kBT + w * W;  // first stacked row of the step
+      const uint32_t tSb = tmem + 2 * D + 2 * W * b + lane_addr;
+#pragma unroll 1
+      for (int hh = 0; hh < W / 32; ++hh) {
+        uint32_t sr[32], pr[32];
+        tmem_ld32_async(tSb + 32 * hh, sr);
+        tmem_ld32_async(tSb + W + 32 * hh, pr);
+        uint32_t vis = 0xffffffffu;  // bit k: row rs0 + 32 hh + k sees this key
+        if (partial) {
+          vis = 0u;
+          const int rr = rs0 + 32 * hh;
+          int i = rr % a.S;
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            if (rr + k < R && thr <= i) vis |= 1u << k;
+            i = i + 1 == a.S ? 0 : i + 1;
+          }
+        }
+        tmem_wait_ld(sr);
+        tmem_wait_ld(pr);
+        const float* lam = sm.rowv[s][0] + w * W + 32 * hh;
+        const float* dr = sm.rowv[s][1] + w * W + 32 * hh;
+        uint32_t pk[16], dk[16];
+#pragma unroll
+        for (int k = 0; k < 32; k += 4) {
+          const float4 l4 = *reinterpret_cast<const float4*>(lam + k);
+          const float4 d4 = *reinterpret_cast<const float4*>(dr + k);
+#pragma unroll
+          for (int x = 0; x < 4; x += 2) {
+            const float l0 = x == 0 ? l4.x : l4.z, l1 = x == 0 ? l4.y : l4.w;
+            const float e0 = x == 0 ? d4.x : d4.z, e1 = x == 0 ? d4.y : d4.w;
+            const float2 z = ffma2(make_float2(__uint_as_float(sr[k + x]), __uint_as_float(sr[k + x + 1])),
+                                   sc, make_float2(-l0, -l1));
+            float p0 = fast_exp2(z.x), p1 = fast_exp2(z.y);
+            const float2 dd = fadd2(make_float2(__uint_as_float(pr[k + x]), __uint_as_float(pr[k + x + 1])),
+                                    make_float2(-e0, -e1));
+            float g0 = p0 * dd.x, g1 = p1 * dd.y;
+            if (partial) {
+              const bool v0 = (vis >> (k + x)) & 1u, v1 = (vis >> (k + x + 1)) & 1u;
+              p0 = v0 ? p0 : 0.f;
+              p1 = v1 ? p1 : 0.f;
+              g0 = v0 ? g0 : 0.f;
+              g1 = v1 ? g1 : 0.f;
+            }
+            pk[(k + x) / 2] = pack_bf16x2(p0, p1);
+            dk[(k + x) / 2] = pack_bf16x2(g0, g1);
+          }
+        }
+        // rows 32 hh .. 32 hh + 31 of the step as bf16 pairs over columns
+        // 16 hh .. of S^T and of dP^T (columns this thread has already loaded)
+        tmem_st16_async(tSb + 16 * hh, pk);
+        tmem_st16_async(tSb + W + 16 * hh, dk);
+      }
+      tmem_wait_st();
+      tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) bar_arrive(&sm.bar_pfull[b]);
+    }
+    // ------------------------------------------------------------ epilogue --
+    // team 0 stores dv = dV, team 1 dk = scale dK, one key row per thread
+    if (ok && n_steps > 0) ok = wwait(&sm.bar_acc, 0, abort_flag);
+    if (ok) {
+      tc_fence_after_sync();
+      float* base = team == 0 ? (chunk ? a.dv_new : a.dv_cache) : (chunk ? a.dk_new : a.dk_cache);
+      const float f = team == 0 ? 1.f : a.scale;
+      const int rows = chunk ? a.S : a.M;
+      float* dst = base + (static_cast<size_t>(grp) * rows + key0 + kl) * D;
+#pragma unroll 1
+      for (int c = 0; c < D; c += 32) {
+        uint32_t v[32];
+        if (n_steps > 0) {
+          tmem_ld32((team == 0 ? tdV : tdK) + lane_addr + c, v);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) v[k] = 0u;
+        }
+        if (kl < n_keys) {
+          float4* d4 = reinterpret_cast<float4*>(dst + c);
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            d4[k] = make_float4(f * __uint_as_float(v[4 * k]), f * __uint_as_float(v[4 * k + 1]),
+                                f * __uint_as_float(v[4 * k + 2]), f * __uint_as_float(v[4 * k + 3]));
+        }
+      }
     }
   }
-}
-
-// ------------------------------------------------------------ cuBLASLt --
-struct LtState {
-  std::once_flag once;
-  cublasStatus_t status = CUBLAS_STATUS_SUCCESS;
-  cublasLtHandle_t handle = nullptr;
-};
-LtState g_lt[64];
-
-int ptr_align(const void* p, size_t stride_bytes) {
-  uintptr_t v = reinterpret_cast<uintptr_t>(p) | static_cast<uintptr_t>(stride_bytes) | 256u;
-  return static_cast<int>(v & (~v + 1));  // lowest set bit, at most 256
-}
-
-// C[m x n] (col-major, ldc, fp32) = alpha op(A) op(B) + beta C, batched over
-// `batch` with the given element strides; A and B bf16, stored col-major.
-cublasStatus_t lt_gemm(cublasLtHandle_t lt, bool ta, bool tb, int m, int n, int k, float alpha,
-                       const uint16_t* A, int lda, int64_t sa, const uint16_t* B, int ldb,
-                       int64_t sb, float beta, float* C, int ldc, int64_t sc, int batch,
-                       void* ws, size_t ws_bytes, cudaStream_t stream) {
-  if (m == 0 || n == 0 || k == 0) return CUBLAS_STATUS_SUCCESS;  // callers never need C = beta C
-  cublasLtMatmulDesc_t op = nullptr;
-  cublasLtMatrixLayout_t la = nullptr, lb = nullptr, lc = nullptr;
-  cublasLtMatmulPreference_t pref = nullptr;
-  cublasStatus_t st = cublasLtMatmulDescCreate(&op, CUBLAS_COMPUTE_32F, CUDA_R_32F);
-  const cublasOperation_t opa = ta ? CUBLAS_OP_T : CUBLAS_OP_N;
-  const cublasOperation_t opb = tb ? CUBLAS_OP_T : CUBLAS_OP_N;
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof(opa));
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof(opb));
-  // stored shapes: A is (ta ? k x m : m x k), B is (tb ? n x k : k x n)
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatrixLayoutCreate(&la, CUDA_R_16BF, ta ? k : m, ta ? m : k, lda);
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatrixLayoutCreate(&lb, CUDA_R_16BF, tb ? n : k, tb ? k : n, ldb);
-  if (st == CUBLAS_STATUS_SUCCESS) st = cublasLtMatrixLayoutCreate(&lc, CUDA_R_32F, m, n, ldc);
-  const int32_t nb = batch;
-  for (auto [l, s] : {std::pair<cublasLtMatrixLayout_t, int64_t>{la, sa}, {lb, sb}, {lc, sc}}) {
-    if (st != CUBLAS_STATUS_SUCCESS) break;
-    st = cublasLtMatrixLayoutSetAttribute(l, CUBLASLT_MATRIX_LAYOUT_BATCH_COUNT, &nb, sizeof(nb));
-    if (st == CUBLAS_STATUS_SUCCESS)
-      st = cublasLtMatrixLayoutSetAttribute(l, CUBLASLT_MATRIX_LAYOUT_STRIDED_BATCH_OFFSET, &s,
-                                            sizeof(s));
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, 512);
   }
-  if (st == CUBLAS_STATUS_SUCCESS) st = cublasLtMatmulPreferenceCreate(&pref);
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES,
-                                              &ws_bytes, sizeof(ws_bytes));
-  // the real alignment of every operand (base and batch stride), so that no
-  // algorithm needing more is chosen
-  const uint32_t al_a = static_cast<uint32_t>(ptr_align(A, sa * 2));
-  const uint32_t al_b = static_cast<uint32_t>(ptr_align(B, sb * 2));
-  const uint32_t al_c = static_cast<uint32_t>(ptr_align(C, sc * 4));
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_A_BYTES,
-                                              &al_a, sizeof(al_a));
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_B_BYTES,
-                                              &al_b, sizeof(al_b));
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_C_BYTES,
-                                              &al_c, sizeof(al_c));
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_D_BYTES,
-                                              &al_c, sizeof(al_c));
-  cublasLtMatmulHeuristicResult_t heur = {};
-  int found = 0;
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmulAlgoGetHeuristic(lt, op, la, lb, lc, lc, pref, 1, &heur, &found);
-  if (st == CUBLAS_STATUS_SUCCESS && found == 0) st = CUBLAS_STATUS_NOT_SUPPORTED;
-  if (st == CUBLAS_STATUS_SUCCESS)
-    st = cublasLtMatmul(lt, op, &alpha, A, la, B, lb, &beta, C, lc, C, lc, &heur.algo, ws,
-                        ws_bytes, stream);
-  if (pref) cublasLtMatmulPreferenceDestroy(pref);
-  if (lc) cublasLtMatrixLayoutDestroy(lc);
-  if (lb) cublasLtMatrixLayoutDestroy(lb);
-  if (la) cublasLtMatrixLayoutDestroy(la);
-  if (op) cublasLtMatmulDescDestroy(op);
-  return st;
 }
 
-size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+// One launch for both halves of the gradient: blockIdx.x < n_row_tiles is a
+// dq CTA (row tile blockIdx.x), the rest are dkv CTAs (key tile blockIdx.x -
+// n_row_tiles), so that the two kinds fill the SMs together.
+template <int D>
+__global__ void __launch_bounds__(kBwdThreads, 1) bwd_kernel(const __grid_constant__ BackwardArgs a,
+                                                            int n_row_tiles) {
+  extern __shared__ uint8_t smem_raw[];
+  auto& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw +
+                                            ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
+  const int x = static_cast<int>(blockIdx.x);
+  const int grp = static_cast<int>(blockIdx.y);
+  if (x < n_row_tiles) bwd_dq<D>(a, sm, x, grp);
+  else bwd_dkv<D>(a, sm, x - n_row_tiles, grp);
+  if (threadIdx.x == 0 && sm.abort_flag) atomicOr(a.err, H2O_DEVERR_TIMEOUT);
+}
+
+template <int D>
+cudaError_t launch_backward_d(const BackwardArgs& a, cudaStream_t stream) {
+  const int R = a.qg * a.S;
+  const int rows = a.B * a.Hq * a.S;
+  bwd_drow_kernel<D><<<(rows + 7) / 8, 256, 0, stream>>>(a.out, a.dout, a.drow, rows, R,
+                                                          backward_row_stride(a.qg, a.S));
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const size_t smem = sizeof(BwdSmem<D>) + 1024;
+  static OncePerDevice configured;
+  e = configured.run([smem](int) {
+    return cudaFuncSetAttribute(bwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(smem));
+  });
+  if (e != cudaSuccess) return e;
+  const int n_row_tiles = (R + kBT - 1) / kBT;
+  const int n_key_tiles = (a.M + kBT - 1) / kBT + (a.S + kBT - 1) / kBT;
+  const dim3 grid(static_cast<unsigned>(n_row_tiles + n_key_tiles),
+                  static_cast<unsigned>(a.B * a.Hkv));
+  bwd_kernel<D><<<grid, kBwdThreads, smem, stream>>>(a, n_row_tiles);
+  return cudaGetLastError();
+}
 
 }  // namespace
 
 size_t backward_workspace_bytes(int B, int Hq, int Hkv, int S, int M) {
-  const size_t G = static_cast<size_t>(B) * Hkv, R = static_cast<size_t>(Hq / Hkv) * S;
-  const size_t cells = G * R * (static_cast<size_t>(M) + S);
-  return kLtWorkspace + align256(cells * 4) + 2 * align256(cells * 2) + align256(G * R * 4);
+  (void)M;
+  const int qg = Hkv > 0 ? Hq / Hkv : 0;
+  // lambda and D per stacked row, each group's rows padded to 128
+  return 2 * static_cast<size_t>(B) * Hkv * backward_row_stride(qg, S) * sizeof(float);
 }
 
-BackwardStatus launch_backward(BackwardArgs a, void* workspace, cudaStream_t stream) {
-  BackwardStatus out;
-  int dev = 0;
-  cudaError_t ce = cudaGetDevice(&dev);
-  if (ce != cudaSuccess) { out.cuda = ce; return out; }
-  if (dev >= 64) { out.blas = CUBLAS_STATUS_NOT_SUPPORTED; return out; }
-  LtState& ls = g_lt[dev];
-  std::call_once(ls.once, [&ls] { ls.status = cublasLtCreate(&ls.handle); });
-  if (ls.status != CUBLAS_STATUS_SUCCESS) { out.blas = ls.status; return out; }
-  const int G = a.B * a.Hkv, R = a.qg * a.S, NK = a.M + a.S, M = a.M, S = a.S, d = a.d;
-  const size_t cells = static_cast<size_t>(G) * R * NK;
-  uint8_t* w = static_cast<uint8_t*>(workspace);
-  void* lt_ws = w;
-  w += kLtWorkspace;
-  a.sbuf = reinterpret_cast<float*>(w);
-  w += align256(cells * 4);
-  a.pbuf = reinterpret_cast<uint16_t*>(w);
-  w += align256(cells * 2);
-  a.dsbuf = reinterpret_cast<uint16_t*>(w);
-  w += align256(cells * 2);
-  a.drow = reinterpret_cast<float*>(w);
-
-  const int64_t sQ = static_cast<int64_t>(R) * d, sKc = static_cast<int64_t>(M) * d,
-                sKn = static_cast<int64_t>(S) * d, sS = static_cast<int64_t>(R) * NK;
-  cublasLtHandle_t lt = ls.handle;
-  cublasStatus_t st = CUBLAS_STATUS_SUCCESS;
-  auto gemm = [&](bool ta, bool tb, int m, int n, int k, float alpha, const uint16_t* A, int lda,
-                  int64_t sa, const uint16_t* B, int ldb, int64_t sb, float beta, float* C,
-                  int ldc, int64_t sc) {
-    if (st == CUBLAS_STATUS_SUCCESS)
-      st = lt_gemm(lt, ta, tb, m, n, k, alpha, A, lda, sa, B, ldb, sb, beta, C, ldc, sc, G, lt_ws,
-                   kLtWorkspace, stream);
-  };
-  // S = Q K^T: per group, col-major C (N_k x R): cache block rows 0..M-1, chunk block M..
-  gemm(true, false, M, R, d, 1.f, a.k_cache, d, sKc, a.q, d, sQ, 0.f, a.sbuf, NK, sS);
-  gemm(true, false, S, R, d, 1.f, a.k_new, d, sKn, a.q, d, sQ, 0.f, a.sbuf + M, NK, sS);
-  if (st != CUBLAS_STATUS_SUCCESS) { out.blas = st; return out; }
-  // the vectorised passes need float4 rows (N_k, M multiples of 4) and 16-byte
-  // aligned workspace and slot positions; every other shape takes the scalar ones
-  const bool vec = NK % 4 == 0 && M % 4 == 0 && d <= kVecThreads &&
-                   (reinterpret_cast<uintptr_t>(workspace) & 15u) == 0 &&
-                   (reinterpret_cast<uintptr_t>(a.slot_pos) & 15u) == 0;
-  const unsigned rows = static_cast<unsigned>(static_cast<size_t>(G) * R);
-  if (vec && NK / 4 <= kVecUnroll * kVecThreads)
-    bwd_softmax_vec_kernel<true><<<rows, kVecThreads, 0, stream>>>(a);
-  else if (vec)
-    bwd_softmax_vec_kernel<false><<<rows, kVecThreads, 0, stream>>>(a);
-  else
-    bwd_softmax_kernel<<<rows, kRowThreads, 0, stream>>>(a);
-  if ((ce = cudaGetLastError()) != cudaSuccess) { out.cuda = ce; return out; }
-  // dP = dout V^T into the same buffer
-  gemm(true, false, M, R, d, 1.f, a.v_cache, d, sKc, a.dout, d, sQ, 0.f, a.sbuf, NK, sS);
-  gemm(true, false, S, R, d, 1.f, a.v_new, d, sKn, a.dout, d, sQ, 0.f, a.sbuf + M, NK, sS);
-  if (st != CUBLAS_STATUS_SUCCESS) { out.blas = st; return out; }
-  if (vec) {
-    bwd_ds_vec_kernel<<<rows, kRowThreads, 0, stream>>>(a);
-  } else {
-    const size_t blocks = std::min<size_t>(static_cast<size_t>(G) * R, 152 * 8);
-    bwd_ds_kernel<<<static_cast<unsigned>(blocks), kRowThreads, 0, stream>>>(a);
-  }
-  if ((ce = cudaGetLastError()) != cudaSuccess) { out.cuda = ce; return out; }
-  // dQ^T (d x R) = K^T dS^T: cache block, then += chunk block
-  gemm(false, false, d, R, M, a.scale, a.k_cache, d, sKc, a.dsbuf, NK, sS, 0.f, a.dq, d, sQ);
-  gemm(false, false, d, R, S, a.scale, a.k_new, d, sKn, a.dsbuf + M, NK, sS, M > 0 ? 1.f : 0.f,
-       a.dq, d, sQ);
-  // dK^T (d x M) = Q^T dS (R x M); dV^T = dout^T P
-  gemm(false, true, d, M, R, a.scale, a.q, d, sQ, a.dsbuf, NK, sS, 0.f, a.dk_cache, d, sKc);
-  gemm(false, true, d, S, R, a.scale, a.q, d, sQ, a.dsbuf + M, NK, sS, 0.f, a.dk_new, d, sKn);
-  gemm(false, true, d, M, R, 1.f, a.dout, d, sQ, a.pbuf, NK, sS, 0.f, a.dv_cache, d, sKc);
-  gemm(false, true, d, S, R, 1.f, a.dout, d, sQ, a.pbuf + M, NK, sS, 0.f, a.dv_new, d, sKn);
-  out.blas = st;
-  return out;
+cudaError_t launch_backward(const BackwardArgs& a, cudaStream_t stream) {
+  return a.d == 64 ? launch_backward_d<64>(a, stream) : launch_backward_d<128>(a, stream);
 }
 
 }  // namespace h2o

@@ -63,6 +63,12 @@ struct SdpaArgs {
   // finish in; otherwise it adds into the zeroed score_inc directly (at most
   // two addends per element onto an exact zero, which commute).
   float* colpart;
+  // Non-null: pass 1 only.  The kernel writes every query row's log-sum-exp
+  // of the scaled logits in log2 units, lse[(b Hkv + h) lse_stride + g S + i]
+  // for query head h q_g + g, and nothing else (the backward's softmax
+  // recomputation needs it).
+  float* lse;
+  int lse_stride;
 };
 
 // Row tiles per query head above which the column sums go through colpart.
@@ -194,8 +200,15 @@ cudaError_t launch_kv_dequantize(const int8_t* codes, const float* scales, uint1
                                  int64_t n_rows, int d, cudaStream_t stream);
 cudaError_t launch_kv_scatter_q8(const Q8ScatterArgs& a, cudaStream_t stream);
 
-// h2o_sdpa_chunk_backward (h2o_backward.cu)
+// h2o_sdpa_chunk_backward (h2o_backward.cu): fused tcgen05 kernels, no
+// materialised score matrices.  The workspace holds, per stacked query row of
+// each (b, kv head) group, the row's log-sum-exp (log2 units, from the
+// forward kernel's pass 1) and D = dout . out.
 struct BackwardArgs {
+  // TMA maps (box {64, 128, 1}, 128-byte swizzle): the stacked query rows of
+  // a group {d, q_g S, B Hkv} for q and dout, the keys and values {d, M or S,
+  // B Hkv} of the cache and of the chunk
+  CUtensorMap tm_q, tm_do, tm_kc, tm_vc, tm_kn, tm_vn;
   const uint16_t* q;         // (B, Hq, S, d) bf16
   const uint16_t* k_cache;   // (B, Hkv, M, d)
   const uint16_t* v_cache;
@@ -209,21 +222,21 @@ struct BackwardArgs {
   float* dv_cache;
   float* dk_new;             // (B, Hkv, S, d) fp32
   float* dv_new;
-  float* sbuf;               // workspace: S, then dP (groups x R x (M + S)) fp32
-  uint16_t* pbuf;            // P, bf16
-  uint16_t* dsbuf;           // dS, bf16
-  float* drow;               // D per stacked row
+  float* lse;                // (B Hkv, R_pad): per stacked row g S + i of a group, its
+                             // log-sum-exp (log2 units); R_pad = q_g S rounded up to 128
+  float* drow;               // (B Hkv, R_pad): D per stacked row
+  int* err;
   int B, Hq, Hkv, d, S, M, qg;
   int pos0;
   float scale;               // softmax scale
   float scale_log2;          // scale * log2(e)
 };
-struct BackwardStatus {
-  cudaError_t cuda = cudaSuccess;
-  int blas = 0;              // cublasStatus_t, 0 = success
-};
+// Rows of a group in the lse / drow layout: q_g S rounded up to 128, so that
+// every 128-row tile of them starts 16-byte aligned.
+__host__ __device__ inline int backward_row_stride(int qg, int S) { return (qg * S + 127) / 128 * 128; }
 size_t backward_workspace_bytes(int B, int Hq, int Hkv, int S, int M);
-BackwardStatus launch_backward(BackwardArgs a, void* workspace, cudaStream_t stream);
+// The forward's pass 1 must have filled a.lse first.
+cudaError_t launch_backward(const BackwardArgs& a, cudaStream_t stream);
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);

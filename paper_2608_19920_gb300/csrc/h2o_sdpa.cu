@@ -383,11 +383,12 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       // with V_{t-2} (ring B), then the last V's
       bool ok = true;
       for (int t = 0; ok && t < n_t; ++t) ok = load(t % R, false, t);
-      for (int t = 0; ok && t < n_t; ++t) {
+      const int n_t2 = a.lse != nullptr ? 0 : n_t;  // pass 2's tiles
+      for (int t = 0; ok && t < n_t2; ++t) {
         ok = load(t % RA, false, t);
         if (ok && t >= 2) ok = load(RA + (t - 2) % RB, true, t - 2);
       }
-      for (int t = max(0, n_t - 2); ok && t < n_t; ++t) ok = load(RA + t % RB, true, t);
+      for (int t = max(0, n_t2 - 2); ok && t < n_t2; ++t) ok = load(RA + t % RB, true, t);
       if (*abort_flag) {
         // Let copies still in flight land before the CTA's shared memory goes
         // away: at most the latest load of each slot can be outstanding.  On a
@@ -474,13 +475,13 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         // pass 2 reuses slots that warp 2 took in pass 1: start once it has
         // waited for all of its pass-1 tiles, so that no full-barrier wait
         // here runs two phases ahead
-        if (ok) ok = wait_b<kPair>(&sm.bar_p1done, 0, abort_flag);
-        for (int n = n_t; ok && n < 2 * n_t; ++n) ok = issue_qk(n);
+        if (ok && a.lse == nullptr) ok = wait_b<kPair>(&sm.bar_p1done, 0, abort_flag);
+        for (int n = n_t; ok && a.lse == nullptr && n < 2 * n_t; ++n) ok = issue_qk(n);
       } else {
         for (int n = 1; ok && n < n_t; n += 2) ok = issue_qk(n);
         bar_arrive(&sm.bar_p1done);
         const uint64_t v_desc0 = sdesc_sw128(smem_addr(sm.kv[RA]), kTileN * 128, 1024);
-        for (int t = 0; ok && t < n_t; ++t) {
+        for (int t = 0; ok && a.lse == nullptr && t < n_t; ++t) {
           const int pb = t % kSBufs2;  // the S buffer of pass-2 tile t holds its P
           if (!wait_b<kPair>(&sm.bar_pfull[pb], (t / kSBufs2) & 1, abort_flag)) {
             ok = false;
@@ -503,7 +504,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           commit_all<kPair>(&sm.bar_empty[vs]);
           commit_all<kPair>(&sm.bar_pvdone[pb]);
         }
-        if (ok) commit_all<kPair>(&sm.bar_ofull);
+        if (ok && a.lse == nullptr) commit_all<kPair>(&sm.bar_ofull);
       }
       // No MMA of this thread may still be running when TMEM is freed.
       uint64_t* drain = &sm.bar_drain[is_qk ? 0 : 1];
@@ -593,7 +594,8 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     bool ok = true;
     bool have_lambda = false;
     int k2 = 0;  // pass-2 tiles this warp has processed (column-sum buffer phase)
-    for (int n = team; ok && n < 2 * n_t; n += 2) {
+    const int n_end = a.lse != nullptr ? n_t : 2 * n_t;  // pass 1 only when lse is asked
+    for (int n = team; ok && n < n_end; n += 2) {
       int buf, suse;
       s_buffer(n, n_t, buf, suse);
       const bool pass2 = n >= n_t;
@@ -863,8 +865,26 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       __syncwarp();
       if (lane == 0) bar_arrive(&sm.bar_rowstat);
     }
+    if (a.lse != nullptr && ok && n_t > 0 && wait_bar(&sm.bar_rowstat, 0, abort_flag, kWaitLimitNs)) {
+      // pass 1 only: the merged log-sum-exp of each row (§A.6.1), one lane
+      // of the four holding a row in the 16x256b layout writes it
+#pragma unroll
+      for (int x = 0; x < 4; ++x) {
+        const int r = q4 * 32 + static_cast<int>(lane >> 2) + 8 * x;
+        int gg, ii;
+        if ((lane & 3u) != 0u || !row_info(r, gg, ii)) continue;
+        float mm = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kNumWG; ++w) mm = fmaxf(mm, sm.rowstat[w][r][0]);
+        float l = 0.f;
+#pragma unroll
+        for (int w = 0; w < kNumWG; ++w)
+          l += sm.rowstat[w][r][1] * fast_exp2(sm.rowstat[w][r][0] - mm);
+        a.lse[static_cast<size_t>(grp) * a.lse_stride + gg * a.S + ii] = mm + fast_log2(l);
+      }
+    }
     // ------------------------------------------------------------ epilogue --
-    if (ok && n_t > 0 && wait_b<kPair>(&sm.bar_ofull, 0, abort_flag)) {
+    if (ok && n_t > 0 && a.lse == nullptr && wait_b<kPair>(&sm.bar_ofull, 0, abort_flag)) {
       tc_fence_after_sync();
       constexpr int kPart = D / kNumWG;  // O columns per warpgroup: 32 or 16
       uint32_t pk[kPart / 2];

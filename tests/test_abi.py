@@ -206,10 +206,9 @@ def test_backward_argument_checks(lib):
     d = _dims()
     n = ctypes.c_size_t(0)
     assert lib.h2o_backward_workspace_size(ctypes.byref(d), ctypes.byref(n)) == OK
-    G, R, NK = 2, 2 * 32, 256 + 32
-    cells = G * R * NK
-    a256 = lambda x: (x + 255) // 256 * 256
-    assert n.value == (32 << 20) + a256(cells * 4) + 2 * a256(cells * 2) + a256(G * R * 4)
+    # lambda and D per stacked row: B Hkv = 2 groups of q_g S = 64 rows, each
+    # padded to 128
+    assert n.value == 2 * 2 * 128 * 4
     bwd = lambda dims, ptrs, ws=p, wsb=n.value, pos0=256: lib.h2o_sdpa_chunk_backward(
         ctypes.byref(dims), pos0, 0.0, *ptrs, ws, wsb, None)
     ok = [p] * 13
@@ -219,6 +218,8 @@ def test_backward_argument_checks(lib):
     assert bwd(d, ok[:8] + [vp(0x1004)] + ok[9:]) == ALIGN
     assert bwd(d, ok, pos0=-1) == ARG
     assert bwd(_dims(d=96), ok) == UNSUP
+    # q_g S = 600000 stacked rows: more than 4096 row tiles in a group
+    assert bwd(_dims(S=300000), ok, pos0=0) == UNSUP
 
 
 def test_selftest_limit_is_checked_on_the_host(lib):

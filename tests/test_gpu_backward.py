@@ -4,7 +4,11 @@ float64 oracle, through the C ABI.
 Tolerance (derived from the arithmetic): the kernel rounds P and dS to bf16
 (relative 2^-9 each) before the fp32-accumulated contractions, and uses the
 bf16 forward output in D = dout . out; each gradient tensor must lie within
-1e-2 of its own max-abs value elementwise.  Slots no row sees get exactly 0."""
+1e-2 of its own max-abs value elementwise.  Slots no row sees get exactly 0.
+
+The cases cover both head sizes, 128-row tiles that hold the rows of two
+query heads (q_g S not a multiple of 128), ragged key tiles, empty and
+future slots, a one-token chunk, no cache, and the Llama-3-8B-shaped chunk."""
 import numpy as np
 import pytest
 import torch
@@ -37,6 +41,9 @@ CASES = [
     (1, 2, 1, 64, 8, 4100, 20, 3, 4200),     # N_k > 4096: the softmax pass reads each row twice
     (1, 4, 4, 128, 200, 0, 0, 0, 0),         # no cache (a prefill)
     (1, 32, 8, 128, 512, 4096, 0, 0, 8192),  # the Llama-3-8B-shaped chunk
+    (2, 8, 2, 128, 300, 700, 11, 20, 3000),  # row tiles across head boundaries, masked tiles
+    (1, 4, 1, 64, 520, 130, 0, 40, 600),     # d = 64, several chunk tiles
+    (1, 6, 2, 128, 45, 260, 9, 7, 400),      # q_g S = 135: a second row tile of 7 rows
 ]
 
 
@@ -73,3 +80,21 @@ def test_backward_matches_oracle(dev, case):
         hidden = (st["slot_pos"] < 0) | (st["slot_pos"] > pos0 + S - 1)
         assert (grads[1].cpu().numpy()[hidden] == 0).all()
         assert (grads[2].cpu().numpy()[hidden] == 0).all()
+
+
+def test_backward_is_deterministic(dev):
+    """No atomics: two calls on the same inputs give bit-identical gradients."""
+    B, Hq, Hkv, d, S, M, pos0 = 1, 32, 8, 128, 512, 4096, 8192
+    rng = np.random.default_rng(5)
+    st = wl.random_state(rng, B, Hkv, M, d, pos0=pos0, n_empty=0)
+    mk = lambda shape: bf(wl.round_bf16(rng.standard_normal(shape, dtype=np.float32)), dev)
+    q, kn, vn, dout = mk((B, Hq, S, d)), mk((B, Hkv, S, d)), mk((B, Hkv, S, d)), mk((B, Hq, S, d))
+    kc, vc = bf(st["k_cache"], dev), bf(st["v_cache"], dev)
+    sp = torch.from_numpy(st["slot_pos"]).to(dev)
+    out, _ = h2o_sdpa_chunk(q, kc, vc, kn, vn, sp, pos0)
+    g1 = h2o_sdpa_chunk_backward(q, kc, vc, kn, vn, sp, pos0, out, dout)
+    g2 = h2o_sdpa_chunk_backward(q, kc, vc, kn, vn, sp, pos0, out, dout)
+    torch.cuda.synchronize()
+    assert h2o_device_errors() == 0
+    for a, b in zip(g1, g2):
+        assert torch.equal(a, b)

@@ -25,9 +25,9 @@
 //    shared memory).
 // Row and key tiles that no (row, key) pair of which is visible are skipped;
 // tiles every pair of which is visible take no mask.  Products whose B
-// operand is a row or key tile read along d (N = d) run as one MMA per
-// 64-column panel.  Every wait is bounded; on expiry a CTA drains its MMAs,
-// frees TMEM and reports H2O_DEVERR_TIMEOUT.
+// operand is a row or key tile read along d (N = d) read it MN-major, the
+// two 64-column panels of d = 128 one LBO apart.  Every wait is bounded;
+// on expiry a CTA drains its MMAs, frees TMEM and reports H2O_DEVERR_TIMEOUT.
 #include <climits>
 #include <cmath>
 
@@ -39,10 +39,10 @@ namespace {
 
 constexpr int kBT = 128;               // rows or keys per tile
 constexpr int kBwdSoftmaxWarps = 8;    // two teams of four warps (one per TMEM lane quarter)
-constexpr int kBwdFirstSoftmax = 2;    // warp 0 TMA, warp 1 MMA issue
-constexpr int kBwdThreads = 32 * (kBwdFirstSoftmax + kBwdSoftmaxWarps);  // 320
+constexpr int kBwdFirstSoftmax = 3;    // warp 0 TMA, warps 1 and 2 MMA issue
+constexpr int kBwdThreads = 32 * (kBwdFirstSoftmax + kBwdSoftmaxWarps);  // 352
 constexpr int kBwdStages = 2;          // shared-memory ring of streamed tile pairs
-constexpr int kBwdBufs = 3;            // S / dP buffer pairs in TMEM
+constexpr int kBwdBufs = 3;            // at most three S / dP buffer pairs in TMEM
 constexpr uint8_t kBClsSkip = 0, kBClsFull = 1, kBClsPartial = 2;
 constexpr uint16_t kBPartial = 0x8000;  // tile-list entry: masked tile
 constexpr uint16_t kBIdxMask = 0x7FFF;
@@ -52,10 +52,13 @@ template <int D>
 struct BwdGeom {
   static constexpr int kPanels = D / 64;
   static constexpr int kTileBytes = kPanels * kBT * 128;  // 128 rows of D bf16
-  // dkv: stacked rows per step.  TMEM holds dV and dK (D columns each) and
-  // three buffers of S^T and dP^T (W columns each): 2D + 6W <= 512.
-  static constexpr int kW = D == 128 ? 32 : 64;
+  // dkv: stacked rows per step (the N of S^T and dP^T: an MMA costs at
+  // least ~45 cycles, so N = 32 would run the tensor pipe at a third of its
+  // rate) and S^T / dP^T buffers; TMEM holds dV and dK (D columns each)
+  // and the buffers (2 W columns each): 2D + 2W bufs <= 512.
+  static constexpr int kW = 64;
   static constexpr int kStepsPerTile = kBT / kW;
+  static constexpr int kDkvBufs = D == 128 ? 2 : 3;
 };
 
 // Shared memory of both kernels: two resident tiles (dq: Q and dO; dkv: K and
@@ -68,7 +71,7 @@ struct __align__(1024) BwdSmem {
   float rowv[kBwdStages][2][kBT];  // dkv: lambda and D of the stage's rows
   uint64_t bar_res, bar_full[kBwdStages], bar_empty[kBwdStages];
   uint64_t bar_sfull[kBwdBufs], bar_pfull[kBwdBufs], bar_done[kBwdBufs];
-  uint64_t bar_acc, bar_drain;
+  uint64_t bar_acc, bar_drain[2];
   uint32_t taddr;
   int abort_flag;
   int n_tiles;
@@ -128,12 +131,6 @@ __device__ __forceinline__ void kmajor_steps(uint32_t base, uint64_t (&d)[D / 16
     d[kk] = d0 + static_cast<uint64_t>((kBT * 128 >> 4) * (kk / 4) + 2 * (kk % 4));
 }
 
-// MN-major descriptor of panel p of a 128-row tile read with K = rows and
-// N = the panel's 64 columns; K-step kk covers rows 16 kk .. 16 kk + 15.
-__device__ __forceinline__ uint64_t mn_step(uint32_t base, int p, int kk) {
-  return sdesc_sw128(base + p * kBT * 128, kBT * 128, 1024) + static_cast<uint64_t>(128 * kk);
-}
-
 // Warp-uniform bounded wait: every lane waits, and the warp goes on only if
 // all of them saw the phase complete (so that the .sync.aligned TMEM
 // instructions after it are reached by the whole warp or by none of it).
@@ -174,8 +171,9 @@ __device__ __forceinline__ void build_tile_list(BwdSmem<D>& sm, int total, uint3
   if (lane == 0) sm.n_tiles = n;
 }
 
+// pfull_count: softmax warps that arrive per step.
 template <int D>
-__device__ __forceinline__ void init_barriers(BwdSmem<D>& sm) {
+__device__ __forceinline__ void init_barriers(BwdSmem<D>& sm, int pfull_count) {
   bar_init(&sm.bar_res, 1);
   for (int s = 0; s < kBwdStages; ++s) {
     bar_init(&sm.bar_full[s], 1);
@@ -183,11 +181,12 @@ __device__ __forceinline__ void init_barriers(BwdSmem<D>& sm) {
   }
   for (int b = 0; b < kBwdBufs; ++b) {
     bar_init(&sm.bar_sfull[b], 1);
-    bar_init(&sm.bar_pfull[b], kBwdSoftmaxWarps / 2);  // the four warps of one team
+    bar_init(&sm.bar_pfull[b], pfull_count);
     bar_init(&sm.bar_done[b], 1);
   }
   bar_init(&sm.bar_acc, 1);
-  bar_init(&sm.bar_drain, 1);
+  bar_init(&sm.bar_drain[0], 1);
+  bar_init(&sm.bar_drain[1], 1);
   sm.abort_flag = 0;
   fence_bar_init();
 }
@@ -202,12 +201,13 @@ __device__ void drain_loads(BwdSmem<D>& sm, const int (&uses)[kBwdStages], bool 
     if (uses[s] > 0) wait_bar(&sm.bar_full[s], (uses[s] - 1) & 1, &never, 100000000ull);
 }
 
-// Issuer epilogue: no MMA may still be running when TMEM is freed.
+// Issuer epilogue: no MMA of this issuing thread may still be running when
+// TMEM is freed.
 template <int D>
-__device__ __forceinline__ void drain_mmas(BwdSmem<D>& sm) {
-  mma_commit(&sm.bar_drain);
+__device__ __forceinline__ void drain_mmas(BwdSmem<D>& sm, int issuer) {
+  mma_commit(&sm.bar_drain[issuer]);
   volatile int never = 0;
-  wait_bar(&sm.bar_drain, 0, &never, kWaitLimitNs);
+  wait_bar(&sm.bar_drain[issuer], 0, &never, kWaitLimitNs);
 }
 
 // ------------------------------------------------------------------ dq ------
@@ -215,10 +215,11 @@ __device__ __forceinline__ void drain_mmas(BwdSmem<D>& sm) {
 // tiles (cache tiles, then chunk tiles) run as steps of 64 keys, step n in
 // TMEM buffer n % 3: S at columns 128 + 128 b, dP 64 columns after it; the
 // softmax writes bf16 dS over S's first 32 columns, dQ (D columns from 0)
-// accumulates dS K.  The issuer puts step n+1's S and dP ahead of step n's
-// dQ, so the tensor pipe has work while the softmax runs; a buffer is
-// refilled only after the dQ that read it has completed (MMAs into
-// different accumulators are not ordered by issue).
+// accumulates dS K.  One thread issues S and dP up to three steps ahead,
+// another the dQ of each step once its dS is in, so the tensor pipe has
+// work while the softmax runs; a buffer is refilled only after the dQ that
+// read it has completed (MMAs into different accumulators are not ordered
+// by issue).
 template <int D>
 __device__ __forceinline__ void bwd_dq(const BackwardArgs& a, BwdSmem<D>& sm, int rt, int grp) {
   using G = BwdGeom<D>;
@@ -233,7 +234,7 @@ __device__ __forceinline__ void bwd_dq(const BackwardArgs& a, BwdSmem<D>& sm, in
   int i_min, i_max;
   row_tile_range(r0, R, a.S, i_min, i_max);
 
-  if (tid == 0) init_barriers(sm);
+  if (tid == 0) init_barriers(sm, kBwdSoftmaxWarps / 2);  // one team per step
   if (warp == 1) {
     tmem_alloc(&sm.taddr, 512);
     tmem_relinquish();
@@ -311,14 +312,29 @@ __device__ __forceinline__ void bwd_dq(const BackwardArgs& a, BwdSmem<D>& sm, in
       }
       if (*abort_flag) drain_loads(sm, uses, true);
     }
-  } else if (warp == 1) {
+  } else if (warp == 1 || warp == 2) {
     // ----------------------------------------------------------- MMA issue --
+    // Warp 1 issues S and dP of every step, warp 2 every dQ: while one
+    // issuing thread waits on a barrier the other keeps the tensor pipe fed
+    // (an issuing thread runs only about one MMA ahead of the pipe).
     if (lane == 0 && n_t > 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBT, kDqStep, false);  // S, dP: N = 64 keys
-      constexpr uint32_t kIdQ = idesc_bf16_f32(kBT, 64, true);        // dQ: one 64-column panel
-      uint64_t qd[D / 16], od[D / 16];
+      constexpr uint32_t kIdQ = idesc_bf16_f32(kBT, D, true);         // dQ: N = D
+      // Descriptors: only the 14-bit start address (bytes >> 4) moves: a
+      // ring stage is 2 kTileBytes, half h of a key tile starts 64 rows
+      // (8 KB) in, a K-step of 16 bf16 is 32 B of a 128-B swizzle row, a
+      // 64-column panel is 16 KB; for the MN-major K in dQ a K-step is 16
+      // key rows (2 KB) and the panels are LBO apart.  Everything but the
+      // stage / half offset is formed once, before the first MMA.
+      constexpr uint64_t kStage = (2 * G::kTileBytes) >> 4;
+      constexpr uint64_t kPanel = (kBT * 128) >> 4;
+      constexpr uint64_t kHalf = (kDqStep * 128) >> 4;
+      uint64_t qd[D / 16], od[D / 16], kd0[D / 16], vd0[D / 16];
       kmajor_steps<D>(smem_addr(sm.res[0]), qd);
       kmajor_steps<D>(smem_addr(sm.res[1]), od);
+      kmajor_steps<D>(smem_addr(sm.ring[0][0]), kd0);
+      kmajor_steps<D>(smem_addr(sm.ring[0][1]), vd0);
+      const uint64_t kmn0 = sdesc_sw128(smem_addr(sm.ring[0][0]), kBT * 128, 1024);
       // S = Q K^T and dP = dO V^T of step m (keys 64 h .. of tile m / 2)
       auto issue_sdp = [&](int m) -> bool {
         const int b = m % kBwdBufs, t = m >> 1, h = m & 1, s = t % kBwdStages;
@@ -326,47 +342,51 @@ __device__ __forceinline__ void bwd_dq(const BackwardArgs& a, BwdSmem<D>& sm, in
           return false;
         if (h == 0 && !bwait(&sm.bar_full[s], (t / kBwdStages) & 1, abort_flag)) return false;
         tc_fence_after_sync();
+        const uint64_t off = kStage * s + kHalf * h;
         uint64_t kd[D / 16], vd[D / 16];
-        kmajor_steps<D>(smem_addr(sm.ring[s][0]) + h * kDqStep * 128, kd);
-        kmajor_steps<D>(smem_addr(sm.ring[s][1]) + h * kDqStep * 128, vd);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          kd[kk] = kd0[kk] + off;
+          vd[kk] = vd0[kk] + off;
+        }
         const uint32_t tSb = tmem + 128 + 128 * b;
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) mma_ss(tSb, qd[kk], kd[kk], kIdS, kk > 0 ? 1u : 0u);
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk)
-          mma_ss(tSb + kDqStep, od[kk], vd[kk], kIdS, kk > 0 ? 1u : 0u);
+        if constexpr (D == 128) {
+          mma_ss_x8<false>(tSb, qd, kd, kIdS, 0u);
+          mma_ss_x8<false>(tSb + kDqStep, od, vd, kIdS, 0u);
+        } else {
+          mma_ss_x4(tSb, qd, kd, kIdS, 0u);
+          mma_ss_x4(tSb + kDqStep, od, vd, kIdS, 0u);
+        }
         mma_commit(&sm.bar_sfull[b]);
         return true;
       };
       // dQ += dS K_step (A = dS from TMEM, 4 K-steps of 16 keys; B = the
-      // step's 64 key rows, MN-major, one MMA per 64-column panel)
+      // step's 64 key rows, MN-major, N = D)
       auto issue_dq = [&](int n) -> bool {
         const int b = n % kBwdBufs, t = n >> 1, h = n & 1, s = t % kBwdStages;
         if (!bwait(&sm.bar_pfull[b], (n / kBwdBufs) & 1, abort_flag)) return false;
         tc_fence_after_sync();
+        const uint64_t kb = kmn0 + kStage * s + 128 * 4 * h;
+        const uint64_t bd[4] = {kb, kb + 128, kb + 256, kb + 384};
         const uint32_t tSb = tmem + 128 + 128 * b;
-        const uint32_t kb = smem_addr(sm.ring[s][0]);
-#pragma unroll
-        for (int p = 0; p < P; ++p)
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            mma_ts(tdQ + 64 * p, tSb + 8 * kk, mn_step(kb, p, 4 * h + kk), kIdQ,
-                   (n > 0 || kk > 0) ? 1u : 0u);
+        mma_ts_x4(tdQ, tSb, tSb + 16, bd, kIdQ, n > 0 ? 1u : 0u);
         mma_commit(&sm.bar_done[b]);
         if (h == 1) mma_commit(&sm.bar_empty[s]);  // both halves of K_t, V_t read
         return true;
       };
-      bool ok = bwait(&sm.bar_res, 0, abort_flag) && issue_sdp(0);
-      for (int n = 0; ok && n < n_steps; ++n) {
-        if (n + 1 < n_steps) ok = issue_sdp(n + 1);
-        if (ok) ok = issue_dq(n);
+      bool ok = true;
+      if (warp == 1) {
+        ok = bwait(&sm.bar_res, 0, abort_flag);
+        for (int m = 0; ok && m < n_steps; ++m) ok = issue_sdp(m);
+      } else {
+        for (int n = 0; ok && n < n_steps; ++n) ok = issue_dq(n);
+        if (ok) mma_commit(&sm.bar_acc);
       }
-      if (ok) mma_commit(&sm.bar_acc);
-      drain_mmas(sm);
+      drain_mmas(sm, warp - 1);
     }
   } else {
     // ---------------------------------------------------- dS = P (dP - D) --
-    // Team t (warps 2-5 or 6-9) takes steps n = t, t + 2, ...; each thread
+    // Team t (warps 3-6 or 7-10) takes steps n = t, t + 2, ...; each thread
     // owns one stacked row (the 32x32b layout: lane quarter warp % 4).
     const int sw = warp - kBwdFirstSoftmax;
     const int team = sw >> 2;
@@ -482,17 +502,20 @@ __device__ __forceinline__ void bwd_dq(const BackwardArgs& a, BwdSmem<D>& sm, in
 // ----------------------------------------------------------------- dkv ------
 // One CTA per key tile kt of a group (cache tiles, then chunk tiles), K and V
 // resident.  The row tiles of the group's stacked rows stream through the
-// ring with their lambda and D and run as steps of W rows, step n in TMEM
-// buffer n % 3: S^T at columns 2D + 2W b, dP^T W columns after it; the
-// softmax writes bf16 P^T over S^T's first W/2 columns and dS^T over
-// dP^T's, dV (columns 0 ..) accumulates P^T dO and dK (columns D ..) dS^T Q.
-// The issue order is that of the dq kernel.
+// ring with their lambda and D and run as steps of W = 64 rows, step n in
+// TMEM buffer n % NB (two buffers for d = 128, three for d = 64): S^T at
+// columns 2D + 2W b, dP^T W columns after it; the softmax writes bf16 P^T
+// over S^T's first W/2 columns and dS^T over dP^T's, dV (columns 0 ..)
+// accumulates P^T dO and dK (columns D ..) dS^T Q.  The two issuing
+// threads work as in the dq kernel.
 template <int D>
 __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, int kt, int grp) {
   using G = BwdGeom<D>;
   constexpr int P = G::kPanels;
   constexpr int W = G::kW;
   constexpr int SPT = G::kStepsPerTile;
+  constexpr int NB = G::kDkvBufs;
+  static_assert(W == 64, "each softmax team takes 32 rows of a step");
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const uint32_t lane = tid & 31;
@@ -514,7 +537,7 @@ __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, i
     return pos >= 0 ? pos - a.pos0 : INT_MAX;
   };
 
-  if (tid == 0) init_barriers(sm);
+  if (tid == 0) init_barriers(sm, kBwdSoftmaxWarps);  // both teams on every step
   if (warp == 1) {
     tmem_alloc(&sm.taddr, 512);
     tmem_relinquish();
@@ -583,68 +606,83 @@ __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, i
       }
       if (*abort_flag) drain_loads(sm, uses, true);
     }
-  } else if (warp == 1) {
+  } else if (warp == 1 || warp == 2) {
     // ----------------------------------------------------------- MMA issue --
+    // warp 1: S^T and dP^T of every step; warp 2: dV and dK
     if (lane == 0 && n_t > 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBT, W, false);  // S^T, dP^T: N = W rows
-      constexpr uint32_t kIdG = idesc_bf16_f32(kBT, 64, true);  // dV, dK: one 64-column panel
-      uint64_t kd[D / 16], vd[D / 16];
+      constexpr uint32_t kIdG = idesc_bf16_f32(kBT, D, true);   // dV, dK: N = D
+      // descriptors as in the dq kernel; step w of a row tile starts W rows
+      // (W * 128 B) into it
+      constexpr uint64_t kStage = (2 * G::kTileBytes) >> 4;
+      constexpr uint64_t kRows = (W * 128) >> 4;
+      uint64_t kd[D / 16], vd[D / 16], qd0[D / 16], od0[D / 16];
       kmajor_steps<D>(smem_addr(sm.res[0]), kd);
       kmajor_steps<D>(smem_addr(sm.res[1]), vd);
+      kmajor_steps<D>(smem_addr(sm.ring[0][0]), qd0);
+      kmajor_steps<D>(smem_addr(sm.ring[0][1]), od0);
+      const uint64_t qmn0 = sdesc_sw128(smem_addr(sm.ring[0][0]), kBT * 128, 1024);
+      const uint64_t omn0 = sdesc_sw128(smem_addr(sm.ring[0][1]), kBT * 128, 1024);
       // S^T = K Q_w^T and dP^T = V dO_w^T of step m (rows W w .. of row tile m / SPT)
       auto issue_sdp = [&](int m) -> bool {
-        const int b = m % kBwdBufs, t = m / SPT, w = m % SPT, s = t % kBwdStages;
-        if (m >= kBwdBufs && !bwait(&sm.bar_done[b], (m / kBwdBufs - 1) & 1, abort_flag))
+        const int b = m % NB, t = m / SPT, w = m % SPT, s = t % kBwdStages;
+        if (m >= NB && !bwait(&sm.bar_done[b], (m / NB - 1) & 1, abort_flag))
           return false;
         if (w == 0 && !bwait(&sm.bar_full[s], (t / kBwdStages) & 1, abort_flag)) return false;
         tc_fence_after_sync();
+        const uint64_t off = kStage * s + kRows * w;
         uint64_t qd[D / 16], od[D / 16];
-        kmajor_steps<D>(smem_addr(sm.ring[s][0]) + w * W * 128, qd);
-        kmajor_steps<D>(smem_addr(sm.ring[s][1]) + w * W * 128, od);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          qd[kk] = qd0[kk] + off;
+          od[kk] = od0[kk] + off;
+        }
         const uint32_t tSb = tmem + 2 * D + 2 * W * b;
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) mma_ss(tSb, kd[kk], qd[kk], kIdS, kk > 0 ? 1u : 0u);
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) mma_ss(tSb + W, vd[kk], od[kk], kIdS, kk > 0 ? 1u : 0u);
+        if constexpr (D == 128) {
+          mma_ss_x8<false>(tSb, kd, qd, kIdS, 0u);
+          mma_ss_x8<false>(tSb + W, vd, od, kIdS, 0u);
+        } else {
+          mma_ss_x4(tSb, kd, qd, kIdS, 0u);
+          mma_ss_x4(tSb + W, vd, od, kIdS, 0u);
+        }
         mma_commit(&sm.bar_sfull[b]);
         return true;
       };
       // dV += P^T dO_w, dK += dS^T Q_w (A from TMEM, W / 16 K-steps of 16
-      // rows; B = the step's rows, MN-major, one MMA per 64-column panel)
+      // rows; B = the step's rows, MN-major, N = D)
       auto issue_kv = [&](int n) -> bool {
-        const int b = n % kBwdBufs, t = n / SPT, w = n % SPT, s = t % kBwdStages;
-        if (!bwait(&sm.bar_pfull[b], (n / kBwdBufs) & 1, abort_flag)) return false;
+        const int b = n % NB, t = n / SPT, w = n % SPT, s = t % kBwdStages;
+        if (!bwait(&sm.bar_pfull[b], (n / NB) & 1, abort_flag)) return false;
         tc_fence_after_sync();
         const uint32_t tSb = tmem + 2 * D + 2 * W * b;
-        const uint32_t qb = smem_addr(sm.ring[s][0]), ob = smem_addr(sm.ring[s][1]);
-#pragma unroll
-        for (int p = 0; p < P; ++p)
-#pragma unroll
-          for (int kk = 0; kk < W / 16; ++kk)
-            mma_ts(tdV + 64 * p, tSb + 8 * kk, mn_step(ob, p, (W / 16) * w + kk), kIdG,
-                   (n > 0 || kk > 0) ? 1u : 0u);
-#pragma unroll
-        for (int p = 0; p < P; ++p)
-#pragma unroll
-          for (int kk = 0; kk < W / 16; ++kk)
-            mma_ts(tdK + 64 * p, tSb + W + 8 * kk, mn_step(qb, p, (W / 16) * w + kk), kIdG,
-                   (n > 0 || kk > 0) ? 1u : 0u);
+        const uint64_t off = kStage * s + 128 * (W / 16) * w;
+        const uint32_t acc = n > 0 ? 1u : 0u;
+        // rows 0-31 of the step (K-steps 0, 1) as bf16 pairs at columns 0-15
+        // of the buffer half, rows 32-63 (K-steps 2, 3) at columns 32-47
+        const uint64_t bo[4] = {omn0 + off, omn0 + off + 128, omn0 + off + 256, omn0 + off + 384};
+        const uint64_t bq[4] = {qmn0 + off, qmn0 + off + 128, qmn0 + off + 256, qmn0 + off + 384};
+        mma_ts_x4(tdV, tSb, tSb + 32, bo, kIdG, acc);
+        mma_ts_x4(tdK, tSb + W, tSb + W + 32, bq, kIdG, acc);
         mma_commit(&sm.bar_done[b]);
         if (w == SPT - 1) mma_commit(&sm.bar_empty[s]);  // the row tile's last step
         return true;
       };
-      bool ok = bwait(&sm.bar_res, 0, abort_flag) && issue_sdp(0);
-      for (int n = 0; ok && n < n_steps; ++n) {
-        if (n + 1 < n_steps) ok = issue_sdp(n + 1);
-        if (ok) ok = issue_kv(n);
+      bool ok = true;
+      if (warp == 1) {
+        ok = bwait(&sm.bar_res, 0, abort_flag);
+        for (int m = 0; ok && m < n_steps; ++m) ok = issue_sdp(m);
+      } else {
+        for (int n = 0; ok && n < n_steps; ++n) ok = issue_kv(n);
+        if (ok) mma_commit(&sm.bar_acc);
       }
-      if (ok) mma_commit(&sm.bar_acc);
-      drain_mmas(sm);
+      drain_mmas(sm, warp - 1);
     }
   } else {
     // ------------------------------------ P^T and dS^T = P^T (dP^T - D) --
-    // Team t takes steps n = t, t + 2, ...; each thread owns one key (the
-    // 32x32b layout: lane quarter warp % 4), the columns are stacked rows.
+    // Both teams work on every step, team t on its rows 32 t .. 32 t + 31
+    // (with two buffers at d = 128 the steps cannot overlap, so the step's
+    // softmax latency is what matters); each thread owns one key (the 32x32b
+    // layout: lane quarter warp % 4), the columns are stacked rows.
     const int sw = warp - kBwdFirstSoftmax;
     const int team = sw >> 2;
     const int q4 = warp & 3;
@@ -654,10 +692,10 @@ __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, i
     const float2 sc = make_float2(sl2, sl2);
     const uint32_t lane_addr = static_cast<uint32_t>(q4 * 32) << 16;
     bool ok = true;
-    for (int n = team; n < n_steps; n += 2) {
-      const int b = n % kBwdBufs, t = n / SPT, w = n % SPT, s = t % kBwdStages;
+    for (int n = 0; n < n_steps; ++n) {
+      const int b = n % NB, t = n / SPT, w = n % SPT, s = t % kBwdStages;
       // the S^T buffer, and the stage's lambda and D (complete with its tiles)
-      if (!wwait(&sm.bar_sfull[b], (n / kBwdBufs) & 1, abort_flag) ||
+      if (!wwait(&sm.bar_sfull[b], (n / NB) & 1, abort_flag) ||
           !wwait(&sm.bar_full[s], (t / kBwdStages) & 1, abort_flag)) {
         ok = false;
         break;
@@ -667,8 +705,8 @@ __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, i
       const bool partial = (e & kBPartial) != 0;
       const int rs0 = (e & kBIdxMask) * kBT + w * W;  // first stacked row of the step
       const uint32_t tSb = tmem + 2 * D + 2 * W * b + lane_addr;
-#pragma unroll 1
-      for (int hh = 0; hh < W / 32; ++hh) {
+      {
+        const int hh = team;
         uint32_t sr[32], pr[32];
         tmem_ld32_async(tSb + 32 * hh, sr);
         tmem_ld32_async(tSb + W + 32 * hh, pr);
@@ -713,10 +751,10 @@ __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, i
             dk[(k + x) / 2] = pack_bf16x2(g0, g1);
           }
         }
-        // rows 32 hh .. 32 hh + 31 of the step as bf16 pairs over columns
-        // 16 hh .. of S^T and of dP^T (columns this thread has already loaded)
-        tmem_st16_async(tSb + 16 * hh, pk);
-        tmem_st16_async(tSb + W + 16 * hh, dk);
+        // rows 32 hh .. 32 hh + 31 of the step as bf16 pairs over the first
+        // 16 of the columns this thread has just loaded, in S^T and in dP^T
+        tmem_st16_async(tSb + 32 * hh, pk);
+        tmem_st16_async(tSb + W + 32 * hh, dk);
       }
       tmem_wait_st();
       tc_fence_before_sync();
@@ -759,19 +797,24 @@ __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, i
   }
 }
 
-// One launch for both halves of the gradient: blockIdx.x < n_row_tiles is a
-// dq CTA (row tile blockIdx.x), the rest are dkv CTAs (key tile blockIdx.x -
-// n_row_tiles), so that the two kinds fill the SMs together.
+// One launch for both halves of the gradient, a 1-D grid: the first
+// n_row_tiles x groups CTAs form dq (row tile, group), the rest dk / dv (key
+// tile, group).  The dq CTAs, the longest, are dispatched first, and the
+// shorter dk / dv CTAs fill the SMs around them and after them.
 template <int D>
 __global__ void __launch_bounds__(kBwdThreads, 1) bwd_kernel(const __grid_constant__ BackwardArgs a,
-                                                            int n_row_tiles) {
+                                                            int n_row_tiles, int n_key_tiles) {
   extern __shared__ uint8_t smem_raw[];
   auto& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw +
                                             ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
   const int x = static_cast<int>(blockIdx.x);
-  const int grp = static_cast<int>(blockIdx.y);
-  if (x < n_row_tiles) bwd_dq<D>(a, sm, x, grp);
-  else bwd_dkv<D>(a, sm, x - n_row_tiles, grp);
+  const int n_dq = n_row_tiles * a.B * a.Hkv;
+  if (x < n_dq) {
+    bwd_dq<D>(a, sm, x % n_row_tiles, x / n_row_tiles);
+  } else {
+    const int y = x - n_dq;
+    bwd_dkv<D>(a, sm, y % n_key_tiles, y / n_key_tiles);
+  }
   if (threadIdx.x == 0 && sm.abort_flag) atomicOr(a.err, H2O_DEVERR_TIMEOUT);
 }
 
@@ -792,9 +835,9 @@ cudaError_t launch_backward_d(const BackwardArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const int n_row_tiles = (R + kBT - 1) / kBT;
   const int n_key_tiles = (a.M + kBT - 1) / kBT + (a.S + kBT - 1) / kBT;
-  const dim3 grid(static_cast<unsigned>(n_row_tiles + n_key_tiles),
-                  static_cast<unsigned>(a.B * a.Hkv));
-  bwd_kernel<D><<<grid, kBwdThreads, smem, stream>>>(a, n_row_tiles);
+  const int64_t ctas = static_cast<int64_t>(n_row_tiles + n_key_tiles) * a.B * a.Hkv;
+  bwd_kernel<D><<<static_cast<unsigned>(ctas), kBwdThreads, smem, stream>>>(a, n_row_tiles,
+                                                                            n_key_tiles);
   return cudaGetLastError();
 }
 

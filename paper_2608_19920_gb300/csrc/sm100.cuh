@@ -368,6 +368,43 @@ __device__ __forceinline__ void mma_ts_x8(uint32_t d_tmem, uint32_t a_lo, uint32
 }
 #undef H2O_MMA8
 
+// Four (two) 1-SM MMAs issued back to back from one asm block; the first
+// accumulates into D iff acc_first != 0.  ss: A and B from shared memory;
+// ts: A from TMEM.
+__device__ __forceinline__ void mma_ss_x4(uint32_t d_tmem, const uint64_t (&a)[4],
+                                          const uint64_t (&b)[4], uint32_t idesc,
+                                          uint32_t acc_first) {
+  asm volatile(
+      "{\n\t.reg .pred p0, p1;\n\t"
+      "setp.ne.b32 p0, %2, 0;\n\t"
+      "setp.eq.b32 p1, %2, %2;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %3, %7, %1, p0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %4, %8, %1, p1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %5, %9, %1, p1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %6, %10, %1, p1;\n\t}" ::"r"(d_tmem),
+      "r"(idesc), "r"(acc_first), "l"(a[0]), "l"(a[1]), "l"(a[2]), "l"(a[3]), "l"(b[0]),
+      "l"(b[1]), "l"(b[2]), "l"(b[3])
+      : "memory");
+}
+
+// (ts_x4: K-steps 0-1 at a_lo + 8k, 2-3 at a_hi + 8(k - 2).)
+__device__ __forceinline__ void mma_ts_x4(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi,
+                                          const uint64_t (&b)[4], uint32_t idesc,
+                                          uint32_t acc_first) {
+  asm volatile(
+      "{\n\t.reg .pred p0, p1;\n\t"
+      "setp.ne.b32 p0, %2, 0;\n\t"
+      "setp.eq.b32 p1, %2, %2;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%3], %7, %1, p0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%4], %8, %1, p1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%5], %9, %1, p1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%6], %10, %1, p1;\n\t}" ::"r"(d_tmem),
+      "r"(idesc), "r"(acc_first), "r"(a_lo), "r"(a_lo + 8), "r"(a_hi), "r"(a_hi + 8), "l"(b[0]),
+      "l"(b[1]), "l"(b[2]), "l"(b[3])
+      : "memory");
+}
+
+
 // Arrives on `bar` once every MMA issued so far by this thread has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile(

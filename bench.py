@@ -699,12 +699,15 @@ def run_kernel_only(args, w, n_fill: int = 8):
 
 
 def run_backward(args, w, n_fill: int = 8):
-    """Times h2o_sdpa_chunk_backward on the chunk after a prefill and ``n_fill``
-    chunks (the forward's inputs and output, an all-ones-scaled random dout),
-    L2 flushed before each launch, replayed from a CUDA graph."""
+    """Times the chunk-SDPA gradient on the chunk after a prefill and ``n_fill``
+    chunks (the forward's inputs and output, a random dout), L2 flushed before
+    each launch, replayed from a CUDA graph: h2o_sdpa_chunk_backward (which
+    recomputes each row's log-sum-exp) and h2o_sdpa_chunk_backward_lse (given
+    the forward's, from h2o_sdpa_chunk_lse)."""
     import torch
     from paper_2608_19920_gb300 import (H2OLayer, build as build_mod, h2o_backward_workspace_size,
-                                       h2o_device_errors, h2o_sdpa_chunk, h2o_sdpa_chunk_backward)
+                                       h2o_device_errors, h2o_sdpa_chunk_backward,
+                                       h2o_sdpa_chunk_lse)
     from paper_2608_19920_gb300._binding import H2ODims
     build_mod.build()
     dev = torch.device("cuda", 0)
@@ -718,46 +721,52 @@ def run_backward(args, w, n_fill: int = 8):
     p, e = plan[-1]
     q, k, v = ins[-1]
     S = e - p
-    out, _ = h2o_sdpa_chunk(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p)
+    out, _, lse = h2o_sdpa_chunk_lse(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p)
     dout = torch.randn(out.shape, device=dev, generator=torch.Generator(dev).manual_seed(0))
     dout = dout.to(torch.bfloat16)
     ws = torch.empty(h2o_backward_workspace_size(H2ODims(w.B, w.Hq, w.Hkv, w.d, S, w.M)),
                      dtype=torch.uint8, device=dev)
-
-    def call():
-        h2o_sdpa_chunk_backward(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out,
-                                dout, workspace=ws)
-
-    call()
-    torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        call()
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     clean = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
-    times = []
-    for _ in range(args.reps + 2):
-        flush.zero_()
-        clean.sum()
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        graph.replay()
-        b.record(stream)
+
+    def timed(saved):
+        def call():
+            h2o_sdpa_chunk_backward(q, layer.k_cache, layer.v_cache, k, v, layer.slot_pos, p, out,
+                                    dout, workspace=ws, lse=lse if saved else None)
+
+        call()
         torch.cuda.synchronize()
-        times.append(a.elapsed_time(b))
-    assert h2o_device_errors() == 0
-    avg_ms = sum(times[2:]) / len(times[2:])
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            call()
+        times = []
+        for _ in range(args.reps + 2):
+            flush.zero_()
+            clean.sum()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            graph.replay()
+            b.record(stream)
+            torch.cuda.synchronize()
+            times.append(a.elapsed_time(b))
+        assert h2o_device_errors() == 0
+        return sum(times[2:]) / len(times[2:])
+
+    avg_ms = timed(False)
+    avg_ms_lse = timed(True)
     # five contractions over the visible keys (Q K^T again, dout V^T, dS K,
     # dS^T Q, P^T dout): 2.5 times the forward's algorithmic flops
     flops = 2.5 * chunk_flops(w.B, w.Hq, w.d, S, w.M)
-    executed = 10.0 * w.B * w.Hq * S * w.d * (w.M + S)
     pk = peaks()
     tf = flops / (avg_ms / 1e3) / 1e12
-    print(json.dumps({"mode": "backward", "workload": w.name, "S": S, "avg_us": avg_ms * 1e3,
-                      "flops": flops, "alg_tflops": tf, "executed_tflops": executed / flops * tf,
-                      "frac_of_bf16_peak": tf / pk["bf16"], "workspace_bytes": ws.numel()}))
+    tf_lse = flops / (avg_ms_lse / 1e3) / 1e12
+    print(json.dumps({"mode": "backward", "workload": w.name, "S": S, "flops": flops,
+                      "avg_us": avg_ms * 1e3, "alg_tflops": tf, "frac_of_bf16_peak": tf / pk["bf16"],
+                      "saved_lse_avg_us": avg_ms_lse * 1e3, "saved_lse_alg_tflops": tf_lse,
+                      "saved_lse_frac_of_bf16_peak": tf_lse / pk["bf16"],
+                      "workspace_bytes": ws.numel()}))
     return 0
 
 

@@ -24,7 +24,9 @@
  *                                    (write first, then attend; §3.1, §3.3.1)
  *   h2o_kv_replace, h2o_kv_restore   replay-cache row writes and the reverse
  *                                    recurrence (§3.2, §A.1.1)
- *   h2o_sdpa_chunk_backward          the gradient of one chunk's SDPA
+ *   h2o_sdpa_chunk_lse, h2o_sdpa_chunk_backward, h2o_sdpa_chunk_backward_lse
+ *                                    the gradient of one chunk's SDPA (given
+ *                                    the forward's lse, or recomputing it)
  *   h2o_sdpa_decode_static           S = 1 SDPA on a fixed internal scratch
  *   h2o_kv_quantize, h2o_kv_dequantize, h2o_update_q8, h2o_evict_insert_q8,
  *   h2o_sdpa_chunk_q8, h2o_sdpa_cache_q8, h2o_q8_workspace_size
@@ -130,6 +132,22 @@ H2O_API int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_s
                    const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
                    h2o_bf16* out, float* score_inc, void* workspace, size_t workspace_bytes,
                    void* stream);
+
+/*
+ * h2o_sdpa_chunk that also writes, for a later h2o_sdpa_chunk_backward_lse,
+ * each query row's log-sum-exp of the visible scaled logits (§3.1 Eq. 2's
+ * normaliser, natural log):
+ *
+ *   lse  (B, Hq, S) f32, written: lse[b, hq, i] = log sum_{j visible} exp(scale q_i . k_j)
+ *
+ * Other arguments, results and the workspace as for h2o_sdpa_chunk.  S = 1
+ * also runs the chunk kernel here (the decode kernels keep no lse).
+ */
+H2O_API int h2o_sdpa_chunk_lse(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                   const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
+                   h2o_bf16* out, float* score_inc, float* lse, void* workspace,
+                   size_t workspace_bytes, void* stream);
 
 /*
  * h2o_sdpa_chunk for one query token per sequence (dims->S == 1, M >= 1,
@@ -387,6 +405,23 @@ H2O_API int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float 
                    const h2o_bf16* out, const h2o_bf16* dout, float* dq, float* dk_cache,
                    float* dv_cache, float* dk_new, float* dv_new, void* workspace,
                    size_t workspace_bytes, void* stream);
+
+/*
+ * h2o_sdpa_chunk_backward given the forward's lse (h2o_sdpa_chunk_lse on the
+ * same inputs), as a fine-tuning step that keeps it has it: the log-sum-exp
+ * is read instead of recomputed (a row kernel forms D = dout . out and the
+ * log2-unit copy the kernel uses), then the fused kernel runs.
+ *
+ *   lse  (B, Hq, S) f32, read
+ *
+ * Other arguments, results, workspace and errors as h2o_sdpa_chunk_backward.
+ */
+H2O_API int h2o_sdpa_chunk_backward_lse(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                   const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                   const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
+                   const h2o_bf16* out, const h2o_bf16* dout, const float* lse, float* dq,
+                   float* dk_cache, float* dv_cache, float* dk_new, float* dv_new,
+                   void* workspace, size_t workspace_bytes, void* stream);
 
 /* Empties a cache before a new sequence: slot_pos (B, Hkv, M) int32 := -1 and
  * scores (B, Hkv, M) f32 := 0, enqueued on `stream` (the K/V buffers need no

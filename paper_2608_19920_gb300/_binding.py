@@ -24,7 +24,8 @@ H2O_DEVERR_INDEX = 4
 EXPORTS = ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
            "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
            "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
-           "h2o_sdpa_chunk_backward", "h2o_selftest_bounded_wait",
+           "h2o_sdpa_chunk_backward", "h2o_sdpa_chunk_lse", "h2o_sdpa_chunk_backward_lse",
+           "h2o_selftest_bounded_wait",
            "h2o_kv_quantize", "h2o_kv_dequantize", "h2o_q8_workspace_size", "h2o_update_q8",
            "h2o_evict_insert_q8", "h2o_sdpa_chunk_q8", "h2o_sdpa_cache_q8",
            "h2o_cache_reset", "h2o_status_string", "h2o_last_cuda_error", "h2o_device_errors",
@@ -78,6 +79,9 @@ def load(path: str = LIB_PATH):
     lib.h2o_kv_restore.argtypes = [dims_p, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.h2o_backward_workspace_size.argtypes = [dims_p, ctypes.POINTER(ctypes.c_size_t)]
     lib.h2o_sdpa_chunk_backward.argtypes = [dims_p, i64, f32] + [vp] * 14 + [ctypes.c_size_t, vp]
+    lib.h2o_sdpa_chunk_lse.argtypes = [dims_p, i64, f32] + [vp] * 10 + [ctypes.c_size_t, vp]
+    lib.h2o_sdpa_chunk_backward_lse.argtypes = ([dims_p, i64, f32] + [vp] * 15 +
+                                                [ctypes.c_size_t, vp])
     lib.h2o_selftest_bounded_wait.argtypes = [i64, vp]
     lib.h2o_kv_quantize.argtypes = [i64, i32, vp, vp, vp, vp]
     lib.h2o_kv_dequantize.argtypes = [i64, i32, vp, vp, vp, vp]
@@ -92,7 +96,8 @@ def load(path: str = LIB_PATH):
     for fn in ("h2o_workspace_size", "h2o_sdpa_chunk", "h2o_sdpa_decode_static", "h2o_update",
                "h2o_update_policy", "h2o_evict_insert", "h2o_sdpa_cache", "h2o_scores_add",
                "h2o_kv_replace", "h2o_kv_restore", "h2o_backward_workspace_size",
-               "h2o_sdpa_chunk_backward", "h2o_selftest_bounded_wait", "h2o_cache_reset",
+               "h2o_sdpa_chunk_backward", "h2o_sdpa_chunk_lse", "h2o_sdpa_chunk_backward_lse",
+               "h2o_selftest_bounded_wait", "h2o_cache_reset",
                "h2o_kv_quantize", "h2o_kv_dequantize", "h2o_q8_workspace_size",
                "h2o_update_q8", "h2o_evict_insert_q8", "h2o_sdpa_chunk_q8", "h2o_sdpa_cache_q8",
                "h2o_last_cuda_error",
@@ -182,6 +187,38 @@ def h2o_sdpa_chunk(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale
                             _ptr(score_inc), _ptr(workspace), ws_bytes, _stream(stream))
     _check("h2o_sdpa_chunk", st)
     return out, score_inc
+
+
+def h2o_sdpa_chunk_lse(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, scale: float = 0.0,
+                       workspace=None, stream=None):
+    """h2o_sdpa_chunk that also returns each query row's log-sum-exp (natural
+    log), for h2o_sdpa_chunk_backward_lse.  Returns (out, score_inc, lse
+    (B,Hq,S) f32)."""
+    lib = load()
+    dev = q.device
+    B, Hq, S, d = q.shape
+    Hkv, M = k_new.shape[1], k_cache.shape[2]
+    bf = torch.bfloat16
+    for t, n, shp, dt in ((q, "q", (B, Hq, S, d), bf), (k_cache, "k_cache", (B, Hkv, M, d), bf),
+                          (v_cache, "v_cache", (B, Hkv, M, d), bf),
+                          (k_new, "k_new", (B, Hkv, S, d), bf), (v_new, "v_new", (B, Hkv, S, d), bf),
+                          (slot_pos, "slot_pos", (B, Hkv, M), torch.int32)):
+        _expect(t, n, shp, dt, dev)
+    out = torch.empty((B, Hq, S, d), dtype=bf, device=dev)
+    score_inc = torch.empty((B, Hq, M + S), dtype=torch.float32, device=dev)
+    lse = torch.empty((B, Hq, S), dtype=torch.float32, device=dev)
+    dims = H2ODims(B, Hq, Hkv, d, S, M)
+    if workspace is None:
+        n = h2o_workspace_size(dims)
+        if n:
+            workspace = torch.empty(n, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.h2o_sdpa_chunk_lse(ctypes.byref(dims), int(pos0), float(scale), _ptr(q),
+                                _ptr(k_cache), _ptr(v_cache), _ptr(k_new), _ptr(v_new),
+                                _ptr(slot_pos), _ptr(out), _ptr(score_inc), _ptr(lse),
+                                _ptr(workspace), ws_bytes, _stream(stream))
+    _check("h2o_sdpa_chunk_lse", st)
+    return out, score_inc, lse
 
 
 def h2o_sdpa_decode_static(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int,
@@ -401,9 +438,10 @@ def h2o_backward_workspace_size(dims: H2ODims) -> int:
 
 
 def h2o_sdpa_chunk_backward(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, out, dout,
-                            scale: float = 0.0, workspace=None, stream=None):
+                            scale: float = 0.0, workspace=None, stream=None, lse=None):
     """Gradient of sum(out * dout) for one h2o_sdpa_chunk call (see include/h2o.h).
-    Returns fp32 (dq, dk_cache, dv_cache, dk_new, dv_new)."""
+    Returns fp32 (dq, dk_cache, dv_cache, dk_new, dv_new).  With ``lse`` (the
+    forward's, from h2o_sdpa_chunk_lse) this calls h2o_sdpa_chunk_backward_lse."""
     lib = load()
     dev = q.device
     B, Hq, S, d = q.shape
@@ -425,13 +463,26 @@ def h2o_sdpa_chunk_backward(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: i
     if workspace is None:
         workspace = torch.empty(h2o_backward_workspace_size(dims), dtype=torch.uint8, device=dev)
     ws_bytes = workspace.numel() * workspace.element_size()
-    st = lib.h2o_sdpa_chunk_backward(
-        ctypes.byref(dims), int(pos0), float(scale), _ptr(q), _ptr(k_cache), _ptr(v_cache),
-        _ptr(k_new), _ptr(v_new), _ptr(slot_pos), _ptr(out), _ptr(dout), _ptr(dq),
-        _ptr(dkc if M else None), _ptr(dvc if M else None), _ptr(dkn), _ptr(dvn),
-        _ptr(workspace), ws_bytes, _stream(stream))
-    _check("h2o_sdpa_chunk_backward", st)
+    head = (ctypes.byref(dims), int(pos0), float(scale), _ptr(q), _ptr(k_cache), _ptr(v_cache),
+            _ptr(k_new), _ptr(v_new), _ptr(slot_pos), _ptr(out), _ptr(dout))
+    tail = (_ptr(dq), _ptr(dkc if M else None), _ptr(dvc if M else None), _ptr(dkn), _ptr(dvn),
+            _ptr(workspace), ws_bytes, _stream(stream))
+    if lse is None:
+        st = lib.h2o_sdpa_chunk_backward(*head, *tail)
+        _check("h2o_sdpa_chunk_backward", st)
+    else:
+        _expect(lse, "lse", (B, Hq, S), torch.float32, dev)
+        st = lib.h2o_sdpa_chunk_backward_lse(*head, _ptr(lse), *tail)
+        _check("h2o_sdpa_chunk_backward_lse", st)
     return dq, dkc, dvc, dkn, dvn
+
+
+def h2o_sdpa_chunk_backward_lse(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0: int, out, dout,
+                                lse, scale: float = 0.0, workspace=None, stream=None):
+    """h2o_sdpa_chunk_backward given the forward's lse (h2o_sdpa_chunk_lse):
+    the log-sum-exp is not recomputed."""
+    return h2o_sdpa_chunk_backward(q, k_cache, v_cache, k_new, v_new, slot_pos, pos0, out, dout,
+                                   scale, workspace, stream, lse=lse)
 
 
 def h2o_cache_reset(slot_pos, scores, stream=None):

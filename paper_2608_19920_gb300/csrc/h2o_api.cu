@@ -125,12 +125,15 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
               const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
               const h2o_bf16* v_new, const int32_t* slot_pos, h2o_bf16* out, float* score_inc,
               void* workspace, size_t workspace_bytes, void* stream, bool cache_only,
-              const Q8Buffers* q8 = nullptr, float* lse = nullptr, int lse_stride = 0) {
+              const Q8Buffers* q8 = nullptr, const SdpaArgs* lse_req = nullptr,
+              float* lse_out = nullptr) {
+  // lse_req (the backward's recomputation): its lse, lse_stride, bwd_out,
+  // bwd_dout and drow fields; the chunk kernel's pass 1 alone then writes the
+  // rows' log-sum-exp and D, and neither out nor score_inc
+  float* lse = lse_req ? lse_req->lse : nullptr;
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
-  // lse (the backward's recomputation): the chunk kernel's pass 1 alone,
-  // which writes the rows' log-sum-exp and neither out nor score_inc
   if (!q || (!lse && (!out || !score_inc)) || (!cache_only && (!k_new || !v_new)))
     return H2O_ERR_NULL;
   // (q8: the codes were checked by the caller; the decode kernels need no rows)
@@ -146,8 +149,11 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
   int split_len = 0, n_split = 0;
   size_t ws_need = 0;
-  const bool decode =
-      !lse && decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
+  // lse_out (the forward's lse for a later backward): the chunk kernel, also
+  // for S = 1, which writes each row's lambda as it enters its second pass
+  if (lse_out && misaligned(lse_out)) return H2O_ERR_ALIGN;
+  const bool decode = !lse && !lse_out &&
+                      decode_plan(D.B, D.Hq, D.Hkv, D.d, D.S, D.M, &split_len, &n_split, &ws_need);
   if (!decode) ws_need = lse ? 0 : sdpa_colpart_bytes(D.B, D.Hq, D.S, D.M);
   if (ws_need > 0 && (!workspace || workspace_bytes < ws_need)) return H2O_ERR_WORKSPACE;
   if (ws_need > 0 && misaligned(workspace)) return H2O_ERR_ALIGN;
@@ -209,8 +215,14 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
   a.score_inc = score_inc;
   a.err = di->err_word;
   a.colpart = ws_need > 0 ? static_cast<float*>(workspace) : nullptr;
-  a.lse = lse;
-  a.lse_stride = lse_stride;
+  a.lse_out = lse_out;
+  if (lse_req) {
+    a.lse = lse_req->lse;
+    a.lse_stride = lse_req->lse_stride;
+    a.bwd_out = lse_req->bwd_out;
+    a.bwd_dout = lse_req->bwd_dout;
+    a.drow = lse_req->drow;
+  }
 
   const uint64_t G = static_cast<uint64_t>(D.B) * D.Hkv;
   {
@@ -434,6 +446,16 @@ int h2o_sdpa_chunk(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, co
                    float* score_inc, void* workspace, size_t workspace_bytes, void* stream) {
   return sdpa_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, k_new, v_new, slot_pos, out,
                    score_inc, workspace, workspace_bytes, stream, false);
+}
+
+int h2o_sdpa_chunk_lse(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                       const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                       const h2o_bf16* k_new, const h2o_bf16* v_new, const int32_t* slot_pos,
+                       h2o_bf16* out, float* score_inc, float* lse, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+  if (!lse) return H2O_ERR_NULL;
+  return sdpa_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, k_new, v_new, slot_pos, out,
+                   score_inc, workspace, workspace_bytes, stream, false, nullptr, nullptr, lse);
 }
 
 int h2o_sdpa_cache(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
@@ -671,23 +693,26 @@ int h2o_backward_workspace_size(const h2o_dims_t* dims, size_t* bytes) {
   return H2O_OK;
 }
 
-int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
-                            const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
-                            const h2o_bf16* k_new, const h2o_bf16* v_new,
-                            const int32_t* slot_pos, const h2o_bf16* out,
-                            const h2o_bf16* dout, float* dq, float* dk_cache, float* dv_cache,
-                            float* dk_new, float* dv_new, void* workspace,
-                            size_t workspace_bytes, void* stream) {
+// h2o_sdpa_chunk_backward (lse_saved = NULL: the rows' log-sum-exp is
+// recomputed by the forward kernel's first pass, which also forms D) and
+// h2o_sdpa_chunk_backward_lse (the forward's saved lse; a row kernel forms D).
+static int backward_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h2o_bf16* q,
+                  const h2o_bf16* k_cache, const h2o_bf16* v_cache, const h2o_bf16* k_new,
+                  const h2o_bf16* v_new, const int32_t* slot_pos, const h2o_bf16* out,
+                  const h2o_bf16* dout, const float* lse_saved, float* dq, float* dk_cache,
+                  float* dv_cache, float* dk_new, float* dv_new, void* workspace,
+                  size_t workspace_bytes, void* stream, bool with_lse) {
   int st = check_dims(dims);
   if (st != H2O_OK) return st;
   const h2o_dims_t& D = *dims;
   if (!q || !k_new || !v_new || !out || !dout || !dq || !dk_new || !dv_new) return H2O_ERR_NULL;
+  if (with_lse && !lse_saved) return H2O_ERR_NULL;
   if (D.M > 0 && (!k_cache || !v_cache || !slot_pos || !dk_cache || !dv_cache))
     return H2O_ERR_NULL;
   if (misaligned(q) || misaligned(k_cache) || misaligned(v_cache) || misaligned(k_new) ||
       misaligned(v_new) || misaligned(slot_pos) || misaligned(out) || misaligned(dout) ||
       misaligned(dq) || misaligned(dk_cache) || misaligned(dv_cache) || misaligned(dk_new) ||
-      misaligned(dv_new) || misaligned(workspace))
+      misaligned(dv_new) || misaligned(workspace) || misaligned(lse_saved))
     return H2O_ERR_ALIGN;
   if (pos0 < 0 || pos0 + D.S >= (int64_t(1) << 31)) return H2O_ERR_ARG;
   if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale)) return H2O_ERR_ARG;
@@ -702,8 +727,7 @@ int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(D.d));
   BackwardArgs a;
   std::memset(&a, 0, sizeof(a));
-  a.q = q; a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
-  a.slot_pos = slot_pos; a.out = out; a.dout = dout;
+  a.slot_pos = slot_pos;
   a.dq = dq; a.dk_cache = dk_cache; a.dv_cache = dv_cache; a.dk_new = dk_new; a.dv_new = dv_new;
   a.err = di->err_word;
   a.B = D.B; a.Hq = D.Hq; a.Hkv = D.Hkv; a.d = D.d; a.S = D.S; a.M = D.M; a.qg = qg;
@@ -729,12 +753,52 @@ int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_
       if ((st = encode(&a.tm_vc, v_cache, 3, dc, box)) != H2O_OK) return st;
     }
   }
-  // each row's log-sum-exp, from the forward kernel's first pass
+  if (with_lse) {
+    // the saved lse and D = dout . out, into the padded row layout
+    cudaError_t e = launch_backward_rows(a, out, dout, lse_saved, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e);
+    e = launch_backward(a, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+  }
+  // each row's log-sum-exp and D = dout . out, from the forward kernel's
+  // first pass
+  SdpaArgs req;
+  std::memset(&req, 0, sizeof(req));
+  req.lse = a.lse;
+  req.lse_stride = Rp;
+  req.bwd_out = out;
+  req.bwd_dout = dout;
+  req.drow = a.drow;
   st = sdpa_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, k_new, v_new, slot_pos, nullptr,
-                 nullptr, nullptr, 0, stream, false, nullptr, a.lse, Rp);
+                 nullptr, nullptr, 0, stream, false, nullptr, &req);
   if (st != H2O_OK) return st;
   const cudaError_t e = launch_backward(a, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? H2O_OK : cuda_fail(e);
+}
+
+int h2o_sdpa_chunk_backward(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                            const h2o_bf16* q, const h2o_bf16* k_cache, const h2o_bf16* v_cache,
+                            const h2o_bf16* k_new, const h2o_bf16* v_new,
+                            const int32_t* slot_pos, const h2o_bf16* out,
+                            const h2o_bf16* dout, float* dq, float* dk_cache, float* dv_cache,
+                            float* dk_new, float* dv_new, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  return backward_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, k_new, v_new, slot_pos, out,
+                       dout, nullptr, dq, dk_cache, dv_cache, dk_new, dv_new, workspace,
+                       workspace_bytes, stream, false);
+}
+
+int h2o_sdpa_chunk_backward_lse(const h2o_dims_t* dims, int64_t pos0, float softmax_scale,
+                                const h2o_bf16* q, const h2o_bf16* k_cache,
+                                const h2o_bf16* v_cache, const h2o_bf16* k_new,
+                                const h2o_bf16* v_new, const int32_t* slot_pos,
+                                const h2o_bf16* out, const h2o_bf16* dout, const float* lse,
+                                float* dq, float* dk_cache, float* dv_cache, float* dk_new,
+                                float* dv_new, void* workspace, size_t workspace_bytes,
+                                void* stream) {
+  return backward_impl(dims, pos0, softmax_scale, q, k_cache, v_cache, k_new, v_new, slot_pos, out,
+                       dout, lse, dq, dk_cache, dv_cache, dk_new, dv_new, workspace,
+                       workspace_bytes, stream, true);
 }
 
 int h2o_cache_reset(const h2o_dims_t* dims, int32_t* slot_pos, float* scores, void* stream) {

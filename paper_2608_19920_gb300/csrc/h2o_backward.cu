@@ -13,8 +13,9 @@
 // Hidden (i, j) pairs have m_ij = 0, so cache slots no row sees get zero
 // gradients.
 //
-// Two tcgen05 kernels, neither materialising a score matrix and neither
-// using atomics (so the result does not depend on scheduling):
+// Two kinds of tcgen05 CTA in one launch, neither materialising a score
+// matrix and neither using atomics (so the result does not depend on
+// scheduling):
 //  * bwd_dq_kernel: one CTA per 128 stacked rows; per key tile, S = Q K^T and
 //    dP = dO V^T into TMEM, the softmax warps (one row per thread) form dS in
 //    bf16 over S's columns, and dQ += dS K accumulates in TMEM.
@@ -89,13 +90,15 @@ __device__ __forceinline__ void split_row(int r, int S, int& g, int& i) {
   i = r - g * S;
 }
 
-// D_i = dout_i . out_i (fp32) for every stacked row: one warp per row; row
-// r of group grp (memory row grp R + r) goes to drow[grp R_pad + r].
+// From a saved forward lse (natural log) and the output: lambda (log2 units)
+// and D = dout . out (fp32) of every stacked row, one warp per row; row r of
+// group grp (memory row grp R + r) goes to index grp R_pad + r.
 template <int D>
-__global__ void __launch_bounds__(256) bwd_drow_kernel(const uint16_t* __restrict__ out,
+__global__ void __launch_bounds__(256) bwd_rows_kernel(const uint16_t* __restrict__ out,
                                                       const uint16_t* __restrict__ dout,
-                                                      float* __restrict__ drow, int rows, int R,
-                                                      int R_pad) {
+                                                      const float* __restrict__ lse_saved,
+                                                      float* __restrict__ lam, float* __restrict__ drow,
+                                                      int rows, int R, int R_pad) {
   const int r = blockIdx.x * 8 + static_cast<int>(threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
@@ -118,7 +121,11 @@ __global__ void __launch_bounds__(256) bwd_drow_kernel(const uint16_t* __restric
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if (lane == 0) drow[static_cast<size_t>(r / R) * R_pad + r % R] = s;
+  if (lane == 0) {
+    const size_t i = static_cast<size_t>(r / R) * R_pad + r % R;
+    drow[i] = s;
+    lam[i] = lse_saved[r] * 1.4426950408889634f;
+  }
 }
 
 // K-major 128-byte-swizzled operand descriptors of a 128-row tile (kPanels
@@ -327,7 +334,6 @@ __device__ __forceinline__ void bwd_dq(const BackwardArgs& a, BwdSmem<D>& sm, in
       // key rows (2 KB) and the panels are LBO apart.  Everything but the
       // stage / half offset is formed once, before the first MMA.
       constexpr uint64_t kStage = (2 * G::kTileBytes) >> 4;
-      constexpr uint64_t kPanel = (kBT * 128) >> 4;
       constexpr uint64_t kHalf = (kDqStep * 128) >> 4;
       uint64_t qd[D / 16], od[D / 16], kd0[D / 16], vd0[D / 16];
       kmajor_steps<D>(smem_addr(sm.res[0]), qd);
@@ -799,8 +805,10 @@ __device__ __forceinline__ void bwd_dkv(const BackwardArgs& a, BwdSmem<D>& sm, i
 
 // One launch for both halves of the gradient, a 1-D grid: the first
 // n_row_tiles x groups CTAs form dq (row tile, group), the rest dk / dv (key
-// tile, group).  The dq CTAs, the longest, are dispatched first, and the
-// shorter dk / dv CTAs fill the SMs around them and after them.
+// tile, group), key-tile major.  The dq CTAs, the longest, are dispatched
+// first; the dk / dv CTAs fill the SMs around them and after them, the
+// cache tiles (every row sees them) before the chunk tiles (causal, fewer
+// rows the later the tile).
 template <int D>
 __global__ void __launch_bounds__(kBwdThreads, 1) bwd_kernel(const __grid_constant__ BackwardArgs a,
                                                             int n_row_tiles, int n_key_tiles) {
@@ -813,7 +821,8 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_kernel(const __grid_consta
     bwd_dq<D>(a, sm, x % n_row_tiles, x / n_row_tiles);
   } else {
     const int y = x - n_dq;
-    bwd_dkv<D>(a, sm, y % n_key_tiles, y / n_key_tiles);
+    const int groups = a.B * a.Hkv;
+    bwd_dkv<D>(a, sm, y / groups, y % groups);
   }
   if (threadIdx.x == 0 && sm.abort_flag) atomicOr(a.err, H2O_DEVERR_TIMEOUT);
 }
@@ -821,14 +830,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_kernel(const __grid_consta
 template <int D>
 cudaError_t launch_backward_d(const BackwardArgs& a, cudaStream_t stream) {
   const int R = a.qg * a.S;
-  const int rows = a.B * a.Hq * a.S;
-  bwd_drow_kernel<D><<<(rows + 7) / 8, 256, 0, stream>>>(a.out, a.dout, a.drow, rows, R,
-                                                          backward_row_stride(a.qg, a.S));
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
   const size_t smem = sizeof(BwdSmem<D>) + 1024;
   static OncePerDevice configured;
-  e = configured.run([smem](int) {
+  const cudaError_t e = configured.run([smem](int) {
     return cudaFuncSetAttribute(bwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 static_cast<int>(smem));
   });
@@ -848,6 +852,19 @@ size_t backward_workspace_bytes(int B, int Hq, int Hkv, int S, int M) {
   const int qg = Hkv > 0 ? Hq / Hkv : 0;
   // lambda and D per stacked row, each group's rows padded to 128
   return 2 * static_cast<size_t>(B) * Hkv * backward_row_stride(qg, S) * sizeof(float);
+}
+
+cudaError_t launch_backward_rows(const BackwardArgs& a, const uint16_t* out, const uint16_t* dout,
+                                 const float* lse_saved, cudaStream_t stream) {
+  const int rows = a.B * a.Hq * a.S;
+  const int R = a.qg * a.S;
+  const unsigned grid = static_cast<unsigned>((rows + 7) / 8);
+  const int Rp = backward_row_stride(a.qg, a.S);
+  if (a.d == 64)
+    bwd_rows_kernel<64><<<grid, 256, 0, stream>>>(out, dout, lse_saved, a.lse, a.drow, rows, R, Rp);
+  else
+    bwd_rows_kernel<128><<<grid, 256, 0, stream>>>(out, dout, lse_saved, a.lse, a.drow, rows, R, Rp);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_backward(const BackwardArgs& a, cudaStream_t stream) {

@@ -69,6 +69,15 @@ struct SdpaArgs {
   // recomputation needs it).
   float* lse;
   int lse_stride;
+  // With lse: when drow is non-null, also D = dout . out (fp32) of every
+  // query row, at the same index as its log-sum-exp; out / dout (B, Hq, S, d)
+  // bf16 are the forward output and the loss gradient the backward is given.
+  const uint16_t* bwd_out;
+  const uint16_t* bwd_dout;
+  float* drow;
+  // Full mode: when non-null, each query row's log-sum-exp of the scaled
+  // logits (natural log), (B, Hq, S) fp32, as the forward's own lambda.
+  float* lse_out;
 };
 
 // Row tiles per query head above which the column sums go through colpart.
@@ -209,14 +218,7 @@ struct BackwardArgs {
   // a group {d, q_g S, B Hkv} for q and dout, the keys and values {d, M or S,
   // B Hkv} of the cache and of the chunk
   CUtensorMap tm_q, tm_do, tm_kc, tm_vc, tm_kn, tm_vn;
-  const uint16_t* q;         // (B, Hq, S, d) bf16
-  const uint16_t* k_cache;   // (B, Hkv, M, d)
-  const uint16_t* v_cache;
-  const uint16_t* k_new;     // (B, Hkv, S, d)
-  const uint16_t* v_new;
   const int32_t* slot_pos;   // (B, Hkv, M)
-  const uint16_t* out;       // (B, Hq, S, d) forward output
-  const uint16_t* dout;      // (B, Hq, S, d) gradient of the loss w.r.t. out
   float* dq;                 // (B, Hq, S, d) fp32
   float* dk_cache;           // (B, Hkv, M, d) fp32
   float* dv_cache;
@@ -235,8 +237,12 @@ struct BackwardArgs {
 // every 128-row tile of them starts 16-byte aligned.
 __host__ __device__ inline int backward_row_stride(int qg, int S) { return (qg * S + 127) / 128 * 128; }
 size_t backward_workspace_bytes(int B, int Hq, int Hkv, int S, int M);
-// The forward's pass 1 must have filled a.lse first.
+// The forward's pass 1 must have filled a.lse and a.drow first.
 cudaError_t launch_backward(const BackwardArgs& a, cudaStream_t stream);
+// Fills a.lse (from a saved natural-log lse, (B, Hq, S)) and a.drow (from out
+// and dout) in the backward's padded row layout.
+cudaError_t launch_backward_rows(const BackwardArgs& a, const uint16_t* out, const uint16_t* dout,
+                                 const float* lse_saved, cudaStream_t stream);
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);

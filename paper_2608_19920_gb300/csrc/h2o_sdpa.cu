@@ -623,6 +623,14 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
             l += sm.rowstat[w][r][1] * fast_exp2(sm.rowstat[w][r][0] - mm);
           lam4[x] = (v4[x] && mm > -INFINITY) ? mm + fast_log2(l) : INFINITY;
           nl4[x] = make_float2(-lam4[x], -lam4[x]);
+          // the row's log-sum-exp in natural-log units, for a later backward
+          // (the first warpgroup of a team, one lane of the four per row)
+          if (a.lse_out != nullptr && u == 0 && (lane & 3u) == 0u && v4[x]) {
+            int gg, ii;
+            row_info(r, gg, ii);
+            a.lse_out[static_cast<size_t>(b * a.Hq + hkv * a.qg + gg) * a.S + ii] =
+                lam4[x] * 0.6931471805599453f;
+          }
         }
         have_lambda = true;
       }
@@ -866,13 +874,33 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       if (lane == 0) bar_arrive(&sm.bar_rowstat);
     }
     if (a.lse != nullptr && ok && n_t > 0 && wait_bar(&sm.bar_rowstat, 0, abort_flag, kWaitLimitNs)) {
-      // pass 1 only: the merged log-sum-exp of each row (§A.6.1), one lane
-      // of the four holding a row in the 16x256b layout writes it
+      // pass 1 only: the merged log-sum-exp of each row (§A.6.1) and, for the
+      // backward, D = dout . out.  Warpgroup wg takes rows q4 32 + lane/4 +
+      // 8 wg; the four lanes holding a row (16x256b layout) each take a
+      // quarter of d for D, and the first of them writes both values.
+      const int r = q4 * 32 + static_cast<int>(lane >> 2) + 8 * wg;
+      int gg = 0, ii = 0;
+      const bool has = row_info(r, gg, ii);
+      float dsum = 0.f;
+      if (has && a.drow != nullptr) {
+        const size_t orow = (static_cast<size_t>(b * a.Hq + hkv * a.qg + gg) * a.S + ii) * D +
+                            (lane & 3u) * (D / 4);
+        const uint4* o4 = reinterpret_cast<const uint4*>(a.bwd_out + orow);
+        const uint4* g4 = reinterpret_cast<const uint4*>(a.bwd_dout + orow);
 #pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const int r = q4 * 32 + static_cast<int>(lane >> 2) + 8 * x;
-        int gg, ii;
-        if ((lane & 3u) != 0u || !row_info(r, gg, ii)) continue;
+        for (int k = 0; k < D / 32; ++k) {
+          const uint4 o = __ldg(o4 + k), g = __ldg(g4 + k);
+          const uint32_t ow[4] = {o.x, o.y, o.z, o.w}, gw[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            dsum = fmaf(__uint_as_float(ow[e] << 16), __uint_as_float(gw[e] << 16), dsum);
+            dsum = fmaf(__uint_as_float(ow[e] & 0xFFFF0000u), __uint_as_float(gw[e] & 0xFFFF0000u), dsum);
+          }
+        }
+      }
+      dsum += __shfl_xor_sync(0xffffffffu, dsum, 1);
+      dsum += __shfl_xor_sync(0xffffffffu, dsum, 2);
+      if (has && (lane & 3u) == 0u) {
         float mm = -INFINITY;
 #pragma unroll
         for (int w = 0; w < kNumWG; ++w) mm = fmaxf(mm, sm.rowstat[w][r][0]);
@@ -880,7 +908,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
 #pragma unroll
         for (int w = 0; w < kNumWG; ++w)
           l += sm.rowstat[w][r][1] * fast_exp2(sm.rowstat[w][r][0] - mm);
-        a.lse[static_cast<size_t>(grp) * a.lse_stride + gg * a.S + ii] = mm + fast_log2(l);
+        const size_t li = static_cast<size_t>(grp) * a.lse_stride + gg * a.S + ii;
+        a.lse[li] = mm + fast_log2(l);
+        if (a.drow != nullptr) a.drow[li] = dsum;
       }
     }
     // ------------------------------------------------------------ epilogue --

@@ -220,6 +220,15 @@ def test_backward_argument_checks(lib):
     assert bwd(_dims(d=96), ok) == UNSUP
     # q_g S = 600000 stacked rows: more than 4096 row tiles in a group
     assert bwd(_dims(S=300000), ok, pos0=0) == UNSUP
+    # the saved-lse form: the lse pointer is checked like the others
+    bwl = lambda lse: lib.h2o_sdpa_chunk_backward_lse(ctypes.byref(d), 256, 0.0, *ok[:8], lse,
+                                                      *ok[8:], p, n.value, None)
+    assert bwl(None) == NULL
+    assert bwl(vp(0x1004)) == ALIGN
+    fl = lambda lse: lib.h2o_sdpa_chunk_lse(ctypes.byref(d), 256, 0.0, *[p] * 8, lse, None, 0,
+                                            None)
+    assert fl(None) == NULL
+    assert fl(vp(0x1008)) == ALIGN
 
 
 def test_selftest_limit_is_checked_on_the_host(lib):

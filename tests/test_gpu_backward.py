@@ -14,8 +14,9 @@ import pytest
 import torch
 
 from oracle import sdpa_chunk_backward as ref_backward
+from oracle import sdpa_chunk as ref_sdpa
 from paper_2608_19920_gb300 import (build, h2o_device_errors, h2o_sdpa_chunk,
-                                   h2o_sdpa_chunk_backward)
+                                   h2o_sdpa_chunk_backward, h2o_sdpa_chunk_lse)
 from paper_2608_19920_gb300 import workloads as wl
 
 from test_gpu_parity import bf, f32
@@ -47,8 +48,13 @@ CASES = [
 ]
 
 
+# lse: log-sum-exp of fp32 logits of exact bf16 products (hardware exp2 / log2)
+LSE_ATOL = 2e-3
+
+
+@pytest.mark.parametrize("mode", ["recompute", "saved_lse"])
 @pytest.mark.parametrize("case", CASES, ids=lambda c: "x".join(map(str, c)))
-def test_backward_matches_oracle(dev, case):
+def test_backward_matches_oracle(dev, case, mode):
     B, Hq, Hkv, d, S, M, n_empty, n_future, pos0 = case
     rng = np.random.default_rng(hash(case) % 2**32)
     st = wl.random_state(rng, B, Hkv, M, d, pos0=pos0, n_empty=n_empty)
@@ -63,9 +69,13 @@ def test_backward_matches_oracle(dev, case):
     dout = wl.round_bf16(rng.standard_normal((B, Hq, S, d), dtype=np.float32))
     g = dict(q=bf(q, dev), kc=bf(st["k_cache"], dev), vc=bf(st["v_cache"], dev), kn=bf(kn, dev),
              vn=bf(vn, dev), sp=torch.from_numpy(st["slot_pos"]).to(dev))
-    out, _ = h2o_sdpa_chunk(g["q"], g["kc"], g["vc"], g["kn"], g["vn"], g["sp"], pos0)
+    lse = None
+    if mode == "recompute":
+        out, _ = h2o_sdpa_chunk(g["q"], g["kc"], g["vc"], g["kn"], g["vn"], g["sp"], pos0)
+    else:
+        out, _, lse = h2o_sdpa_chunk_lse(g["q"], g["kc"], g["vc"], g["kn"], g["vn"], g["sp"], pos0)
     grads = h2o_sdpa_chunk_backward(g["q"], g["kc"], g["vc"], g["kn"], g["vn"], g["sp"], pos0, out,
-                                    bf(dout, dev))
+                                    bf(dout, dev), lse=lse)
     torch.cuda.synchronize()
     assert h2o_device_errors() == 0
     refs = ref_backward(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"], pos0, dout)
@@ -98,3 +108,28 @@ def test_backward_is_deterministic(dev):
     assert h2o_device_errors() == 0
     for a, b in zip(g1, g2):
         assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: "x".join(map(str, c)))
+def test_forward_lse_matches_oracle(dev, case):
+    """h2o_sdpa_chunk_lse: the same out and score_inc as h2o_sdpa_chunk (the
+    same kernel when S > 1), and each row's log-sum-exp within LSE_ATOL of the
+    oracle's (every row sees at least its own token, so lse is finite)."""
+    B, Hq, Hkv, d, S, M, n_empty, n_future, pos0 = case
+    rng = np.random.default_rng(hash(case) % 2**32 + 1)
+    st = wl.random_state(rng, B, Hkv, M, d, pos0=pos0, n_empty=n_empty)
+    q = wl.round_bf16(rng.standard_normal((B, Hq, S, d), dtype=np.float32))
+    kn = wl.round_bf16(rng.standard_normal((B, Hkv, S, d), dtype=np.float32))
+    vn = wl.round_bf16(rng.standard_normal((B, Hkv, S, d), dtype=np.float32))
+    args = (bf(q, dev), bf(st["k_cache"], dev), bf(st["v_cache"], dev), bf(kn, dev), bf(vn, dev),
+            torch.from_numpy(st["slot_pos"]).to(dev), pos0)
+    out, inc, lse = h2o_sdpa_chunk_lse(*args)
+    torch.cuda.synchronize()
+    assert h2o_device_errors() == 0
+    if S > 1:
+        out0, inc0 = h2o_sdpa_chunk(*args)
+        torch.cuda.synchronize()
+        assert torch.equal(out, out0) and torch.equal(inc, inc0)
+    _, _, lse_ref = ref_sdpa(q, st["k_cache"], st["v_cache"], kn, vn, st["slot_pos"], pos0)
+    err = np.abs(lse.cpu().numpy().astype(np.float64) - lse_ref).max()
+    assert err <= LSE_ATOL, f"lse max abs err {err:.3e}"

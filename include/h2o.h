@@ -156,7 +156,7 @@ H2O_API int h2o_sdpa_chunk_lse(const h2o_dims_t* dims, int64_t pos0, float softm
  * allocate device memory around the call.
  *
  * Its scratch (the per-split partial max, sum and output of every query head,
- * h2o_workspace_size(dims) bytes) is a fixed device array of 8 MiB inside the
+ * h2o_workspace_size(dims) bytes) is a fixed device array of 16 MiB inside the
  * library, one per device; dims needing more are rejected with
  * H2O_ERR_WORKSPACE and nothing runs.  Other sizes outside the decode case
  * give H2O_ERR_UNSUPPORTED.  Arguments, outputs and the other errors are

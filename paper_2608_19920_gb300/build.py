@@ -19,7 +19,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libh2o_gb300.so")
 SOURCES = ["h2o_api.cu", "h2o_sdpa.cu", "h2o_decode.cu", "h2o_update.cu", "h2o_replay.cu",
-           "h2o_quant.cu", "h2o_backward.cu"]
+           "h2o_quant.cu", "h2o_backward.cu", "h2o_decode_tc.cu"]
 HEADERS = ["h2o_internal.h", "sm100.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden",

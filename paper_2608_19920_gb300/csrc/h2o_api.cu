@@ -102,6 +102,25 @@ int encode(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, con
   return res == CUDA_SUCCESS ? H2O_OK : H2O_ERR_SHAPE;
 }
 
+// The tensor-core decode kernel's TMA maps (d = 128, bf16 cache buffers);
+// otherwise a.tc stays 0 and the CUDA-core split kernel runs.
+int decode_maps(DecodeArgs& a) {
+  a.tc = 0;
+  if (a.d != 128 || a.q8) return H2O_OK;
+  int st = get_encoder();
+  if (st != H2O_OK) return st;
+  const uint64_t G = static_cast<uint64_t>(a.B) * a.Hkv;
+  const uint64_t dq[3] = {128, static_cast<uint64_t>(a.Hq), static_cast<uint64_t>(a.B)};
+  const uint32_t bq[3] = {64, 16, 1};
+  const uint64_t dc[3] = {128, static_cast<uint64_t>(a.M), G};
+  const uint32_t bc[3] = {64, static_cast<uint32_t>(kDecodeTcTileKeys), 1};
+  if ((st = encode(&a.tm_q, a.q, 3, dq, bq)) != H2O_OK) return st;
+  if ((st = encode(&a.tm_kc, a.k_cache, 3, dc, bc)) != H2O_OK) return st;
+  if ((st = encode(&a.tm_vc, a.v_cache, 3, dc, bc)) != H2O_OK) return st;
+  a.tc = 1;
+  return H2O_OK;
+}
+
 int check_dims(const h2o_dims_t* d) {
   if (!d) return H2O_ERR_NULL;
   if (d->B < 1 || d->Hq < 1 || d->Hkv < 1 || d->S < 1 || d->M < 0 || d->d < 1) return H2O_ERR_SHAPE;
@@ -186,6 +205,7 @@ int sdpa_impl(const h2o_dims_t* dims, int64_t pos0, float softmax_scale, const h
     a.k_scales = q8 ? q8->k_scales : nullptr;
     a.v_codes = q8 ? q8->v_codes : nullptr;
     a.v_scales = q8 ? q8->v_scales : nullptr;
+    if ((st = decode_maps(a)) != H2O_OK) return st;
     const cudaError_t e = launch_decode(a, s);
     return e == cudaSuccess ? H2O_OK : cuda_fail(e);
   }
@@ -508,6 +528,7 @@ int h2o_sdpa_decode_static(const h2o_dims_t* dims, int64_t pos0, float softmax_s
   a.n_split = n_split;
   a.with_new = 1;
   a.nk = D.M + 1;
+  if ((st = decode_maps(a)) != H2O_OK) return st;
   e = launch_decode(a, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? H2O_OK : cuda_fail(e);
 }

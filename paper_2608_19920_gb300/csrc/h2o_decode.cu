@@ -202,6 +202,7 @@ __global__ void __launch_bounds__(kDecThreads, QG == 4 ? 2 : 1)
   const int tid = threadIdx.x, warp = tid >> 5;
   const uint32_t lane = static_cast<uint32_t>(tid & 31);
   const int n_items = a.n_split * a.B * a.Hkv;
+  if (tid == 0) launch_dependents();  // the combine may be placed (it waits for this grid)
 
   if (tid == 0) {
 #pragma unroll
@@ -560,12 +561,28 @@ __device__ __forceinline__ float block_sum(float v, float* sh) {
   return r;
 }
 
+// Per (b, hq) row and block of score_inc columns: merge the splits'
+// partials into lambda (and, in the first column block, out), then rewrite
+// the block's logits as weights.  The block's logits are loaded first, so
+// that their round trip overlaps the merge.
 template <int D>
 __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const DecodeArgs a) {
   extern __shared__ float fac[];  // [max(n_split, threads)]: exp2(m_s - m) per split
   __shared__ float sh[kCombineThreads / 32];
+  grid_dependency_wait();  // the split kernel's partials and logits
   const int tid = threadIdx.x;
   const size_t row = blockIdx.x;  // b * Hq + hq
+  float* inc = a.score_inc + row * static_cast<size_t>(a.nk);
+  const int per = (a.nk + static_cast<int>(gridDim.y) - 1) / static_cast<int>(gridDim.y);
+  const int c0 = static_cast<int>(blockIdx.y) * per;
+  const int c1 = min(c0 + per, a.nk);
+  constexpr int kPer = kCombineCols / kCombineThreads;  // per <= kCombineCols
+  float lg[kPer];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int j = c0 + tid + k * kCombineThreads;
+    lg[k] = j < c1 ? inc[j] : 0.f;
+  }
   const float* part = a.part + row * a.n_split * (2 + D);
   float m = -INFINITY;
   for (int s = tid; s < a.n_split; s += kCombineThreads) m = fmaxf(m, part[s * (2 + D)]);
@@ -580,6 +597,11 @@ __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const D
   l = block_sum(l, sh);  // (its barriers also publish fac)
   // every row sees its own token, so m is finite and l >= 1
   const float lam = m + fast_log2(l);
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int j = c0 + tid + k * kCombineThreads;
+    if (j < c1) inc[j] = fast_exp2(lg[k] - lam);
+  }
   if (blockIdx.y == 0) {
     const float inv = 1.0f / l;
     // thread (dd, q): output element dd, splits q, q + 2, ... (two halves)
@@ -603,11 +625,6 @@ __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const D
       a.out[row * D + dd] = static_cast<uint16_t>(pack_bf16x2(t * inv, 0.f) & 0xFFFFu);
     }
   }
-  float* inc = a.score_inc + row * static_cast<size_t>(a.nk);
-  const int c0 = static_cast<int>(blockIdx.y) * kCombineCols;
-  const int c1 = min(c0 + kCombineCols, a.nk);
-#pragma unroll 4
-  for (int j = c0 + tid; j < c1; j += kCombineThreads) inc[j] = fast_exp2(inc[j] - lam);
 }
 
 template <int D, int QG, bool Q8>
@@ -653,16 +670,28 @@ cudaError_t launch_split(const DecodeArgs& a, cudaStream_t stream) {
 template <int D>
 cudaError_t launch_d(const DecodeArgs& a, cudaStream_t stream) {
   cudaError_t e;
-  if (a.q8)
+  if (a.tc)
+    e = launch_decode_tc(a, stream);
+  else if (a.q8)
     e = a.qg <= 4 ? launch_split<D, 4, true>(a, stream) : launch_split<D, 8, true>(a, stream);
   else
     e = a.qg <= 4 ? launch_split<D, 4, false>(a, stream) : launch_split<D, 8, false>(a, stream);
   if (e != cudaSuccess) return e;
-  const dim3 grid(static_cast<unsigned>(a.B * a.Hq),
-                  static_cast<unsigned>((a.nk + kCombineCols - 1) / kCombineCols));
-  const size_t smem = static_cast<size_t>(std::max(a.n_split, kCombineThreads)) * sizeof(float);
-  decode_combine_kernel<D><<<grid, kCombineThreads, smem, stream>>>(a);
-  return cudaGetLastError();
+  // launched as a programmatic dependent of the split kernel: its CTAs are
+  // placed while the split kernel's last CTAs run and wait for its results
+  // in grid_dependency_wait
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(a.B * a.Hq),
+                     static_cast<unsigned>((a.nk + kCombineCols - 1) / kCombineCols));
+  cfg.blockDim = dim3(kCombineThreads);
+  cfg.dynamicSmemBytes = static_cast<size_t>(std::max(a.n_split, kCombineThreads)) * sizeof(float);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_combine_kernel<D>, a);
 }
 
 }  // namespace
@@ -671,15 +700,23 @@ bool decode_plan(int B, int Hq, int Hkv, int d, int S, int M, int* split_len, in
                  size_t* ws_bytes) {
   if (S != 1 || M < 1 || Hq / Hkv > kDecodeMaxQg) return false;
   // Work items are (b, kv head, split); the persistent split kernel deals them
-  // round-robin to kDecodeResidentCtas CTAs, so a step costs about
-  // ceil(items / CTAs) items of (split_len + per-item overhead) keys.  Take
-  // the split length (a multiple of 16 in [128, 1536]) that minimises that.
+  // round-robin to its resident CTAs, so a step costs about ceil(items / CTAs)
+  // items of (split_len + per-item overhead) keys.  Take the split length in
+  // [128, 1536] that minimises that: a multiple of the tensor-core kernel's
+  // 128-key tiles for d = 128 (one CTA per SM), of 16 otherwise (two CTAs per
+  // SM).  A function of the sizes only, so that h2o_workspace_size and the
+  // calls agree whichever kernel runs.
   const int64_t groups = static_cast<int64_t>(B) * Hkv;
-  int64_t best_len = kDecodeMaxSplitLen, best_cost = INT64_MAX;
-  for (int64_t len = kDecodeMinSplitLen; len <= kDecodeMaxSplitLen; len += 16) {
+  const int64_t gran = d == 128 ? kDecodeTcTileKeys : 16;
+  const int64_t ctas = d == 128 ? kDecodeTcCtas : kDecodeResidentCtas;
+  const int64_t max_len = d == 128 ? kDecodeTcMaxSplitLen : kDecodeMaxSplitLen;
+  const int64_t min_len = d == 128 ? kDecodeTcMinSplitLen : kDecodeMinSplitLen;
+  int64_t best_len = max_len, best_cost = INT64_MAX;
+  for (int64_t len = min_len; len <= max_len; len += gran) {
     const int64_t n = (M + len - 1) / len;
-    const int64_t rounds = (groups * n + kDecodeResidentCtas - 1) / kDecodeResidentCtas;
-    const int64_t cost = rounds * (std::min<int64_t>(len, M) + kDecodeItemOverheadKeys);
+    const int64_t rounds = (groups * n + ctas - 1) / ctas;
+    const int64_t cost = rounds * (std::min<int64_t>(len, M) +
+                                   (d == 128 ? kDecodeTcItemOverheadKeys : kDecodeItemOverheadKeys));
     if (cost < best_cost) {
       best_cost = cost;
       best_len = len;

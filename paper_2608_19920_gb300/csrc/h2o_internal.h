@@ -121,9 +121,22 @@ constexpr int kDecodeMaxQg = 8;         // larger GQA groups take the chunk kern
 constexpr int kDecodeMaxSplitLen = 1536;
 constexpr int kDecodeMinSplitLen = 128;
 constexpr int kDecodeResidentCtas = 304;     // split-kernel CTAs resident on a GB300 (2 x 152)
+constexpr int kDecodeTcCtas = 152;           // tensor-core split kernel: one CTA per GB300 SM
+constexpr int kDecodeTcTileKeys = 128;       // its K / V tiles (split lengths are multiples)
+// its per-item cost, in keys of streaming (the items of a CTA overlap, K
+// tiles of one with V tiles of the previous)
+constexpr int kDecodeTcItemOverheadKeys = 16;
+constexpr int kDecodeTcMaxSplitLen = 1024;   // its largest split (two items' logits in shared memory)
+// and its smallest: the end of a phase costs ~1400 cycles that a phase of
+// fewer than four tiles per stream no longer hides (measured)
+constexpr int kDecodeTcMinSplitLen = 512;
 constexpr int kDecodeItemOverheadKeys = 32;  // per-item cost, in keys, for choosing the split
 
 struct DecodeArgs {
+  // tensor-core path (d = 128, bf16 buffers): TMA maps of q {d, Hq, B} with
+  // box {64, 16, 1} and of the cache K / V {d, M, B*Hkv} with box {64, 128, 1}
+  CUtensorMap tm_q, tm_kc, tm_vc;
+  int tc;                   // 1: decode_tc_kernel (maps valid); 0: decode_split_kernel
   const uint16_t* q;        // (B, Hq, 1, d)
   const uint16_t* k_cache;  // (B, Hkv, M, d)
   const uint16_t* v_cache;
@@ -159,7 +172,7 @@ bool decode_plan(int B, int Hq, int Hkv, int d, int S, int M, int* split_len, in
 // Fixed scratch of h2o_sdpa_decode_static (a file-scope device array in
 // h2o_decode.cu, shared by every call on a device): its size and its address
 // on the current device.
-constexpr size_t kDecodeStaticScratchBytes = size_t(8) << 20;
+constexpr size_t kDecodeStaticScratchBytes = size_t(16) << 20;
 cudaError_t decode_static_scratch(void** ptr);
 
 // h2o_kv_replace / h2o_kv_restore (h2o_replay.cu)
@@ -245,6 +258,9 @@ cudaError_t launch_backward_rows(const BackwardArgs& a, const uint16_t* out, con
                                  const float* lse_saved, cudaStream_t stream);
 cudaError_t launch_sdpa(const SdpaArgs& a, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
+// The tensor-core split kernel (h2o_decode_tc.cu): same partials as
+// decode_split_kernel; launch_decode runs the combine after it.
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t stream);
 cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream);
 cudaError_t launch_scores_add(const ScoresAddArgs& a, cudaStream_t stream);
 

@@ -71,10 +71,11 @@ def test_decode_workspace(lib):
     n = ctypes.c_size_t(0)
     dims = _dims(B=8, Hq=32, Hkv=8, d=128, S=1, M=65536)
     assert lib.h2o_workspace_size(ctypes.byref(dims), ctypes.byref(n)) == OK
-    # 64 (b, kv head) groups x 65536 slots in about 3648 work items -> splits of
-    # 1152 slots (a multiple of 16), 57 per group
-    assert n.value == 8 * 32 * 57 * (2 + 128) * 4
-    assert n.value <= 8 << 20  # fits the fixed scratch of h2o_sdpa_decode_static
+    # 64 (b, kv head) groups x 65536 slots: splits of 1024 slots (a multiple of
+    # the 128-key tiles of the d = 128 kernel, at most 1024), 64 per group,
+    # 4096 work items in 27 rounds over 152 CTAs
+    assert n.value == 8 * 32 * 64 * (2 + 128) * 4
+    assert n.value <= 16 << 20  # fits the fixed scratch of h2o_sdpa_decode_static
     small = _dims(B=1, Hq=4, Hkv=2, d=64, S=1, M=100)
     assert lib.h2o_workspace_size(ctypes.byref(small), ctypes.byref(n)) == OK
     assert n.value == 1 * 4 * 1 * (2 + 64) * 4

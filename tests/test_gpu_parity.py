@@ -147,6 +147,8 @@ DECODE_CASES = [
     (1, 8, 2, 64, 3000, 0, 0, 5000, (256, 768)), # d = 64; whole splits see no key
     (1, 32, 2, 64, 200, 0, 0, 300, None),        # q_g = 16: the chunk kernel takes S = 1
     (8, 32, 8, 128, 4096, 0, 0, 4200, None),     # the decode workload's shape, M = 4096
+    (1, 8, 2, 128, 2500, 10, 5, 3000, (300, 700)),  # several splits, ragged last tile, empty block
+    (1, 16, 2, 128, 1700, 0, 9, 1800, None),     # q_g = 8 over several splits
 ]
 
 

@@ -49,6 +49,13 @@
  *  - Calls only enqueue work on `stream` (a cudaStream_t; NULL = legacy
  *    default stream) and return without synchronising.  Arguments are
  *    validated on the host first; on any error nothing is enqueued.
+ *  - Stream order holds as usual, with one refinement: the update kernels,
+ *    and the reduction and combine steps of the attention calls, are
+ *    launched as programmatic dependents of the kernel before them.  If that
+ *    kernel allows an early start (only this library's attention kernels
+ *    do), they may begin while it finishes, reading before its completion
+ *    only what it does not write (scores, slot_pos, k_new, v_new), and
+ *    everything else after it has completed.
  *  - Return value: H2O_OK (0) or a negative H2O_ERR_* code; h2o_status_string
  *    gives a message.  For H2O_ERR_CUDA, h2o_last_cuda_error() gives the
  *    cudaError_t of the failing runtime call on this host thread.

@@ -569,7 +569,8 @@ template <int D>
 __global__ void __launch_bounds__(kCombineThreads) decode_combine_kernel(const DecodeArgs a) {
   extern __shared__ float fac[];  // [max(n_split, threads)]: exp2(m_s - m) per split
   __shared__ float sh[kCombineThreads / 32];
-  grid_dependency_wait();  // the split kernel's partials and logits
+  if (threadIdx.x == 0) launch_dependents();  // the S = 1 update may be placed now
+  grid_dependency_wait();                      // the split kernel's partials and logits
   const int tid = threadIdx.x;
   const size_t row = blockIdx.x;  // b * Hq + hq
   float* inc = a.score_inc + row * static_cast<size_t>(a.nk);

@@ -213,6 +213,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
   const bool peer_rows = kPair && row_range(a, rt ^ 1, pg, p_lo, p_hi);
   // rows the Q box covers (the rest of the tile is zero-filled here)
   const int box_rows = a.tiles_per_head > 0 ? kTileM : a.rows_box * a.heads_box;
+  // the kernels after it on the stream (column-sum reduction, update) may be
+  // placed now; they wait for this grid before reading what it writes
+  if (tid == 0) launch_dependents();
 
   if (tid == 0) {
     bar_init(&sm.bar_q, 1);
@@ -992,6 +995,8 @@ constexpr int kReduceThreads = 256;
 // (all loads issued before the adds).
 __global__ void __launch_bounds__(kReduceThreads) colsum_reduce_kernel(
     const float* __restrict__ part, float* __restrict__ score_inc, int rows, int tph, int nk) {
+  if (threadIdx.x == 0) launch_dependents();  // the update may be placed now
+  grid_dependency_wait();                      // the attention kernel's partials
   const int col = blockIdx.x * kReduceThreads + static_cast<int>(threadIdx.x);
   if (col >= nk) return;
   for (int row = blockIdx.y; row < rows; row += gridDim.y) {
@@ -1022,8 +1027,16 @@ cudaError_t launch_colsum_reduce(const float* colpart, float* score_inc, int row
                                  cudaStream_t stream) {
   const dim3 grid(static_cast<unsigned>((nk + kReduceThreads - 1) / kReduceThreads),
                   static_cast<unsigned>(rows < 65535 ? rows : 65535));
-  colsum_reduce_kernel<<<grid, kReduceThreads, 0, stream>>>(colpart, score_inc, rows, tph, nk);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kReduceThreads);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, colsum_reduce_kernel, colpart, score_inc, rows, tph, nk);
 }
 
 }  // namespace h2o

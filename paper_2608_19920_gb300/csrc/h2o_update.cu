@@ -129,6 +129,7 @@ __device__ __forceinline__ void copy_row(const UpdateArgs& a, int grp, int c, in
 }
 
 __global__ void __launch_bounds__(kUpdThreads, 1) update_kernel(const UpdateArgs a) {
+  grid_dependency_wait();  // (a no-op unless launched as a programmatic dependent)
   __shared__ UpdSmem sm;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // one (b, h) per CTA; h2o_orig: one KV head per CTA, for every b
@@ -341,6 +342,17 @@ __global__ void __launch_bounds__(kCThreads, 1) update_cluster_kernel(const Upda
   // so each thread's run of slots lies in one share.)
   const int share = ((M + C - 1) / C + R - 1) / R * R;
   const int lo = min(M, rank * share), hi = min(M, lo + share);
+  // Launched as a programmatic dependent of the attention kernels before it
+  // on the stream, this kernel can start while they finish: what it reads
+  // besides score_inc (scores, positions, the chunk's rows above) they do not
+  // write, so it is pulled toward L2 first; then wait for them (score_inc,
+  // and the cache rows they read, which phase 5 overwrites).
+  for (int bi = 0; bi < nb; ++bi)
+    for (int x = lo + tid * 32; x < hi; x += kCThreads * 32) {
+      prefetch_l2(scores_of(b0 + bi) + x);
+      prefetch_l2(pos_of(b0 + bi) + x);
+    }
+  grid_dependency_wait();
   {
     const int* sp = pos_of(b0);
     uint32_t key_dst[8];
@@ -626,6 +638,7 @@ constexpr size_t kDStashBytes = 96 * 1024;
 
 __global__ void __launch_bounds__(kDThreads, 2)
     update_decode_kernel(const UpdateArgs a, int C, int stash_ok) {
+  grid_dependency_wait();  // score_inc of the attention kernels before it
   extern __shared__ float stash[];  // [nb][per] when stash_ok
   __shared__ unsigned long long wmin[kDThreads / 32];
   __shared__ unsigned long long cmin[8];
@@ -809,13 +822,15 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
     cfg.blockDim = dim3(kDThreads);
     cfg.dynamicSmemBytes = stash_ok ? stash : 0;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = static_cast<unsigned>(C);
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, update_decode_kernel, a, C, stash_ok);
   }
   if (!smem_path) {
@@ -843,13 +858,15 @@ cudaError_t launch_update(const UpdateArgs& a, cudaStream_t stream) {
   cfg.blockDim = dim3(kCThreads);
   cfg.dynamicSmemBytes = prefetch ? rows_off + rows_bytes : smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(C);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, update_cluster_kernel, a, C, prefetch);
 }
 

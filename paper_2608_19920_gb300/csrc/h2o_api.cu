@@ -83,11 +83,12 @@ int get_encoder() {
 
 bool misaligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
 
-// bf16 tensor map, 128-byte swizzle, dims/box innermost first.
-int encode(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint32_t* box) {
+// Dense tensor map, dims/box innermost first, elements of `esize` bytes.
+int encode_any(CUtensorMap* m, CUtensorMapDataType type, int esize, CUtensorMapSwizzle swizzle,
+               const void* base, int rank, const uint64_t* dims, const uint32_t* box) {
   cuuint64_t gd[5], gs[4];
   cuuint32_t bx[5], es[5];
-  uint64_t stride = 2;
+  uint64_t stride = static_cast<uint64_t>(esize);
   for (int r = 0; r < rank; ++r) {
     gd[r] = dims[r];
     bx[r] = box[r];
@@ -95,28 +96,58 @@ int encode(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, con
     if (r > 0) gs[r - 1] = stride;
     stride *= dims[r];
   }
-  const CUresult res = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base),
-                                gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  const CUresult res = g_encode(m, type, rank, const_cast<void*>(base), gd, gs, bx, es,
+                                CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return res == CUDA_SUCCESS ? H2O_OK : H2O_ERR_SHAPE;
 }
 
-// The tensor-core decode kernel's TMA maps (d = 128, bf16 cache buffers);
-// otherwise a.tc stays 0 and the CUDA-core split kernel runs.
+// bf16 tensor map, 128-byte swizzle, dims/box innermost first.
+int encode(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint32_t* box) {
+  return encode_any(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, CU_TENSOR_MAP_SWIZZLE_128B, base, rank,
+                    dims, box);
+}
+
+// The tensor-core decode kernel's TMA maps (d = 128): bf16 cache rows, or
+// with 8-bit buffers the code rows (128 bytes, no swizzle) and the row
+// scales (one flat fp32 array; a 128-scale tile starts 16-byte aligned only
+// when M is a multiple of 4, else the CUDA-core kernel runs).  Otherwise a.tc
+// stays 0 and the CUDA-core split kernel runs.
 int decode_maps(DecodeArgs& a) {
   a.tc = 0;
-  if (a.d != 128 || a.q8) return H2O_OK;
+  if (a.d != 128) return H2O_OK;
+  if (a.q8 && (a.M % 4 != 0 || static_cast<int64_t>(a.B) * a.Hkv * a.M >= (int64_t(1) << 31)))
+    return H2O_OK;
   int st = get_encoder();
   if (st != H2O_OK) return st;
   const uint64_t G = static_cast<uint64_t>(a.B) * a.Hkv;
   const uint64_t dq[3] = {128, static_cast<uint64_t>(a.Hq), static_cast<uint64_t>(a.B)};
   const uint32_t bq[3] = {64, 16, 1};
-  const uint64_t dc[3] = {128, static_cast<uint64_t>(a.M), G};
-  const uint32_t bc[3] = {64, static_cast<uint32_t>(kDecodeTcTileKeys), 1};
   if ((st = encode(&a.tm_q, a.q, 3, dq, bq)) != H2O_OK) return st;
-  if ((st = encode(&a.tm_kc, a.k_cache, 3, dc, bc)) != H2O_OK) return st;
-  if ((st = encode(&a.tm_vc, a.v_cache, 3, dc, bc)) != H2O_OK) return st;
+  if (!a.q8) {
+    const uint64_t dc[3] = {128, static_cast<uint64_t>(a.M), G};
+    const uint32_t bc[3] = {64, static_cast<uint32_t>(kDecodeTcTileKeys), 1};
+    if ((st = encode(&a.tm_kc, a.k_cache, 3, dc, bc)) != H2O_OK) return st;
+    if ((st = encode(&a.tm_vc, a.v_cache, 3, dc, bc)) != H2O_OK) return st;
+  } else {
+    const uint64_t dc[3] = {128, static_cast<uint64_t>(a.M), G};
+    const uint32_t bc[3] = {128, static_cast<uint32_t>(kDecodeTcTileKeys), 1};
+    const uint64_t ds[1] = {G * static_cast<uint64_t>(a.M)};
+    const uint32_t bs[1] = {static_cast<uint32_t>(kDecodeTcTileKeys)};
+    if ((st = encode_any(&a.tm_kc, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, CU_TENSOR_MAP_SWIZZLE_NONE,
+                         a.k_codes, 3, dc, bc)) != H2O_OK)
+      return st;
+    if ((st = encode_any(&a.tm_vc, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, CU_TENSOR_MAP_SWIZZLE_NONE,
+                         a.v_codes, 3, dc, bc)) != H2O_OK)
+      return st;
+    if ((st = encode_any(&a.tm_ks, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, CU_TENSOR_MAP_SWIZZLE_NONE,
+                         a.k_scales, 1, ds, bs)) != H2O_OK)
+      return st;
+    if ((st = encode_any(&a.tm_vs, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, CU_TENSOR_MAP_SWIZZLE_NONE,
+                         a.v_scales, 1, ds, bs)) != H2O_OK)
+      return st;
+  }
   a.tc = 1;
   return H2O_OK;
 }

@@ -30,6 +30,7 @@
 // H2O_DEVERR_TIMEOUT.
 #include <climits>
 #include <cmath>
+#include <cstddef>
 
 #include "h2o_internal.h"
 #include "sm100.cuh"
@@ -37,9 +38,23 @@
 namespace h2o {
 namespace {
 
-constexpr int kTcThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 keys
 constexpr int kTcKeyWarps = 4;
-constexpr int kTcStages = 4;
+// 8-bit buffers: warps turning code tiles into bf16 tiles (~17 instructions
+// per four codes: eight warps keep up with the code stream, four did not)
+constexpr int kTcConvWarps = 8;
+// warp 0 TMA, warp 1 MMA, warps 2-5 keys, with 8-bit buffers warps 6-13 convert
+template <bool Q8>
+constexpr int tc_threads() { return 32 * (2 + kTcKeyWarps + (Q8 ? kTcConvWarps : 0)); }
+// bf16 tile ring (with 8-bit buffers the code ring in front of it streams)
+template <bool Q8, int QG>
+constexpr int tc_stages() { return Q8 ? 2 : 4; }
+// code ring: the bytes it keeps in flight set the stream's rate (a code tile
+// arrived 5-6 k cycles after its TMA was issued under the full stream, so
+// four 16 KB stages held it to ~22 GB/s per SM); six fit beside q_g <= 4's
+// smaller logit buffers
+template <int QG>
+constexpr int tc_code_stages() { return QG <= 4 ? 6 : 4; }
+constexpr int kTcCodeBytes = 128 * 128;      // a tile of 128 code rows
 constexpr int kTcKeys = kDecodeTcTileKeys;   // 128 keys per tile
 constexpr int kTcD = 128;
 constexpr int kTcPanel = kTcKeys * 128;      // one 64-column panel of a tile: 16 KB
@@ -52,22 +67,45 @@ constexpr int kTcMaxItemTiles = kTcMaxItemKeys / kDecodeTcTileKeys;
 constexpr uint32_t kTcTmemCols = 64;
 constexpr uint32_t kTcO = 32;
 
-template <int QG>
+// 8-bit buffers: the code tiles and their row scales, as loaded
+template <bool Q8, int CS>
+struct TcCodeRing {};
+template <int CS>
+struct TcCodeRing<true, CS> {
+  alignas(1024) uint8_t codes[CS][kTcCodeBytes];
+  float scl[CS][kTcKeys];
+  uint64_t cfull[CS], cempty[CS];
+};
+
+template <int QG, bool Q8>
 struct __align__(1024) TcSmem {
-  uint8_t ring[kTcStages][kTcTileBytes];  // K or V tiles, 2 panels of 128 rows
-  uint8_t q[2][2][kTcSmallPanel];         // per item parity: q rows, 2 panels of 16 rows
-  uint8_t p[2][2][kTcSmallPanel];         // P^T of a tile (double buffer), 2 panels of 64 keys
+  uint8_t ring[tc_stages<Q8, QG>()][kTcTileBytes];  // bf16 K or V tiles, 2 panels of 128 rows
+  TcCodeRing<Q8, tc_code_stages<QG>()> cr;
+  // (128-byte-swizzled operands: 1024-byte aligned swizzle atoms)
+  alignas(1024) uint8_t q[2][2][kTcSmallPanel];  // per item parity: q rows, 2 panels of 16 rows
+  alignas(1024) uint8_t p[2][2][kTcSmallPanel];  // P^T of a tile (double buffer), 2 panels of 64 keys
   float lg[2][kTcMaxItemKeys * QG];       // per item parity: its logits (log2 units), key-major
   int32_t pos[2][kTcMaxItemKeys];         // per item parity: its slots' positions
   float red[2][kTcKeyWarps][QG];          // per phase parity: per-warp maxima
   float red2[2][kTcKeyWarps][QG];         // per phase parity: per-warp sums
   float newlg[2][QG];                     // per item parity: the new token's logits
-  uint64_t full[kTcStages], empty[kTcStages];
+  uint64_t full[tc_stages<Q8, QG>()], empty[tc_stages<Q8, QG>()];
   uint64_t qfull[2], qempty[2], sfull[2], sfree[2], pfull[2], pempty[2];
   uint64_t ofull, oempty, ksync, drain;
   uint32_t taddr;
   int abort_flag;
 };
+
+// swizzled operands start on 1024-byte boundaries, TMA tiles at least 128
+template <int QG, bool Q8>
+constexpr bool tc_layout_ok() {
+  using T = TcSmem<QG, Q8>;
+  return offsetof(T, ring) % 1024 == 0 && offsetof(T, q) % 1024 == 0 &&
+         offsetof(T, p) % 1024 == 0 && offsetof(T, cr) % 1024 == 0;
+}
+static_assert(tc_layout_ok<4, false>() && tc_layout_ok<8, false>() && tc_layout_ok<4, true>() &&
+                  tc_layout_ok<8, true>(),
+              "decode_tc_kernel shared-memory layout");
 
 __device__ __forceinline__ bool twait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   return wait_bar(bar, parity, abort, kWaitLimitNs);
@@ -96,6 +134,20 @@ __device__ __forceinline__ TcItem tc_item(const DecodeArgs& a, int it) {
   return x;
 }
 
+// Two 8-bit codes of a cache row read back as the 8-bit format defines,
+// bf16(code * scale), packed (element i in the low half).  `wb` holds four
+// codes with their sign bits flipped (code + 128 as unsigned bytes); byte i
+// placed under the exponent of 2^23 gives the float 2^23 + 128 + code
+// exactly, and subtracting 2^23 + 128 leaves the code; then an fp32
+// multiply and round-to-nearest-even to bf16, as in the read-back kernel.
+__device__ __forceinline__ uint32_t q8_bf16x2(uint32_t wb, int i, float s) {
+  const float lo = __uint_as_float(__byte_perm(wb, 0x4B000000u, 0x7650u | i));
+  const float hi = __uint_as_float(__byte_perm(wb, 0x4B000000u, 0x7650u | (i + 1)));
+  const float2 c = __fadd2_rn(make_float2(lo, hi), make_float2(-8388736.f, -8388736.f));
+  const float2 x = __fmul2_rn(c, make_float2(s, s));
+  return pack_bf16x2(x.x, x.y);
+}
+
 // K-major SW128 descriptors of the eight K-steps (16 of d each) of an
 // operand of 64-column panels `panel` bytes apart.
 __device__ __forceinline__ void kmajor8(uint32_t base, uint32_t panel, uint64_t (&d)[8]) {
@@ -113,11 +165,13 @@ __device__ __forceinline__ void kmajor8(uint32_t base, uint32_t panel, uint64_t 
 // warps completes item ph's maximum and item ph - 1's sum, then item ph - 1's
 // output is read out.  So the K and V streams of consecutive items overlap
 // and no item waits for its own maximum with an idle ring.
-template <int QG>
-__global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_constant__ DecodeArgs a) {
+template <int QG, bool Q8>
+__global__ void __launch_bounds__(tc_threads<Q8>(), 1) decode_tc_kernel(const __grid_constant__ DecodeArgs a) {
+  constexpr int NS = tc_stages<Q8, QG>();
+  constexpr int CSt = tc_code_stages<QG>();
   extern __shared__ uint8_t smem_raw[];
-  auto& sm = *reinterpret_cast<TcSmem<QG>*>(smem_raw +
-                                            ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
+  auto& sm = *reinterpret_cast<TcSmem<QG, Q8>*>(smem_raw +
+                                                ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const uint32_t lane = tid & 31;
@@ -129,9 +183,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
 
   if (tid == 0) launch_dependents();  // the combine may be placed (it waits for this grid)
   if (tid == 0) {
-    for (int s = 0; s < kTcStages; ++s) {
-      bar_init(&sm.full[s], 1);
+    for (int s = 0; s < NS; ++s) {
+      bar_init(&sm.full[s], Q8 ? kTcConvWarps : 1);  // (8-bit: the converter warps)
       bar_init(&sm.empty[s], 1);
+    }
+    if constexpr (Q8) {
+      for (int s = 0; s < CSt; ++s) {
+        bar_init(&sm.cr.cfull[s], 1);
+        bar_init(&sm.cr.cempty[s], kTcConvWarps);
+      }
     }
     for (int x = 0; x < 2; ++x) {
       bar_init(&sm.qfull[x], 1);
@@ -169,14 +229,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
       bool ok = true;
       // one tile into the next ring slot; K and V are read once: evict-first,
       // so that the logits written to score_inc stay in L2 for the combine
+      // (8-bit buffers: the code tile and its scales into the code ring)
+      constexpr int RS = Q8 ? CSt : NS;
       auto load = [&](const CUtensorMap* m, const TcItem& x, int t) -> bool {
-        const int s = slot % kTcStages;
-        if (slot >= kTcStages && !twait(&sm.empty[s], ((slot / kTcStages) - 1) & 1, abort_flag))
-          return false;
-        bar_expect_tx(&sm.full[s], kTcTileBytes);
-        for (int p = 0; p < 2; ++p)
-          tma_load_3d_once(sm.ring[s] + p * kTcPanel, m, &sm.full[s], 64 * p, x.j0 + kTcKeys * t,
-                           x.grp);
+        const int s = slot % RS;
+        if constexpr (Q8) {
+          if (slot >= RS && !twait(&sm.cr.cempty[s], ((slot / RS) - 1) & 1, abort_flag))
+            return false;
+          const bool is_v = m == &a.tm_vc;
+          bar_expect_tx(&sm.cr.cfull[s], kTcCodeBytes + kTcKeys * 4);
+          tma_load_3d_once(sm.cr.codes[s], m, &sm.cr.cfull[s], 0, x.j0 + kTcKeys * t, x.grp);
+          tma_load_1d(sm.cr.scl[s], is_v ? &a.tm_vs : &a.tm_ks, &sm.cr.cfull[s],
+                      x.grp * a.M + x.j0 + kTcKeys * t);
+        } else {
+          if (slot >= RS && !twait(&sm.empty[s], ((slot / RS) - 1) & 1, abort_flag)) return false;
+          bar_expect_tx(&sm.full[s], kTcTileBytes);
+          for (int p = 0; p < 2; ++p)
+            tma_load_3d_once(sm.ring[s] + p * kTcPanel, m, &sm.full[s], 64 * p,
+                             x.j0 + kTcKeys * t, x.grp);
+        }
         ++slot;
         return true;
       };
@@ -204,8 +275,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
         // let the copies still in flight land: the latest load of each stage
         // and of each q buffer
         volatile int never = 0;
-        for (uint32_t u = slot > kTcStages ? slot - kTcStages : 0; u < slot; ++u)
-          wait_bar(&sm.full[u % kTcStages], (u / kTcStages) & 1, &never, 100000000ull);
+        for (uint32_t u = slot > RS ? slot - RS : 0; u < slot; ++u) {
+          if constexpr (Q8)
+            wait_bar(&sm.cr.cfull[u % RS], (u / RS) & 1, &never, 100000000ull);
+          else
+            wait_bar(&sm.full[u % RS], (u / RS) & 1, &never, 100000000ull);
+        }
         for (int u = qloads > 2 ? qloads - 2 : 0; u < qloads; ++u)
           wait_bar(&sm.qfull[u & 1], (u >> 1) & 1, &never, 100000000ull);
       }
@@ -227,11 +302,18 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
       const uint64_t vd0 = sdesc_sw128(smem_addr(sm.ring[0]), kTcPanel, 1024);
       uint32_t slot = 0, kt_g = 0, vt_g = 0;
       bool ok = true;
+      // a tile in the ring: with 8-bit buffers it is signalled by the
+      // converter warps, whose arrivals a suspended wait noticed only
+      // ~650 cycles later (measured), so it is polled
+      auto tile_wait = [&](uint64_t* bar, uint32_t parity, volatile int* abort) -> bool {
+        if constexpr (Q8) return wait_bar_poll(bar, parity, abort, kWaitLimitNs);
+        else return twait(bar, parity, abort);
+      };
       // S^T of item k's tile t
       auto issue_s = [&](int qb) -> bool {
-        const int sb = kt_g & 1, s = slot % kTcStages;
+        const int sb = kt_g & 1, s = slot % NS;
         if ((kt_g >= 2 && !twait(&sm.sfree[sb], ((kt_g >> 1) - 1) & 1, abort_flag)) ||
-            !twait(&sm.full[s], (slot / kTcStages) & 1, abort_flag))
+            !tile_wait(&sm.full[s], (slot / NS) & 1, abort_flag))
           return false;
         tc_fence_after_sync();
         uint64_t kd[8], qd[8];
@@ -249,9 +331,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
       };
       // O^T (+)= V^T P^T of the previous item's tile t
       auto issue_pv = [&](int t) -> bool {
-        const int pb = vt_g & 1, s = slot % kTcStages;
+        const int pb = vt_g & 1, s = slot % NS;
         if (!twait(&sm.pfull[pb], (vt_g >> 1) & 1, abort_flag) ||
-            !twait(&sm.full[s], (slot / kTcStages) & 1, abort_flag))
+            !tile_wait(&sm.full[s], (slot / NS) & 1, abort_flag))
           return false;
         tc_fence_after_sync();
         uint64_t vd[8], pd[8];
@@ -288,7 +370,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
       volatile int never = 0;
       wait_bar(&sm.drain, 0, &never, kWaitLimitNs);
     }
-  } else {
+  } else if (warp < 2 + kTcKeyWarps) {
     // -------------------------------------------------------------- key warps --
     // Thread kl holds key kl of each tile (TMEM lane kl of S^T) and row d = kl
     // of O^T; lane quarter warp % 4.
@@ -498,6 +580,65 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
         }
       }
     }
+  } else if constexpr (Q8) {
+    // ------------------------------------------------------------ converters --
+    // 8-bit buffers: the converter warps turn each code tile into the bf16
+    // tile the MMA reads, in the ring order of the producer: warp cw takes
+    // rows 4 (8 i + cw) .. + 3, sixteen codes of a row per lane, read back as
+    // the 8-bit format defines, bf16(code * scale) (q8_bf16x2), and written
+    // where a 128-byte-swizzled TMA load of the bf16 row would have put them.
+    const int cw = warp - 2 - kTcKeyWarps;
+    // lane: codes 16 g .. 16 g + 15 (g = lane % 8) of row 4 i + lane / 8 of
+    // the warp's rows; bf16 columns 16 g .. are chunks 2 g' and 2 g' + 1 of
+    // panel g / 4 (g' = g % 4)
+    const int g8 = static_cast<int>(lane & 7u), rsub = static_cast<int>(lane >> 3);
+    const uint32_t c_lo = static_cast<uint32_t>(2 * (g8 & 3));
+    uint32_t n = 0;  // tiles converted so far
+    bool ok = true;
+    for (int ph = 0; ok && ph <= n_mine; ++ph) {
+      const int tk = ph < n_mine ? item_of(ph).n_kt : 0, tv = ph > 0 ? item_of(ph - 1).n_kt : 0;
+      for (int t = 0; ok && t < max(tk, tv); ++t) {
+        for (int v = 0; v < 2; ++v) {
+          if (t >= (v == 0 ? tk : tv)) continue;
+          const int cs = n % CSt, s = n % NS;
+          if (!twait(&sm.cr.cfull[cs], (n / CSt) & 1, abort_flag) ||
+              (n >= static_cast<uint32_t>(NS) && !twait(&sm.empty[s], ((n / NS) - 1) & 1, abort_flag))) {
+            ok = false;
+            break;
+          }
+          const uint8_t* src = sm.cr.codes[cs] + 16 * g8;
+          uint8_t* dst = sm.ring[s] + (g8 >> 2) * kTcPanel;
+#pragma unroll
+          for (int i = 0; i < kTcKeys / (4 * kTcConvWarps); ++i) {
+            const int r = (i * kTcConvWarps + cw) * 4 + rsub;  // row of the tile
+            const uint4 w = *reinterpret_cast<const uint4*>(src + r * 128);
+            const float sc = sm.cr.scl[cs][r];
+            const uint32_t w4[4] = {w.x ^ 0x80808080u, w.y ^ 0x80808080u, w.z ^ 0x80808080u,
+                                    w.w ^ 0x80808080u};
+            uint4 o0, o1;
+            o0.x = q8_bf16x2(w4[0], 0, sc);
+            o0.y = q8_bf16x2(w4[0], 2, sc);
+            o0.z = q8_bf16x2(w4[1], 0, sc);
+            o0.w = q8_bf16x2(w4[1], 2, sc);
+            o1.x = q8_bf16x2(w4[2], 0, sc);
+            o1.y = q8_bf16x2(w4[2], 2, sc);
+            o1.z = q8_bf16x2(w4[3], 0, sc);
+            o1.w = q8_bf16x2(w4[3], 2, sc);
+            uint8_t* row = dst + r * 128;
+            const uint32_t sw = static_cast<uint32_t>(r & 7);
+            *reinterpret_cast<uint4*>(row + ((c_lo ^ sw) << 4)) = o0;
+            *reinterpret_cast<uint4*>(row + (((c_lo + 1) ^ sw) << 4)) = o1;
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            bar_arrive(&sm.full[s]);
+            bar_arrive(&sm.cr.cempty[cs]);
+          }
+          ++n;
+        }
+      }
+    }
   }
   tc_fence_before_sync();
   __syncthreads();
@@ -508,19 +649,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) decode_tc_kernel(const __grid_c
   if (tid == 0 && sm.abort_flag) atomicOr(a.err, H2O_DEVERR_TIMEOUT);
 }
 
-template <int QG>
+template <int QG, bool Q8>
 cudaError_t launch_tc(const DecodeArgs& a, cudaStream_t stream) {
-  const size_t smem = sizeof(TcSmem<QG>) + 1024;
+  const size_t smem = sizeof(TcSmem<QG, Q8>) + 1024;
   static OncePerDevice once;
   static int resident[kMaxDevices];
   cudaError_t e = once.run([smem](int d) {
-    cudaError_t r = cudaFuncSetAttribute(decode_tc_kernel<QG>,
+    cudaError_t r = cudaFuncSetAttribute(decode_tc_kernel<QG, Q8>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (r != cudaSuccess) return r;
     int per_sm = 0, sms = 0;
-    r = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_tc_kernel<QG>, kTcThreads,
-                                                      smem);
+    r = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_tc_kernel<QG, Q8>,
+                                                      tc_threads<Q8>(), smem);
     if (r != cudaSuccess) return r;
     r = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, d);
     if (r != cudaSuccess) return r;
@@ -533,14 +674,15 @@ cudaError_t launch_tc(const DecodeArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const int n_items = a.n_split * a.B * a.Hkv;
   const int grid = n_items < resident[dev] ? n_items : resident[dev];
-  decode_tc_kernel<QG><<<grid, kTcThreads, smem, stream>>>(a);
+  decode_tc_kernel<QG, Q8><<<grid, tc_threads<Q8>(), smem, stream>>>(a);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t stream) {
-  return a.qg <= 4 ? launch_tc<4>(a, stream) : launch_tc<8>(a, stream);
+  if (a.q8) return a.qg <= 4 ? launch_tc<4, true>(a, stream) : launch_tc<8, true>(a, stream);
+  return a.qg <= 4 ? launch_tc<4, false>(a, stream) : launch_tc<8, false>(a, stream);
 }
 
 }  // namespace h2o

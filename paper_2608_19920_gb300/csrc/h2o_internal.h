@@ -133,9 +133,12 @@ constexpr int kDecodeTcMinSplitLen = 512;
 constexpr int kDecodeItemOverheadKeys = 32;  // per-item cost, in keys, for choosing the split
 
 struct DecodeArgs {
-  // tensor-core path (d = 128, bf16 buffers): TMA maps of q {d, Hq, B} with
-  // box {64, 16, 1} and of the cache K / V {d, M, B*Hkv} with box {64, 128, 1}
-  CUtensorMap tm_q, tm_kc, tm_vc;
+  // tensor-core path (d = 128): TMA maps of q {d, Hq, B} with box {64, 16, 1}
+  // and of the cache K / V {d, M, B*Hkv} with box {64, 128, 1} (bf16, 128-byte
+  // swizzle); with 8-bit buffers tm_kc / tm_vc map the codes {d, M, B*Hkv}
+  // (uint8, box {128, 128, 1}, no swizzle) and tm_ks / tm_vs the scales
+  // {B*Hkv*M} (fp32, box {128})
+  CUtensorMap tm_q, tm_kc, tm_vc, tm_ks, tm_vs;
   int tc;                   // 1: decode_tc_kernel (maps valid); 0: decode_split_kernel
   const uint16_t* q;        // (B, Hq, 1, d)
   const uint16_t* k_cache;  // (B, Hkv, M, d)

@@ -158,6 +158,8 @@ SDPA_CASES = [
     (1, 4, 1, 128, 1, 255, 300, False),       # S = 1: a ring slot of 127 code rows + the new bf16 row
     (2, 16, 2, 64, 1, 777, 900, False),       # S = 1, q_g = 8, d = 64
     (1, 8, 1, 128, 1, 1537, 1600, True),      # S = 1, q_g = 8, a last tile of one code row
+    (1, 16, 2, 128, 1, 2052, 2100, False),    # S = 1, d = 128, M % 4 = 0: the tensor-core kernel
+    (2, 8, 1, 128, 1, 1536, 1600, True),      # the same with q_g = 8, cache only
 ]
 
 

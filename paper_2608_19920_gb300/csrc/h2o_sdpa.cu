@@ -65,13 +65,19 @@ constexpr uint16_t kTileIdxMask = 0x3FFF;
 constexpr uint8_t kClsSkip = 0, kClsFull = 1, kClsPartial = 2;
 // TMEM (512 columns).  Pass 1 needs no P or O: four S buffers (fp32, 128
 // columns each), each free again as soon as the softmax has loaded it.
-// Pass 2: three S buffers and the O accumulator (columns 384..).  The softmax
-// loads a tile's S, then writes the bf16 P of warpgroup u's 64 keys as pairs
-// into columns 64u .. 64u+31 of the same buffer (columns only that warpgroup
-// loaded), where the P V MMA reads it; the buffer is free again when that P V
-// has completed.  So writing P never waits for an earlier P V.
+// Pass 2: three S buffers and the O accumulator (columns 384..).  Every
+// warpgroup takes every pass-2 tile: warpgroup w loads the S of keys
+// 32w .. 32w+31, then writes their bf16 P as pairs into columns 32w .. 32w+15
+// of the same buffer (columns only that warpgroup loaded), where the P V MMA
+// reads it; the buffer is free again when that P V has completed.  So writing
+// P never waits for an earlier P V.
 constexpr int kSBufs1 = 4;
 constexpr int kSBufs2 = 3;
+// Column-sum buffers, used round robin by the pass-2 tiles.  Buffer c of tile
+// t is written again by tile t + 4, whose Q K^T was issued after the P V of
+// tile t + 1 had completed, which needed every softmax warp's arrival for
+// tile t + 1, which each warp makes after its reads of tile t's buffer.
+constexpr int kColBufs = 4;
 
 __device__ __forceinline__ int pass1_buffer_uses(int n_t, int b) {
   return n_t > b ? (n_t - 1 - b) / kSBufs1 + 1 : 0;
@@ -120,13 +126,13 @@ struct __align__(1024) SdpaSmem {
   using G = Geom<D, kPair>;
   uint8_t q[G::kPanels][kTileM * 128];
   uint8_t kv[G::kR][G::kSlotBytes];
-  float colsum[2][kNumWG][4][64];  // [buffer][warpgroup][warp][column]
+  float colsum[kColBufs][kNumWG][4][32];  // [buffer][warpgroup][warp][column]
   float rowstat[kNumWG][kTileM][2];
   uint64_t bar_q;
   uint64_t bar_full[G::kR], bar_empty[G::kR];
   uint64_t bar_sfull[kSBufs1], bar_sread[kSBufs1], bar_pfull[kSBufs2], bar_pvdone[kSBufs2];
   uint64_t bar_rowstat, bar_ofull, bar_drain[2], bar_p1done;
-  uint32_t cs_count[2][kNumWG];  // column-sum partials deposited (4 per tile)
+  uint32_t cs_count[kColBufs][kNumWG];  // column-sum partials deposited (4 per tile)
   uint32_t taddr;
   int abort_flag;
   int n_tiles;
@@ -229,10 +235,11 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       bar_init(&sm.bar_sread[x], G::kCtas * kSoftmaxWarps / 2);
     }
     for (int x = 0; x < kSBufs2; ++x) {
-      bar_init(&sm.bar_pfull[x], G::kCtas * kSoftmaxWarps / 2);
+      // every softmax warp, in every CTA of the pair
+      bar_init(&sm.bar_pfull[x], G::kCtas * kSoftmaxWarps);
       bar_init(&sm.bar_pvdone[x], 1);
     }
-    for (int x = 0; x < 2; ++x)
+    for (int x = 0; x < kColBufs; ++x)
       for (int w = 0; w < kNumWG; ++w) sm.cs_count[x][w] = 0u;
     bar_init(&sm.bar_rowstat, kSoftmaxWarps);
     bar_init(&sm.bar_ofull, 1);
@@ -501,9 +508,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           uint64_t bd[8];
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) bd[kk] = vd + 128 * kk;
-          // keys 0-63 (16 per K-step) as bf16 pairs in columns 0-31 of the
-          // buffer, keys 64-127 in columns 64-95
-          mma_ts_x8<kPair>(tO, tS + 128 * pb, tS + 128 * pb + 64, bd, kIdescPV, t > 0 ? 1u : 0u);
+          // keys 32w .. 32w+31 (two K-steps) as bf16 pairs in columns
+          // 32w .. 32w+15 of the buffer
+          mma_ts_x8<kPair>(tO, tS + 128 * pb, bd, kIdescPV, t > 0 ? 1u : 0u);
           commit_all<kPair>(&sm.bar_empty[vs]);
           commit_all<kPair>(&sm.bar_pvdone[pb]);
         }
@@ -518,10 +525,13 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     }
   } else {
     // ------------------------------------------- softmax / column sums --
-    // Two teams of two warpgroups take alternate tiles (team 0 even, team 1
-    // odd), so one team's exp-bound phase overlaps the other team's TMEM loads,
-    // column sums and barrier waits.  Within a team, warpgroup u owns key
-    // columns 64u .. 64u+63 of its tiles.
+    // Pass 1: two teams of two warpgroups take alternate tiles (team 0 even,
+    // team 1 odd), so one team's exp-bound phase overlaps the other team's TMEM
+    // loads and barrier waits; within a team, warpgroup u owns key columns
+    // 64u .. 64u+63.  Pass 2 is a chain (Q K^T, softmax, P V, and the next
+    // Q K^T into the freed buffer), so there all four warpgroups take every
+    // tile, warpgroup w its key columns 32w .. 32w+31, which halves the
+    // softmax's share of that chain.
     const int sw = warp - kFirstSoftmaxWarp;
     const int wg = sw >> 2;          // 0..3
     const int team = wg >> 1;
@@ -598,7 +608,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
     bool have_lambda = false;
     int k2 = 0;  // pass-2 tiles this warp has processed (column-sum buffer phase)
     const int n_end = a.lse != nullptr ? n_t : 2 * n_t;  // pass 1 only when lse is asked
-    for (int n = team; ok && n < n_end; n += 2) {
+    // this team's pass-1 tiles, then every pass-2 tile
+    auto next_step = [n_t](int n) { return n >= n_t ? n + 1 : (n + 2 < n_t ? n + 2 : n_t); };
+    for (int n = team < n_t ? team : n_t; ok && n < n_end; n = next_step(n)) {
       int buf, suse;
       s_buffer(n, n_t, buf, suse);
       const bool pass2 = n >= n_t;
@@ -645,8 +657,8 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       const uint16_t e = sm.tiles[t];
       const bool chunk = (e & kTileChunk) != 0;
       const bool partial = (e & kTilePartial) != 0;
-      const uint32_t s_base = tS + lane_addr + buf * 128 + u * 64;
       if (!pass2) {
+        const uint32_t s_base = tS + lane_addr + buf * 128 + u * 64;
         // pass 1 (one row per thread, 64 columns in two halves of 32): running
         // max and sum of exp2, updated after each half, so that only 32 values
         // are live; the S buffer is released once both halves are loaded
@@ -726,21 +738,18 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           }
         }
       } else {
-        // pass 2 (16x256b layout), in two halves of 32 columns: P in fp32,
-        // bf16 copy to a TMEM P buffer for P V, column sums of the fp32 P
-        const int cb = k2 & 1;
-        // P goes over this warpgroup's own S columns: its 64 keys as bf16
-        // pairs in columns 0-31 of the group's range, which hold the S of half
-        // 0; half 0 is loaded before any P is stored, half 1 (columns 32-63)
-        // is never overwritten.
+        // pass 2 (16x256b layout), this warpgroup's 32 columns: P in fp32,
+        // its bf16 copy over the first 16 of those TMEM columns (loaded
+        // before any P is stored) for P V, column sums of the fp32 P
+        const int cb = k2 & (kColBufs - 1);
+        const uint32_t s_base = tS + lane_addr + buf * 128 + wg * 32;
         const uint32_t p_base = s_base;
-#pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          const int col0 = (e & kTileIdxMask) * kTileN + u * 64 + 32 * h;
+        {
+          const int col0 = (e & kTileIdxMask) * kTileN + wg * 32;
           float pa[16], pb[16];  // rows lane/4 + {0, 8} and + {16, 24}
           {
             uint32_t r[32];
-            tmem_ld_16x256b_x4x2_async(s_base + 32 * h, r);
+            tmem_ld_16x256b_x4x2_async(s_base, r);
             tmem_wait_ld(r);
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
@@ -797,13 +806,13 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
               pk[2 * k] = pack_bf16x2(pa[4 * k], pa[4 * k + 1]);
               pk[2 * k + 1] = pack_bf16x2(pa[4 * k + 2], pa[4 * k + 3]);
             }
-            tmem_st_16x128b_x4_async(p_base + 16 * h, pk);
+            tmem_st_16x128b_x4_async(p_base, pk);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               pk[2 * k] = pack_bf16x2(pb[4 * k], pb[4 * k + 1]);
               pk[2 * k + 1] = pack_bf16x2(pb[4 * k + 2], pb[4 * k + 3]);
             }
-            tmem_st_16x128b_x4_async(p_base + 16 * h + (16u << 16), pk);
+            tmem_st_16x128b_x4_async(p_base + (16u << 16), pk);
           }
           // column sums: 4 rows in-thread, then a reduce-scatter over lane bits
           // 4, 3, 2 leaves one column (summed over the warp's 32 rows) per lane
@@ -819,7 +828,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
           rs_step<8, 16>(v, lane);
           rs_step<4, 8>(v, lane);
           rs_step<2, 4>(v, lane);
-          sm.colsum[cb][wg][q4][32 * h + cl] = v[0];
+          sm.colsum[cb][wg][q4][cl] = v[0];
         }
         if (!ok) break;
         tmem_wait_st();
@@ -838,10 +847,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         last = __shfl_sync(0xffffffffu, last, 0);
         if (last) {
           __syncwarp();
-          const int colb = (e & kTileIdxMask) * kTileN + u * 64;
-#pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            const int c = 32 * hh + static_cast<int>(lane);
+          const int colb = (e & kTileIdxMask) * kTileN + wg * 32;
+          {
+            const int c = static_cast<int>(lane);
             const int col = colb + c;
             if (prow != nullptr && (chunk ? col < a.S : col < a.M)) {
               // one head: the four quarters in order, stored (rows past S

@@ -413,23 +413,23 @@ __device__ __forceinline__ void mma_ss_x8(uint32_t d_tmem, const uint64_t (&a)[8
   }
 }
 
-// D (+)= sum_k A_k B_k over eight K-steps, A from TMEM (K-steps 0-3 at
-// columns a_lo + 8k, K-steps 4-7 at a_hi + 8(k - 4)), B from shared memory.
+// D (+)= sum_k A_k B_k over eight K-steps, A from TMEM, B from shared memory.
+// K-steps 2j and 2j + 1 read A at columns a + 32 j and a + 32 j + 8: the bf16
+// pairs of 32 keys sit in the first 16 of each 32-column group.
 template <bool kPair>
-__device__ __forceinline__ void mma_ts_x8(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi,
-                                          const uint64_t (&b)[8], uint32_t idesc,
-                                          uint32_t acc_first) {
-  const uint32_t a_tmem = a_lo, a1 = a_lo + 8, a2 = a_lo + 16, a3 = a_lo + 24, a4 = a_hi,
-                 a5 = a_hi + 8, a6 = a_hi + 16, a7 = a_hi + 24;
+__device__ __forceinline__ void mma_ts_x8(uint32_t d_tmem, uint32_t a, const uint64_t (&b)[8],
+                                          uint32_t idesc, uint32_t acc_first) {
+  const uint32_t a1 = a + 8, a2 = a + 32, a3 = a + 40, a4 = a + 64, a5 = a + 72, a6 = a + 96,
+                 a7 = a + 104;
   if constexpr (kPair) {
     asm volatile(H2O_MMA8("2", "[%3]", "[%12]", "[%13]", "[%14]", "[%15]", "[%16]", "[%17]", "[%18]")
-                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "r"(a_tmem), "l"(b[0]), "l"(b[1]),
+                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "r"(a), "l"(b[0]), "l"(b[1]),
                  "l"(b[2]), "l"(b[3]), "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]), "r"(a1),
                  "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
                  : "memory");
   } else {
     asm volatile(H2O_MMA8("1", "[%3]", "[%12]", "[%13]", "[%14]", "[%15]", "[%16]", "[%17]", "[%18]")
-                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "r"(a_tmem), "l"(b[0]), "l"(b[1]),
+                 ::"r"(d_tmem), "r"(idesc), "r"(acc_first), "r"(a), "l"(b[0]), "l"(b[1]),
                  "l"(b[2]), "l"(b[3]), "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]), "r"(a1),
                  "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
                  : "memory");

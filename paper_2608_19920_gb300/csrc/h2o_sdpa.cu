@@ -222,6 +222,20 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
   // the kernels after it on the stream (column-sum reduction, update) may be
   // placed now; they wait for this grid before reading what it writes
   if (tid == 0) launch_dependents();
+  // While the tiles are classified, bring Q and the first cache K tiles (this
+  // CTA's halves) into L2, so the loads after the classification hit there.
+  if (warp == 0 && lane == 0 && has_rows) {
+    tma_prefetch_desc(&a.tm_q);
+    for (int p = 0; p < P; ++p) tma_prefetch_4d(&a.tm_q, 64 * p, i_lo, g_first, grp);
+    if (a.n_cache_tiles > 0) {
+      tma_prefetch_desc(&a.tm_kc);
+      const int n_pre = 0;
+      for (int t = 0; t < n_pre; ++t)
+        for (int p = 0; p < P; ++p)
+          tma_prefetch_3d(&a.tm_kc, 64 * p, t * kTileN + (kPair ? (kTileN / 2) * static_cast<int>(rank) : 0),
+                          grp);
+    }
+  }
 
   if (tid == 0) {
     bar_init(&sm.bar_q, 1);
@@ -271,24 +285,37 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
   if (warp >= kFirstSoftmaxWarp) {
     const int sw = warp - kFirstSoftmaxWarp;
     const int* sp = a.slot_pos + static_cast<size_t>(grp) * a.M;
-    for (int ct = sw; ct < a.n_cache_tiles; ct += kSoftmaxWarps) {
-      bool any0 = false, all0 = true, any1 = false, all1 = true;
+    // four tiles per round, all their slot_pos loads in flight at once
+    for (int ct0 = sw; ct0 < a.n_cache_tiles; ct0 += 4 * kSoftmaxWarps) {
+      int pos4[4][4];
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        const int j = ct * kTileN + r * 32 + static_cast<int>(lane);
-        const int pos = j < a.M ? __ldg(sp + j) : -1;
-        any0 |= pos >= 0 && pos <= a.pos0 + i_hi;
-        all0 &= pos >= 0 && pos <= a.pos0 + i_lo;
-        any1 |= pos >= 0 && pos <= a.pos0 + p_hi;
-        all1 &= pos >= 0 && pos <= a.pos0 + p_lo;
+      for (int bt = 0; bt < 4; ++bt)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const int j = (ct0 + bt * kSoftmaxWarps) * kTileN + r * 32 + static_cast<int>(lane);
+          pos4[bt][r] = j < a.M ? __ldg(sp + j) : -1;
+        }
+#pragma unroll
+      for (int bt = 0; bt < 4; ++bt) {
+        const int ct = ct0 + bt * kSoftmaxWarps;
+        if (ct >= a.n_cache_tiles) break;
+        bool any0 = false, all0 = true, any1 = false, all1 = true;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const int pos = pos4[bt][r];
+          any0 |= pos >= 0 && pos <= a.pos0 + i_hi;
+          all0 &= pos >= 0 && pos <= a.pos0 + i_lo;
+          any1 |= pos >= 0 && pos <= a.pos0 + p_hi;
+          all1 &= pos >= 0 && pos <= a.pos0 + p_lo;
+        }
+        any0 = __any_sync(0xffffffffu, any0) && has_rows;
+        all0 = __all_sync(0xffffffffu, all0);
+        any1 = __any_sync(0xffffffffu, any1) && peer_rows;
+        all1 = __all_sync(0xffffffffu, all1);
+        const uint8_t c0 = any0 ? (all0 ? kClsFull : kClsPartial) : kClsSkip;
+        const uint8_t c1 = any1 ? (all1 ? kClsFull : kClsPartial) : kClsSkip;
+        if (lane == 0) sm.cls[ct] = static_cast<uint8_t>(c0 | (c1 << 2));
       }
-      any0 = __any_sync(0xffffffffu, any0) && has_rows;
-      all0 = __all_sync(0xffffffffu, all0);
-      any1 = __any_sync(0xffffffffu, any1) && peer_rows;
-      all1 = __all_sync(0xffffffffu, all1);
-      const uint8_t c0 = any0 ? (all0 ? kClsFull : kClsPartial) : kClsSkip;
-      const uint8_t c1 = any1 ? (all1 ? kClsFull : kClsPartial) : kClsSkip;
-      if (lane == 0) sm.cls[ct] = static_cast<uint8_t>(c0 | (c1 << 2));
     }
     for (int c = sw; c < a.n_chunk_tiles; c += kSoftmaxWarps) {
       const int c0 = c * kTileN;

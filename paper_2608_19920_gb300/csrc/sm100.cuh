@@ -229,6 +229,22 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
 // TMA loads of a CTA pair (.cta_group::2): the data lands in this CTA's shared
 // memory, the transaction bytes are counted on the mbarrier given by its
 // shared::cluster address, which may be in the other CTA of the pair.
+// L2 prefetch of the box that a tiled TMA load with these coordinates reads
+// (no shared memory, no barrier; x times the element size a multiple of 16).
+__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_4d(const CUtensorMap* map, int x, int y, int z, int w) {
+  asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z), "r"(w)
+               : "memory");
+}
+
 __device__ __forceinline__ void tma_load_3d_pair(void* dst, const CUtensorMap* map,
                                                  uint32_t bar_cluster, int x, int y, int z) {
   asm volatile(

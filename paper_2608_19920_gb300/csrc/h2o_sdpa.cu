@@ -56,9 +56,11 @@ namespace h2o {
 namespace {
 
 constexpr int kNumWG = 4;                       // softmax warpgroups
-constexpr int kFirstSoftmaxWarp = 3;  // warp 0 TMA, warp 1 Q K^T issuer, warp 2 P V issuer
+// warp 0 TMA producer, warps 1 and 3 Q K^T issuers (even / odd tiles), warp 2
+// P V issuer
+constexpr int kFirstSoftmaxWarp = 4;
 constexpr int kSoftmaxWarps = 4 * kNumWG;
-constexpr int kThreads = 32 * (kFirstSoftmaxWarp + kSoftmaxWarps);  // 608
+constexpr int kThreads = 32 * (kFirstSoftmaxWarp + kSoftmaxWarps);  // 640
 constexpr uint16_t kTileChunk = 0x8000;
 constexpr uint16_t kTilePartial = 0x4000;
 constexpr uint16_t kTileIdxMask = 0x3FFF;
@@ -131,7 +133,7 @@ struct __align__(1024) SdpaSmem {
   uint64_t bar_q;
   uint64_t bar_full[G::kR], bar_empty[G::kR];
   uint64_t bar_sfull[kSBufs1], bar_sread[kSBufs1], bar_pfull[kSBufs2], bar_pvdone[kSBufs2];
-  uint64_t bar_rowstat, bar_ofull, bar_drain[2], bar_p1done;
+  uint64_t bar_rowstat, bar_ofull, bar_drain[3];
   uint32_t cs_count[kColBufs][kNumWG];  // column-sum partials deposited (4 per tile)
   uint32_t taddr;
   int abort_flag;
@@ -257,9 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       for (int w = 0; w < kNumWG; ++w) sm.cs_count[x][w] = 0u;
     bar_init(&sm.bar_rowstat, kSoftmaxWarps);
     bar_init(&sm.bar_ofull, 1);
-    bar_init(&sm.bar_drain[0], 1);
-    bar_init(&sm.bar_drain[1], 1);
-    bar_init(&sm.bar_p1done, 1);
+    for (int x = 0; x < 3; ++x) bar_init(&sm.bar_drain[x], 1);
     sm.abort_flag = 0;
     fence_bar_init();
   }
@@ -440,13 +440,17 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         }
       }
     }
-  } else if (warp == 1 || warp == 2) {
+  } else if (warp < kFirstSoftmaxWarp) {
     // ------------------------------------------------------- MMA issuers --
-    // Pass 1: warps 1 and 2 issue the Q K^T of alternate tiles (each S buffer
-    // has one issuer, so its phases complete in order).  Pass 2: warp 1 issues
-    // every Q K^T, warp 2 every P V and owns the O accumulator.  With two
-    // issuing threads the tensor pipe keeps working while one of them waits on
-    // a barrier or commits.  On a pair only the even CTA issues.
+    // Warps 1 and 3 issue the Q K^T of the even and the odd tiles of each
+    // pass, warp 2 every P V (it owns the O accumulator).  An issuing thread
+    // runs only about one MMA ahead of the tensor pipe and then spends several
+    // hundred cycles on commits, barrier waits and the next tile's indices, so
+    // the pipe is kept busy by having these threads overlap.  A ring slot's
+    // loads are all consumed by the Q K^T issuer of the slot's parity (slot n
+    // mod 10 in pass 1, t mod 6 in pass 2) or by the P V issuer, in order, so
+    // no full-barrier wait can run two phases ahead.  On a pair only the even
+    // CTA issues.
     if (lane == 0 && n_t > 0 && leader) {
       constexpr int kM = kPair ? 2 * kTileM : kTileM;
       constexpr uint32_t kIdescQK = idesc_bf16_f32(kM, kTileN, false);
@@ -460,7 +464,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
       constexpr uint32_t kKPanel = G::kKPanelBytes >> 4;
       constexpr uint32_t kSlot = G::kSlotBytes >> 4;
       constexpr int RA = G::kRA, RB = G::kRB;
-      const bool is_qk = warp == 1;
+      static_assert(RA % 2 == 0 && (RA + RB) % 2 == 0, "ring slots split by issuer parity");
+      const bool is_pv = warp == 2;
+      const int par = warp == 1 ? 0 : 1;  // the Q K^T issuer's tile parity
       const uint64_t q_desc = sdesc_sw128(smem_addr(sm.q[0]), 16, 1024);
       const uint64_t k_desc0 = sdesc_sw128(smem_addr(sm.kv[0]), 16, 1024);
       uint64_t qd[8];
@@ -506,17 +512,10 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         return true;
       };
       bool ok = wait_b<kPair>(&sm.bar_q, 0, abort_flag);
-      if (is_qk) {
-        // pass 1: even tiles here, odd tiles on warp 2 (idle until pass 2)
-        for (int n = 0; ok && n < n_t; n += 2) ok = issue_qk(n);
-        // pass 2 reuses slots that warp 2 took in pass 1: start once it has
-        // waited for all of its pass-1 tiles, so that no full-barrier wait
-        // here runs two phases ahead
-        if (ok && a.lse == nullptr) ok = wait_b<kPair>(&sm.bar_p1done, 0, abort_flag);
-        for (int n = n_t; ok && a.lse == nullptr && n < 2 * n_t; ++n) ok = issue_qk(n);
+      if (!is_pv) {
+        for (int n = par; ok && n < n_t; n += 2) ok = issue_qk(n);
+        for (int t = par; ok && a.lse == nullptr && t < n_t; t += 2) ok = issue_qk(n_t + t);
       } else {
-        for (int n = 1; ok && n < n_t; n += 2) ok = issue_qk(n);
-        bar_arrive(&sm.bar_p1done);
         const uint64_t v_desc0 = sdesc_sw128(smem_addr(sm.kv[RA]), kTileN * 128, 1024);
         for (int t = 0; ok && a.lse == nullptr && t < n_t; ++t) {
           const int pb = t % kSBufs2;  // the S buffer of pass-2 tile t holds its P
@@ -544,7 +543,7 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         if (ok && a.lse == nullptr) commit_all<kPair>(&sm.bar_ofull);
       }
       // No MMA of this thread may still be running when TMEM is freed.
-      uint64_t* drain = &sm.bar_drain[is_qk ? 0 : 1];
+      uint64_t* drain = &sm.bar_drain[warp - 1];
       if constexpr (kPair) mma_commit_pair(drain, 1);
       else mma_commit(drain);
       volatile int never = 0;

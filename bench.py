@@ -72,7 +72,7 @@ def step_flops(w: wl.Workload, order: str = "chunk"):
 # chunk launch of the current SDPA kernel, from the ncu capture summarised in
 # profiles/sdpa_chunk_kernel_llama8b_32k.md; None whenever the kernel has
 # changed since that capture.
-SDPA_DRAM_BYTES = 23.8779e6
+SDPA_DRAM_BYTES = 23.3321e6
 
 
 def peaks():

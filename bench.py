@@ -587,7 +587,6 @@ def run_e2e(w, layer, plan, outs, dev, args, world):
     ev_in = [torch.cuda.Event() for _ in range(n_c)]
     ev_done = [torch.cuda.Event() for _ in range(n_c)]
     ev_out = torch.cuda.Event()
-    ev_step = torch.cuda.Event()
 
     def upload(i):
         with torch.cuda.stream(s_in):
@@ -595,12 +594,15 @@ def run_e2e(w, layer, plan, outs, dev, args, world):
                 a.copy_(b, non_blocking=True)
             ev_in[i].record(s_in)
 
+    ev_start = torch.cuda.Event()
+
     def step():
-        # the previous step's compute and read-backs are done with the buffers
-        ev_step.record(stream)
-        s_in.wait_event(ev_step)
-        s_in.wait_event(ev_out)
-        stream.wait_event(ev_out)
+        # Fork the copy streams off the compute stream and join them back at
+        # the end, so that a step is self-contained (and capturable): the
+        # previous step's compute and read-backs are done with the buffers.
+        ev_start.record(stream)
+        s_in.wait_event(ev_start)
+        s_out.wait_event(ev_start)
         layer.reset()
         upload(0)
         for i, ((p, e), dx, o, ho) in enumerate(zip(plan, dev_in, outs, host_out)):
@@ -613,24 +615,38 @@ def run_e2e(w, layer, plan, outs, dev, args, world):
             with torch.cuda.stream(s_out):
                 ho.copy_(o, non_blocking=True)
         ev_out.record(s_out)
+        stream.wait_event(ev_out)  # the read-backs are part of the step
 
     for _ in range(2):
         step()
     torch.cuda.synchronize()
+    # As for the resident number, the whole step is replayed from a CUDA
+    # graph: its copy nodes move every step's inputs from pinned host memory
+    # and every chunk's output back on each replay.
+    graph = None
+    if args.graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            step()
+        graph.replay()
+        torch.cuda.synchronize()
     barrier(world)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     n = max(2, args.steps // 2)
     t0.record(stream)
     for _ in range(n):
-        step()
-    stream.wait_event(ev_out)  # the last read-back is inside the timed region
+        if graph is not None:
+            graph.replay()
+        else:
+            step()
     t1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(t0.elapsed_time(t1) / n, world)
     return {"value": w.B * w.T * world / (ms / 1e3), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms,
-            "copies": "overlapped with the compute (two copy streams)"}
+            "copies": "overlapped with the compute (two copy streams)",
+            "launch": "CUDA graph of the whole step, copies included" if args.graph else "eager"}
 
 
 def main():

@@ -109,6 +109,8 @@ SDPA_CASES = [
     (2, 8, 2, 128, 300, 700, 11, 20, 3000),   # 3 row tiles per head (the last of 44 rows):
                                               # column sums through the workspace
     (1, 4, 1, 64, 520, 130, 0, 40, 600),      # d = 64, 5 row tiles per head, future slots
+    (1, 4, 2, 128, 100, 0, 0, 0, 0),          # one key tile: the odd Q K^T issuer has none
+    (1, 4, 2, 128, 48, 128, 0, 0, 300),       # two key tiles: one per Q K^T issuer
 ]
 
 

@@ -865,9 +865,9 @@ __global__ void __launch_bounds__(kThreads, 1) sdpa_chunk_kernel(const __grid_co
         // quarters' partial sums per query head and issues the reductions; the
         // others go straight on to their next tile.  The counter only grows
         // (four per tile), so "last" is old % 4 == 3.  Buffer cb is written
-        // again two tiles later, by a warp that has waited for the P V of the
-        // tile in between, which needed this warp's pfull arrival for that
-        // tile, which comes after the reads below in program order.
+        // again four tiles later, after every warp's P arrival for the next
+        // tile, which comes after the reads below in program order (see
+        // kColBufs).
         int last = 0;
         if (lane == 0) last = (atomic_add_acq_rel_cta(&sm.cs_count[cb][wg], 1u) & 3u) == 3u;
         last = __shfl_sync(0xffffffffu, last, 0);

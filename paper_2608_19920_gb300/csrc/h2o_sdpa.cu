@@ -24,12 +24,13 @@
 //    the other CTA can see is fully masked here.  d = 64 runs one CTA per row
 //    tile with the 1-SM MMA.
 //  * Warp roles: warp 0 issues TMA loads (Q once, then K tiles through ring A
-//    and V tiles through ring B of shared-memory slots); warps 1 and 2 issue
-//    the tcgen05 MMAs (pass 1: Q K^T of alternate tiles; pass 2: warp 1 every
-//    Q K^T, warp 2 every P V), so one issuer keeps the tensor pipe busy while
-//    the other waits on a barrier; warps 3-18 form four softmax
-//    warpgroups in two teams that take alternate tiles; the two warpgroups of a
-//    team own key columns 0-63 and 64-127 of their tiles.
+//    and V tiles through ring B of shared-memory slots); warps 1 and 3 issue
+//    the Q K^T MMAs of the even and the odd tiles of each pass and warp 2 every
+//    P V, so that the tensor pipe keeps working while an issuing thread waits
+//    on a barrier or commits; warps 4-19 form four softmax warpgroups.  In
+//    pass 1 the warpgroups form two teams that take alternate tiles (a team's
+//    two warpgroups own key columns 0-63 and 64-127); in pass 2 every
+//    warpgroup takes every tile, warpgroup w its key columns 32w .. 32w+31.
 //  * TMEM: pass 1 uses four fp32 S buffers; pass 2 three S buffers and the O
 //    accumulator.  In pass 2 the bf16 P of a tile is written over the S
 //    columns it came from (each warpgroup over its own), and the P V MMA reads
@@ -40,8 +41,10 @@
 //    column sum (over the warp's 32 rows) per lane and 32-column block, the
 //    last of the four warps of a warpgroup to finish a tile combines them
 //    through shared memory, and one red.global.add per column and query head
-//    goes to score_inc (zeroed by the host call).  Pass 1 keeps one row per
-//    thread (32x32b layout) for the row statistics.
+//    goes to score_inc (zeroed by the host call), or, with three or more row
+//    tiles per head, a store into the tile's row of column partials that a
+//    second kernel adds in row-tile order.  Pass 1 keeps one row per thread
+//    (32x32b layout) for the row statistics.
 //  * Key tiles are classified up front from slot_pos: tiles no row of the CTA
 //    can see are skipped, tiles every row sees need no mask, the rest are
 //    masked per element.
